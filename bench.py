@@ -1,0 +1,416 @@
+#!/usr/bin/env python3
+"""Benchmark of the turn-aware OPD loss step on GB300.
+
+A step is one pass of the whole hot path over one packed batch: blend weights
+(turnopd_weights), per-token reverse KL + student-logit gradient + weighted
+loss (turnopd_loss_fwd_bwd) and turn statistics (turnopd_turn_stats).
+
+Default workload: 8 trajectories x 4096 tokens, 10-30 turns, 40 % masked
+observation tokens, V = 151,936, bf16 logits (compact rows: one per supervised
+token), bf16 gradient, alpha = 0.5, full-vocabulary mode.  Inputs are seeded
+synthetic data already resident in HBM; each step streams ~17.9 GB, far more
+than the 129 MB L2, so no flush is needed between steps.
+
+Prints one JSON line (rank 0).  --impl reference times the fp64 CPU oracle on a
+bounded sample of the same workload instead.
+
+Under torchrun with N > 1 every rank runs its own batch (weak scaling); the
+ranks exchange the count vector before the weights and the loss after the step
+(NCCL all-reduce of 2*max_turns+2 numbers), the path's only cross-rank data.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "loss fwd+bwd tokens/s at V=151936 bf16 on 1 GB300; achieved HBM GB/s vs peak"
+UNIT = "tokens/s"
+KERNELS_PER_STEP = 9  # counts(2) + weights(1) + compaction(2) + row kernel + loss sum + stats(2)
+ROW_KERNEL_SOURCES = ["paper_2607_05804_gb300/csrc/rowkl_cluster.cu",
+                      "paper_2607_05804_gb300/csrc/loss_kernels.cu",
+                      "paper_2607_05804_gb300/csrc/common.cuh"]
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["native", "reference"], default="native")
+    p.add_argument("--workload", default="packed", choices=["packed", "household", "multihop"])
+    p.add_argument("--mode", default="full", choices=["full", "sampled"])
+    p.add_argument("--alpha", type=float, default=0.5)
+    p.add_argument("--no-e2e", action="store_true")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-sample-rows", type=int, default=0, help="0 = size to ~15 s of oracle work")
+    p.add_argument("--num-traj", type=int, default=0,
+                   help="packed workload only: trajectories (0 = 8); smaller cases serve profiling")
+    p.add_argument("--traj-len", type=int, default=0, help="packed workload only: tokens per trajectory")
+    return p.parse_args()
+
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def load_peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as fh:
+            d = json.load(fh)
+        return float(d["hbm_gbs"]), "measured"
+    except Exception:
+        return 6800.0, "fallback"
+
+
+def source_hash():
+    h = hashlib.sha256()
+    for rel in ROW_KERNEL_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def committed_traffic(workload):
+    """DRAM bytes per row-kernel launch from the committed ncu summary, if it was
+    taken on the current kernel source."""
+    path = os.path.join(ROOT, "profiles", "row_kernel_traffic.json")
+    try:
+        with open(path) as fh:
+            d = json.load(fh)
+        if d.get("source_hash") != source_hash():
+            return None
+        return d.get("bytes_per_launch", {}).get(workload)
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons while the timed region runs."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index, self.rows, self.proc = index, [], None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) >= 8:
+                self.rows.append(parts)
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.thread.join(timeout=2)
+        if not self.rows:
+            return None
+        sm = [float(r[0]) for r in self.rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[k] for r in self.rows for k in range(4) if r[4 + k] == "Active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(self.rows)}
+
+
+def build_inputs(args, rank, device):
+    import torch
+
+    import workloads as W
+    from paper_2607_05804_gb300 import TURNOPD_FULL_VOCAB, TURNOPD_SAMPLED_TOKEN
+    from paper_2607_05804_gb300.step import LossStep, to_device
+
+    if args.workload == "packed" and (args.num_traj or args.traj_len):
+        b = W.packed(seed=rank, num_traj=args.num_traj or 8, traj_len=args.traj_len or 4096)
+    else:
+        b = W.CONFIGS[args.workload](seed=rank)
+    V = W.V_QWEN
+    R = b.num_valid
+    zs, zt = W.make_logits(R, V, "agent", torch.bfloat16, seed=1000 + rank, device=device)
+    mode = TURNOPD_SAMPLED_TOKEN if args.mode == "sampled" else TURNOPD_FULL_VOCAB
+    y = None
+    if mode == TURNOPD_SAMPLED_TOKEN:
+        y_c = W.sample_ids(zs, seed=2000 + rank)  # per row; expand to per token
+        y = torch.zeros(b.num_tokens, dtype=torch.int32, device=device)
+        idx = torch.from_numpy(b.loss_mask.nonzero()[0]).to(device)
+        y[idx] = y_c
+    tid, msk, off, rot = to_device(b, device, compact=True)
+    step = LossStep(tid, msk, off, b.max_turns, V, row_of_token=rot, sampled_ids=y, mode=mode,
+                    alpha=args.alpha)
+    grad = torch.empty_like(zs)
+    return b, V, zs, zt, grad, step
+
+
+def run_step(step, zs, zt, grad, world, dist, ev_pair=None):
+    if world > 1:
+        counts = step.local_counts().clone()
+        dist.all_reduce(counts)
+        step.weights(counts)
+    else:
+        step.weights()
+    if ev_pair is not None:
+        ev_pair[0].record()
+    step.loss_fwd_bwd(zs, zt, grad)
+    if ev_pair is not None:
+        ev_pair[1].record()
+    step.turn_stats()
+    if world > 1:
+        dist.all_reduce(step.loss)
+
+
+def cpu_baseline(b, zs, zt, V, alpha, mode, rows_override=0, budget_s=15.0):
+    """Time the fp64 CPU oracle on a bounded sample of the same workload."""
+    import numpy as np
+
+    import oracle
+    import workloads as W
+
+    oracle.build()
+    R = zs.shape[0]
+    w = oracle.weights(b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns, alpha).astype(np.float32)
+    valid = np.nonzero(b.loss_mask)[0]
+
+    def run(n):
+        zsn, ztn = W.bf16_bits(zs[:n]), W.bf16_bits(zt[:n])
+        mask = np.ones(n, np.uint8)
+        t0 = time.perf_counter()
+        oracle.loss_fwd_bwd(zsn, ztn, V, mask, w[valid[:n]], mode=0)
+        return time.perf_counter() - t0
+
+    cores = oracle.num_threads()
+    if rows_override:
+        n = min(rows_override, R)
+    else:
+        probe = min(R, max(16, 2 * cores))
+        dt = run(probe)
+        n = int(min(R, 2048, max(probe, budget_s * probe / max(dt, 1e-6))))
+    dt = run(n)
+    return {"value": n / dt, "unit": UNIT, "cores": cores, "kind": "oracle",
+            "sample": f"first {n} supervised rows of the same batch (full-vocabulary loss + "
+                      f"gradient, fp64, {dt:.1f} s)"}
+
+
+def reference_arm(args, world, rank):
+    """--impl reference: the fp64 CPU oracle as the reference implementation."""
+    import numpy as np
+
+    import oracle
+    import workloads as W
+
+    if rank != 0:
+        return
+    import torch
+
+    b = W.CONFIGS[args.workload](seed=0)
+    V = W.V_QWEN
+    n = 32  # rows per reference step (bounded so the whole run ends within minutes)
+    zs, zt = W.make_logits(n, V, "agent", torch.bfloat16, seed=1000, device="cpu", chunk_rows=8)
+    zsb, ztb = W.bf16_bits(zs), W.bf16_bits(zt)
+    w = oracle.weights(b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns, args.alpha)
+    valid = np.nonzero(b.loss_mask)[0]
+    w32 = w.astype(np.float32)[valid[:n]]
+    mask = np.ones(n, np.uint8)
+    times = []
+    for k in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        oracle.weights(b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns, args.alpha)
+        _, tl, _ = oracle.loss_fwd_bwd(zsb, ztb, V, mask, w32, mode=0)
+        dt = time.perf_counter() - t0
+        if k >= args.warmup:
+            times.append(dt)
+    tot = sum(times)
+    value = n * len(times) / tot
+    cores = oracle.num_threads()
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": 1e3 * tot / len(times), "higher_is_better": True,
+           "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "impl": "reference",
+           "config": {"workload": f"{b.name}_V{V}", "sample_rows_per_step": n},
+           "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores, "kind": "oracle",
+                            "sample": f"{n} supervised rows per step of the {b.name} batch"},
+           "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    args = parse()
+    world, rank, local = dist_env()
+    if args.impl == "reference":
+        reference_arm(args, world, rank)
+        return
+    import torch
+
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    import paper_2607_05804_gb300 as P
+
+    P.load()
+    b, V, zs, zt, grad, step = build_inputs(args, rank, device)
+    R = b.num_valid
+    torch.cuda.synchronize()
+
+    for _ in range(max(args.warmup, 3)):
+        run_step(step, zs, zt, grad, world, dist)
+    torch.cuda.synchronize()
+    if step.status() != 0:
+        raise RuntimeError(f"device status {step.status()}")
+
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler.start()
+    t_start.record()
+    for k in range(args.steps):
+        run_step(step, zs, zt, grad, world, dist, evs[k])
+    t_end.record()
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    ms = t_start.elapsed_time(t_end)
+    loss_ms = [a.elapsed_time(z) for a, z in evs]
+    if world > 1:
+        t = torch.tensor([ms], device=device, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        tot_rows = torch.tensor([R], device=device, dtype=torch.int64)
+        dist.all_reduce(tot_rows)
+        tot_rows = int(tot_rows.item())
+    else:
+        tot_rows = R
+    if step.status() != 0:
+        raise RuntimeError(f"device status {step.status()}")
+
+    value = tot_rows * args.steps / (ms / 1e3)
+    peak, peak_kind = load_peaks()
+    bytes_per_row = 3 * V * 2  # two bf16 logit rows read + one bf16 gradient row written
+    alg_bytes = R * bytes_per_row
+    loss_avg_ms = statistics.mean(loss_ms)
+    achieved = alg_bytes / (loss_avg_ms / 1e3) / 1e9
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = e2e_leg(args, step, zs, zt, grad, world, dist, device, R)
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(b, zs, zt, V, args.alpha, 0, args.cpu_sample_rows)
+
+    if rank == 0:
+        out = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {
+                "workload": f"{b.name}_V{V}", "tokens": b.num_tokens, "supervised_tokens": R,
+                "tokens_counted": "supervised (assistant) tokens", "vocab": V,
+                "layout": "compact rows (one per supervised token)", "grad_dtype": "bf16",
+                "mode": args.mode, "alpha": args.alpha, "scope": "traj",
+                "l2": "inputs larger than L2 (%.1f GB streamed per step), no flush" % (alg_bytes / 1e9),
+                "packed_tokens_per_s": b.num_tokens * world * args.steps / (ms / 1e3),
+            },
+            "roofline": {
+                "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "peak_kind": peak_kind,
+                "kernel": "turnopd_loss_fwd_bwd launch sequence (row kernel + compaction + loss sum)",
+                "algorithmic_bytes_per_launch": alg_bytes,
+                "launch_ms": loss_avg_ms,
+                "traffic": committed_traffic(args.workload),
+            },
+            "gpu_launches": KERNELS_PER_STEP * args.steps,
+            "clocks": clocks,
+            "e2e": e2e,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def e2e_leg(args, step, zs, zt, grad, world, dist, device, R):
+    """Same metric through the public API with inputs in pinned host memory: each
+    step copies the logits and batch metadata host->device, runs the step and
+    reads the loss back."""
+    import torch
+
+    h_zs = torch.empty(zs.shape, dtype=zs.dtype, pin_memory=True)
+    h_zt = torch.empty(zt.shape, dtype=zt.dtype, pin_memory=True)
+    h_zs.copy_(zs)
+    h_zt.copy_(zt)
+    meta = [step.turn_id, step.loss_mask, step.traj_offsets, step.row_of_token]
+    h_meta = [m.cpu().pin_memory() for m in meta]
+    h_loss = torch.empty(1, dtype=torch.float64, pin_memory=True)
+    steps = max(3, min(args.steps, 10))
+    h2d = sum(t.numel() * t.element_size() for t in [h_zs, h_zt] + h_meta)
+
+    def one():
+        zs.copy_(h_zs, non_blocking=True)
+        zt.copy_(h_zt, non_blocking=True)
+        for d, h in zip(meta, h_meta):
+            d.copy_(h, non_blocking=True)
+        run_step(step, zs, zt, grad, world, dist)
+        h_loss.copy_(step.loss, non_blocking=True)
+
+    for _ in range(2):
+        one()
+    torch.cuda.synchronize()
+    a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    if world > 1:
+        dist.barrier()
+    a.record()
+    for _ in range(steps):
+        one()
+    z.record()
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(z)
+    if world > 1:
+        t = torch.tensor([ms], device=device, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    return {"value": R * world * steps / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
+            "d2h_bytes_per_step": 8, "steps": steps}
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,221 @@
+/*
+ * turnopd.h -- C ABI of libturnopd: the turn-aware on-policy-distillation
+ * (OPD) loss of TurnOPD (arXiv 2607.05804) on NVIDIA GB300 (sm_103a).
+ *
+ * One training step of the method, for a packed batch of multi-turn student
+ * trajectories, is:
+ *   1. turnopd_turn_counts / turnopd_weights -- supervised-token counts per
+ *      (trajectory, turn) and the progressive blend weights
+ *      w_blend = (1 - alpha) w_traj + alpha w_turn            (Sec. 5.2, Algorithm 1)
+ *   2. turnopd_loss_fwd_bwd -- per-token reverse KL(pi_s || pi_T) over the full
+ *      vocabulary (Eq. opd-rkl) or the sampled-token estimator, its gradient
+ *      w.r.t. the student logits, and L = sum_i w_i l_i   (Algorithm 1, L_k)
+ *   3. turnopd_turn_stats -- per-(trajectory, turn) and per-turn-index KL sums
+ *      and counts (Eq. observed-turn-kl; the kl_per_turn / num_traj statistics
+ *      that the rollout-depth controller of Sec. 5.1 reads).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ * - Memory: every array argument is DEVICE memory owned by the caller.  The
+ *   library allocates nothing; scratch space is the caller's `workspace`
+ *   (size from the matching *_workspace_bytes function, 256-byte aligned).
+ * - Execution: calls are asynchronous and stream-ordered on `stream` (a
+ *   cudaStream_t; NULL = legacy default stream).  Calls on different streams
+ *   may run concurrently if they share no output or workspace.
+ * - Host-detected errors (null pointers, bad sizes, unsupported combinations,
+ *   small workspace) return immediately, before any launch or CUDA call.
+ * - Device-detected errors (values inside device arrays) are reported through
+ *   `dev_status`, a caller-zeroed int32 in device memory: the first error
+ *   code stored wins (atomic compare-and-swap from 0), later ones are dropped.
+ *   The offending token or trajectory is skipped; other outputs are still
+ *   written.  Read the word after synchronising the stream.
+ * - Results are deterministic: the same inputs give bit-identical outputs on
+ *   every run (fixed-order reductions, no floating-point atomics).
+ * - Packed batch: trajectory b owns tokens [traj_offsets[b], traj_offsets[b+1]);
+ *   traj_offsets[0] = 0, non-decreasing, traj_offsets[num_traj] = num_tokens.
+ *   loss_mask[i] = 1 marks a supervised (assistant) token, 0 an observation
+ *   token; turn_id[i] is the 0-based turn of token i, read only where
+ *   loss_mask[i] = 1 and required to lie in [0, max_turns) there.
+ * - max_turns must lie in [1, TURNOPD_MAX_TURNS]; vocab in [1, 2^31 - 1].
+ */
+#ifndef TURNOPD_H
+#define TURNOPD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same object as cudaStream_t (a CUstream_st pointer), declared here so the
+ * header needs no CUDA include. */
+typedef struct CUstream_st *turnopd_stream_t;
+
+typedef enum {
+    TURNOPD_OK = 0,
+    TURNOPD_ERR_NULL = 1,        /* a required pointer is NULL                       */
+    TURNOPD_ERR_SHAPE = 2,       /* a size or stride is out of range                 */
+    TURNOPD_ERR_OFFSETS = 3,     /* traj_offsets not 0..num_tokens non-decreasing     */
+    TURNOPD_ERR_TURN_RANGE = 4,  /* supervised token with turn_id outside [0,max)     */
+    TURNOPD_ERR_TOKEN_RANGE = 5, /* row index or sampled id out of range              */
+    TURNOPD_ERR_UNSUPPORTED = 6, /* unsupported dtype / mode / flag combination       */
+    TURNOPD_ERR_CUDA = 7,        /* a CUDA runtime call or launch failed              */
+    TURNOPD_ERR_TIMEOUT = 8,     /* a bounded device-side wait gave up                */
+    TURNOPD_ERR_NONFINITE = 9,   /* a non-finite log-sum-exp or loss value           */
+    TURNOPD_ERR_WORKSPACE = 10   /* workspace NULL, misaligned or too small           */
+} turnopd_status;
+
+enum { TURNOPD_FULL_VOCAB = 0, TURNOPD_SAMPLED_TOKEN = 1 };       /* loss mode     */
+enum { TURNOPD_F32 = 0, TURNOPD_BF16 = 1 };                       /* element type  */
+enum { TURNOPD_SCOPE_TRAJ = 0, TURNOPD_SCOPE_BATCH = 1 };         /* normalisation */
+
+/* Write zeros into the gradient rows of masked tokens that own a row. */
+#define TURNOPD_ZERO_MASKED_GRAD 0x1u
+/* Diagnostic: force the portable one-CTA-per-row kernel instead of the
+ * cluster-resident kernel (results agree within the documented tolerance). */
+#define TURNOPD_FORCE_PORTABLE 0x100u
+
+#define TURNOPD_MAX_TURNS 4096
+
+/*
+ * turnopd_turn_counts -- supervised-token bookkeeping of the multi-turn trace
+ * model (Sec. 3; survivors "trajectories that reach each turn", Sec. 4.1;
+ * n_t of Sec. 5.1 and Sec. 5.2).
+ *
+ * Outputs (device, caller-owned):
+ *   traj_turn_cnt  int32[num_traj * max_turns], row-major [b][t]:
+ *                  n_bt = #{i in b : loss_mask[i] = 1, turn_id[i] = t}
+ *   counts         int64[2 * max_turns + 1]:
+ *                  [0, max_turns)            S_t = #{b : n_bt > 0}
+ *                  [max_turns, 2 max_turns)  C_t = sum_b n_bt
+ *                  [2 max_turns]             B'  = #{b : sum_t n_bt > 0}
+ *                  Summing `counts` over data-parallel ranks (each holding
+ *                  whole trajectories) gives the batch-wide vector that
+ *                  turnopd_weights accepts as `global_counts`.
+ * Device errors: TURNOPD_ERR_OFFSETS, TURNOPD_ERR_TURN_RANGE (token ignored).
+ */
+turnopd_status turnopd_turn_counts(const int32_t *turn_id, const uint8_t *loss_mask,
+                                   const int64_t *traj_offsets, int32_t num_traj,
+                                   int64_t num_tokens, int32_t max_turns,
+                                   int32_t *traj_turn_cnt, int64_t *counts,
+                                   int32_t *dev_status, turnopd_stream_t stream);
+
+/*
+ * turnopd_weights -- per-token progressive blend weights (Sec. 5.2: q^traj =
+ * n_t / sum_j n_j, q^turn = 1/T, q^blend = (1 - alpha) q^traj + alpha q^turn;
+ * Algorithm 1: w_blend = (1 - alpha) w_traj + alpha w_turn on observed tokens).
+ *
+ * scope = TURNOPD_SCOPE_TRAJ (the paper's Eq. opd-rkl normalisation, a token
+ * mean inside each trajectory, then a mean over the B' trajectories that hold
+ * supervised tokens -- "seq-mean-token-mean"):
+ *     w_i = [(1 - alpha) / N_b + alpha / (T_b n_bt)] / B'
+ *   N_b = supervised tokens of b, T_b = non-empty turns of b.
+ * scope = TURNOPD_SCOPE_BATCH (one token mean over the batch):
+ *     w_i = (1 - alpha) / N + alpha / (S n_bt),  N = sum C_t, S = sum S_t.
+ * n_min > 0 enables the turn-reliability floor (hyper-parameter table:
+ * n_min = max(floor, ceil(frac * n_traj)), computed by the caller): turn index
+ * t is reliable iff S_t >= n_min; tokens of unreliable turns keep the token
+ * weight (1/N_b, resp. 1/N), the reliable non-empty turns share the remaining
+ * mass equally; with no reliable turn w_turn = w_traj.  n_min <= 0: no floor.
+ * global_counts: NULL, or a device int64[2 max_turns + 1] vector laid out as
+ *   turnopd_turn_counts' `counts`, summed over data-parallel ranks; it then
+ *   replaces the local S_t, C_t and B' (n_bt, N_b, T_b stay local).
+ * alpha must lie in [0, 1] (see turnopd_alpha_schedule).
+ * Output: w_out float32[num_tokens] (computed in fp64, rounded to nearest);
+ *   0 for masked tokens and for tokens of trajectories without supervision.
+ * Workspace: turnopd_weights_workspace_bytes(num_traj, max_turns) bytes.
+ * Device errors: as turnopd_turn_counts.
+ */
+turnopd_status turnopd_weights(const int32_t *turn_id, const uint8_t *loss_mask,
+                               const int64_t *traj_offsets, int32_t num_traj,
+                               int64_t num_tokens, int32_t max_turns, double alpha,
+                               int32_t scope, int32_t n_min, const int64_t *global_counts,
+                               float *w_out, void *workspace, size_t workspace_bytes,
+                               int32_t *dev_status, turnopd_stream_t stream);
+
+size_t turnopd_weights_workspace_bytes(int32_t num_traj, int32_t max_turns);
+
+/*
+ * turnopd_loss_fwd_bwd -- per-token OPD loss, its student-logit gradient and
+ * the weighted batch loss (Eq. opd-rkl; Algorithm 1: L_k = sum_i w_i l_i).
+ *
+ * For every supervised token i with logit row r = row_of_token[i] (or r = i
+ * when row_of_token is NULL), with ls = z_s - LSE(z_s), lt = z_t - LSE(z_t),
+ * p = exp(ls) (natural log throughout, softmax of the raw logits):
+ *   mode TURNOPD_FULL_VOCAB:    l_i = KL(p_s || p_t) = sum_v p_v (ls_v - lt_v)
+ *                               g_v = w_i p_v (ls_v - lt_v - l_i)
+ *   mode TURNOPD_SAMPLED_TOKEN: l_i = ls_y - lt_y,  y = sampled_ids[i]
+ *                               g_v = w_i l_i (delta_{v,y} - p_v)
+ *     (score-function gradient: its expectation over y ~ p_s is the
+ *      full-vocabulary gradient; l_i itself is treated as a constant).
+ * Inputs:
+ *   z_student, z_teacher  [num_rows, ld] row-major, in_dtype (F32 or BF16);
+ *                          columns [vocab, ld) are never read.
+ *   row_of_token           int32[num_tokens] or NULL (then num_rows >= num_tokens);
+ *                          read only where loss_mask = 1, must lie in [0, num_rows).
+ *   sampled_ids            int32[num_tokens], required for SAMPLED_TOKEN, in [0, vocab).
+ *   loss_mask              uint8[num_tokens];  w  float32[num_tokens] (turnopd_weights).
+ * Outputs:
+ *   grad_student  [num_rows, ld] in grad_dtype (F32 or BF16), or NULL for a
+ *                 forward-only call.  Rows of supervised tokens get g (bf16:
+ *                 round to nearest even from fp32); columns [vocab, ld) and
+ *                 other rows are not written unless TURNOPD_ZERO_MASKED_GRAD,
+ *                 which zero-fills columns [0, vocab) of masked tokens' rows.
+ *                 grad_student may not alias the logits.
+ *   token_loss_out float32[num_tokens]: l_i, 0 for masked tokens.
+ *   loss_out       one double: sum_i w_i l_i (fixed-order fp64 sum).
+ * Workspace: turnopd_loss_workspace_bytes(num_tokens) bytes.
+ * Device errors: TURNOPD_ERR_TOKEN_RANGE (row or sampled id; token skipped,
+ *   l_i = 0), TURNOPD_ERR_NONFINITE (non-finite LSE or l_i).
+ * Precision: fp32 arithmetic on exact fp32/bf16 inputs, fp64 loss sum.
+ */
+turnopd_status turnopd_loss_fwd_bwd(const void *z_student, const void *z_teacher,
+                                    int32_t in_dtype, int64_t ld, int64_t vocab,
+                                    int64_t num_rows, const int32_t *row_of_token,
+                                    const int32_t *sampled_ids, const uint8_t *loss_mask,
+                                    const float *w, int64_t num_tokens, int32_t mode,
+                                    void *grad_student, int32_t grad_dtype, uint32_t flags,
+                                    float *token_loss_out, double *loss_out,
+                                    void *workspace, size_t workspace_bytes,
+                                    int32_t *dev_status, turnopd_stream_t stream);
+
+size_t turnopd_loss_workspace_bytes(int64_t num_tokens);
+
+/*
+ * turnopd_turn_stats -- turn statistics of the per-token losses
+ * (Eq. observed-turn-kl: K_t is the mean per-token reverse KL over the
+ * supervised tokens at turn t, over trajectories that reach t; the survivor
+ * count n_t of Sec. 5.1; the kl_per_turn / num_traj statistics of the
+ * hyper-parameter table).  Sums and counts are returned rather than means so
+ * that ranks can add them; K_t = turn_sum[t] / turn_cnt[t].
+ * Outputs (device, caller-owned):
+ *   traj_turn_sum double[num_traj * max_turns]  sum of token_loss over (b, t)
+ *   traj_turn_cnt int32 [num_traj * max_turns]  n_bt
+ *   turn_sum      double[max_turns]             sum over b of traj_turn_sum
+ *   turn_cnt      int64 [max_turns]             sum over b of n_bt
+ *   turn_surv     int32 [max_turns]             #{b : n_bt > 0}
+ * Device errors: TURNOPD_ERR_OFFSETS, TURNOPD_ERR_TURN_RANGE (token ignored).
+ */
+turnopd_status turnopd_turn_stats(const float *token_loss, const int32_t *turn_id,
+                                  const uint8_t *loss_mask, const int64_t *traj_offsets,
+                                  int32_t num_traj, int64_t num_tokens, int32_t max_turns,
+                                  double *traj_turn_sum, int32_t *traj_turn_cnt,
+                                  double *turn_sum, int64_t *turn_cnt, int32_t *turn_surv,
+                                  int32_t *dev_status, turnopd_stream_t stream);
+
+/*
+ * turnopd_alpha_schedule -- blend coefficient alpha_k = clip((k/K - s)/(e - s), 0, 1)
+ * from training progress k/K (Sec. 5.2; Algorithm 1; s, e = 0, 1 in the
+ * paper's runs).  Host function.  Returns NaN if K <= 0 or e <= s.
+ */
+double turnopd_alpha_schedule(int64_t k, int64_t K, double s, double e);
+
+/* Human-readable name of a status code (static string, never NULL). */
+const char *turnopd_status_string(turnopd_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TURNOPD_H */

@@ -1,0 +1,245 @@
+"""Python binding of libturnopd, the GB300 (sm_103a) turn-aware OPD loss.
+
+Argument marshalling only: every function forwards torch tensors' device
+pointers, sizes and the current CUDA stream to the C entry point of the same
+name (``include/turnopd.h``), and raises ``TurnopdError`` on a non-OK status.
+All compute runs in the library's CUDA kernels; there is no other path.  If
+the library has not been built, importing works but the first call raises.
+
+Build it with ``python -c "import __graft_entry__ as g; g.build()"`` (or
+``python paper_2607_05804_gb300/build.py``).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+__all__ = [
+    "TurnopdError", "library_path", "load",
+    "TURNOPD_FULL_VOCAB", "TURNOPD_SAMPLED_TOKEN", "TURNOPD_F32", "TURNOPD_BF16",
+    "TURNOPD_SCOPE_TRAJ", "TURNOPD_SCOPE_BATCH", "TURNOPD_ZERO_MASKED_GRAD",
+    "TURNOPD_FORCE_PORTABLE", "TURNOPD_MAX_TURNS",
+    "turnopd_turn_counts", "turnopd_weights", "turnopd_weights_workspace_bytes",
+    "turnopd_loss_fwd_bwd", "turnopd_loss_workspace_bytes", "turnopd_turn_stats",
+    "turnopd_alpha_schedule", "turnopd_status_string",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB_PATH = os.path.join(_HERE, "libturnopd.so")
+
+TURNOPD_FULL_VOCAB, TURNOPD_SAMPLED_TOKEN = 0, 1
+TURNOPD_F32, TURNOPD_BF16 = 0, 1
+TURNOPD_SCOPE_TRAJ, TURNOPD_SCOPE_BATCH = 0, 1
+TURNOPD_ZERO_MASKED_GRAD = 0x1
+TURNOPD_FORCE_PORTABLE = 0x100
+TURNOPD_MAX_TURNS = 4096
+
+STATUS_NAMES = {
+    0: "TURNOPD_OK", 1: "TURNOPD_ERR_NULL", 2: "TURNOPD_ERR_SHAPE", 3: "TURNOPD_ERR_OFFSETS",
+    4: "TURNOPD_ERR_TURN_RANGE", 5: "TURNOPD_ERR_TOKEN_RANGE", 6: "TURNOPD_ERR_UNSUPPORTED",
+    7: "TURNOPD_ERR_CUDA", 8: "TURNOPD_ERR_TIMEOUT", 9: "TURNOPD_ERR_NONFINITE",
+    10: "TURNOPD_ERR_WORKSPACE",
+}
+
+
+class TurnopdError(RuntimeError):
+    def __init__(self, code: int, where: str):
+        self.code = int(code)
+        super().__init__(f"{where}: {STATUS_NAMES.get(self.code, self.code)} "
+                         f"({turnopd_status_string(self.code)})")
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+_lib = None
+
+
+def load():
+    """Load libturnopd.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_LIB_PATH):
+        raise RuntimeError(f"libturnopd.so not found at {_LIB_PATH}: the CUDA library has not "
+                           "been built (run __graft_entry__.build())")
+    lib = ctypes.CDLL(_LIB_PATH)
+    P, i32, i64, u32 = ctypes.c_void_p, ctypes.c_int32, ctypes.c_int64, ctypes.c_uint32
+    f64, sz = ctypes.c_double, ctypes.c_size_t
+    sig = {
+        "turnopd_turn_counts": [P, P, P, i32, i64, i32, P, P, P, P],
+        "turnopd_weights": [P, P, P, i32, i64, i32, f64, i32, i32, P, P, P, sz, P, P],
+        "turnopd_loss_fwd_bwd": [P, P, i32, i64, i64, i64, P, P, P, P, i64, i32, P, i32, u32,
+                                 P, P, P, sz, P, P],
+        "turnopd_turn_stats": [P, P, P, P, i32, i64, i32, P, P, P, P, P, P, P],
+    }
+    for name, args in sig.items():
+        fn = getattr(lib, name)
+        fn.argtypes = args
+        fn.restype = ctypes.c_int
+    lib.turnopd_weights_workspace_bytes.argtypes = [i32, i32]
+    lib.turnopd_weights_workspace_bytes.restype = sz
+    lib.turnopd_loss_workspace_bytes.argtypes = [i64]
+    lib.turnopd_loss_workspace_bytes.restype = sz
+    lib.turnopd_alpha_schedule.argtypes = [i64, i64, f64, f64]
+    lib.turnopd_alpha_schedule.restype = f64
+    lib.turnopd_status_string.argtypes = [ctypes.c_int]
+    lib.turnopd_status_string.restype = ctypes.c_char_p
+    _lib = lib
+    return lib
+
+
+# ---------------------------------------------------------------- marshalling helpers
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    import torch
+
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _need(t, name, dtype=None, numel=None):
+    import torch
+
+    if t is None:
+        return
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise ValueError(f"{name} must have dtype {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if numel is not None and t.numel() < numel:
+        raise ValueError(f"{name} needs at least {numel} elements, has {t.numel()}")
+
+
+def _dtype_code(t, name):
+    import torch
+
+    if t.dtype == torch.bfloat16:
+        return TURNOPD_BF16
+    if t.dtype == torch.float32:
+        return TURNOPD_F32
+    raise ValueError(f"{name} must be float32 or bfloat16")
+
+
+def _check(code, where):
+    if code != 0:
+        raise TurnopdError(code, where)
+
+
+# ---------------------------------------------------------------- entry points
+
+def turnopd_status_string(code: int) -> str:
+    return load().turnopd_status_string(int(code)).decode()
+
+
+def turnopd_alpha_schedule(k: int, K: int, s: float = 0.0, e: float = 1.0) -> float:
+    return float(load().turnopd_alpha_schedule(int(k), int(K), float(s), float(e)))
+
+
+def turnopd_weights_workspace_bytes(num_traj: int, max_turns: int) -> int:
+    return int(load().turnopd_weights_workspace_bytes(int(num_traj), int(max_turns)))
+
+
+def turnopd_loss_workspace_bytes(num_tokens: int) -> int:
+    return int(load().turnopd_loss_workspace_bytes(int(num_tokens)))
+
+
+def turnopd_turn_counts(turn_id, loss_mask, traj_offsets, max_turns, traj_turn_cnt, counts,
+                        dev_status, stream=None):
+    import torch
+
+    T, B = turn_id.numel(), traj_offsets.numel() - 1
+    _need(turn_id, "turn_id", torch.int32)
+    _need(loss_mask, "loss_mask", torch.uint8, T)
+    _need(traj_offsets, "traj_offsets", torch.int64)
+    _need(traj_turn_cnt, "traj_turn_cnt", torch.int32, B * max_turns)
+    _need(counts, "counts", torch.int64, 2 * max_turns + 1)
+    _need(dev_status, "dev_status", torch.int32, 1)
+    _check(load().turnopd_turn_counts(_ptr(turn_id), _ptr(loss_mask), _ptr(traj_offsets), B, T,
+                                      int(max_turns), _ptr(traj_turn_cnt), _ptr(counts),
+                                      _ptr(dev_status), _stream(stream)), "turnopd_turn_counts")
+
+
+def turnopd_weights(turn_id, loss_mask, traj_offsets, max_turns, alpha, scope, n_min,
+                    global_counts, w_out, workspace, dev_status, stream=None):
+    import torch
+
+    T, B = turn_id.numel(), traj_offsets.numel() - 1
+    _need(turn_id, "turn_id", torch.int32)
+    _need(loss_mask, "loss_mask", torch.uint8, T)
+    _need(traj_offsets, "traj_offsets", torch.int64)
+    _need(global_counts, "global_counts", torch.int64, 2 * max_turns + 1)
+    _need(w_out, "w_out", torch.float32, T)
+    _need(workspace, "workspace")
+    _need(dev_status, "dev_status", torch.int32, 1)
+    _check(load().turnopd_weights(_ptr(turn_id), _ptr(loss_mask), _ptr(traj_offsets), B, T,
+                                  int(max_turns), float(alpha), int(scope), int(n_min),
+                                  _ptr(global_counts), _ptr(w_out), _ptr(workspace),
+                                  workspace.numel() * workspace.element_size(),
+                                  _ptr(dev_status), _stream(stream)), "turnopd_weights")
+
+
+def turnopd_loss_fwd_bwd(z_student, z_teacher, vocab, row_of_token, sampled_ids, loss_mask, w,
+                         mode, grad_student, flags, token_loss_out, loss_out, workspace,
+                         dev_status, stream=None):
+    """z_student, z_teacher: [num_rows, ld] tensors (row stride ld, unit column stride);
+    grad_student: None or a tensor of the same shape and strides."""
+    import torch
+
+    T = loss_mask.numel()
+    for name, z in (("z_student", z_student), ("z_teacher", z_teacher)):
+        if not z.is_cuda or z.dim() != 2 or z.stride(1) != 1:
+            raise ValueError(f"{name} must be a 2-D CUDA tensor with unit column stride")
+    if z_teacher.shape != z_student.shape or z_teacher.stride() != z_student.stride() \
+            or z_teacher.dtype != z_student.dtype:
+        raise ValueError("z_teacher must match z_student in shape, stride and dtype")
+    ld = z_student.stride(0)
+    if grad_student is not None and (grad_student.shape != z_student.shape
+                                     or grad_student.stride(0) != ld or grad_student.stride(1) != 1
+                                     or not grad_student.is_cuda):
+        raise ValueError("grad_student must match z_student in shape and row stride")
+    _need(row_of_token, "row_of_token", torch.int32, T)
+    _need(sampled_ids, "sampled_ids", torch.int32, T)
+    _need(loss_mask, "loss_mask", torch.uint8)
+    _need(w, "w", torch.float32, T)
+    _need(token_loss_out, "token_loss_out", torch.float32, T)
+    _need(loss_out, "loss_out", torch.float64, 1)
+    _need(workspace, "workspace")
+    _need(dev_status, "dev_status", torch.int32, 1)
+    gdt = _dtype_code(grad_student, "grad_student") if grad_student is not None else TURNOPD_F32
+    _check(load().turnopd_loss_fwd_bwd(
+        _ptr(z_student), _ptr(z_teacher), _dtype_code(z_student, "z_student"), ld, int(vocab),
+        z_student.shape[0], _ptr(row_of_token), _ptr(sampled_ids), _ptr(loss_mask), _ptr(w), T,
+        int(mode), _ptr(grad_student), gdt, int(flags), _ptr(token_loss_out), _ptr(loss_out),
+        _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(dev_status),
+        _stream(stream)), "turnopd_loss_fwd_bwd")
+
+
+def turnopd_turn_stats(token_loss, turn_id, loss_mask, traj_offsets, max_turns, traj_turn_sum,
+                       traj_turn_cnt, turn_sum, turn_cnt, turn_surv, dev_status, stream=None):
+    import torch
+
+    T, B = turn_id.numel(), traj_offsets.numel() - 1
+    _need(token_loss, "token_loss", torch.float32, T)
+    _need(turn_id, "turn_id", torch.int32)
+    _need(loss_mask, "loss_mask", torch.uint8, T)
+    _need(traj_offsets, "traj_offsets", torch.int64)
+    _need(traj_turn_sum, "traj_turn_sum", torch.float64, B * max_turns)
+    _need(traj_turn_cnt, "traj_turn_cnt", torch.int32, B * max_turns)
+    _need(turn_sum, "turn_sum", torch.float64, max_turns)
+    _need(turn_cnt, "turn_cnt", torch.int64, max_turns)
+    _need(turn_surv, "turn_surv", torch.int32, max_turns)
+    _need(dev_status, "dev_status", torch.int32, 1)
+    _check(load().turnopd_turn_stats(_ptr(token_loss), _ptr(turn_id), _ptr(loss_mask),
+                                     _ptr(traj_offsets), B, T, int(max_turns), _ptr(traj_turn_sum),
+                                     _ptr(traj_turn_cnt), _ptr(turn_sum), _ptr(turn_cnt),
+                                     _ptr(turn_surv), _ptr(dev_status), _stream(stream)),
+           "turnopd_turn_stats")

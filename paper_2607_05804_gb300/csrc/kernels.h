@@ -1,0 +1,88 @@
+// Internal launcher declarations of libturnopd (not part of the public ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace turnopd {
+
+cudaError_t launch_turn_counts(const int32_t *turn_id, const uint8_t *mask, const int64_t *off,
+                               int32_t B, int64_t T, int32_t Tmax, int32_t *n_bt,
+                               int64_t *counts, int32_t *status, cudaStream_t stream);
+
+cudaError_t launch_weights(const int32_t *turn_id, const uint8_t *mask, const int64_t *off,
+                           int32_t B, int64_t T, int32_t Tmax, double alpha, int32_t scope,
+                           int32_t n_min, const int32_t *n_bt, const int64_t *counts,
+                           float *w_out, int32_t *status, cudaStream_t stream);
+
+int turn_stats_warps(int32_t Tmax);
+
+cudaError_t launch_turn_stats(const float *token_loss, const int32_t *turn_id,
+                              const uint8_t *mask, const int64_t *off, int32_t B, int64_t T,
+                              int32_t Tmax, double *traj_turn_sum, int32_t *traj_turn_cnt,
+                              double *turn_sum, int64_t *turn_cnt, int32_t *turn_surv,
+                              int32_t *status, cudaStream_t stream);
+
+// Loss path.  `ws` points at a workspace laid out by loss_workspace_layout().
+struct LossWorkspace {
+    int4 *rows;           // [T]  per supervised, in-range token in token order:
+                          //      {token i, row r, sampled id y (or -1), bits of w_i}
+    int32_t *blk_count;   // [nblk] per-block valid counts (compaction)
+    int32_t *nvalid;      // [1]
+    double *row_wl;       // [T]  w_i * l_i per compacted row
+};
+
+constexpr int kCompactBlock = 4096;  // tokens per compaction block
+
+size_t loss_workspace_bytes(int64_t T);
+LossWorkspace loss_workspace_layout(void *ws, int64_t T);
+
+struct LossArgs {
+    const void *zs;
+    const void *zt;
+    int32_t in_dtype;
+    int64_t ld;
+    int64_t vocab;
+    int64_t num_rows;
+    const int32_t *row_of_token;
+    const int32_t *sampled_ids;
+    const uint8_t *mask;
+    const float *w;
+    int64_t T;
+    int32_t mode;
+    void *grad;
+    int32_t grad_dtype;
+    uint32_t flags;
+    float *token_loss;
+    double *loss;
+    int32_t *status;
+};
+
+cudaError_t launch_loss(const LossArgs &a, const LossWorkspace &ws, cudaStream_t stream);
+
+// Row-kernel parameters (compacted supervised rows).
+struct RowIn {
+    const void *zs;
+    const void *zt;
+    int64_t ld;
+    int64_t vocab;
+    const int32_t *row_of_token;
+    const int32_t *sampled_ids;
+    const float *w;
+    int32_t mode;
+    void *grad;
+    float *token_loss;
+    double *row_wl;
+    const int4 *rows;
+    const int32_t *nvalid;
+    int32_t *status;
+};
+
+int device_sm_count();
+
+// Cluster-resident kernel for aligned bf16 rows; sets *used = false (and
+// launches nothing) when the shape does not fit it.
+cudaError_t launch_row_cluster(const RowIn &p, bool fp32_grad, cudaStream_t stream, bool *used);
+
+}  // namespace turnopd

@@ -1,0 +1,457 @@
+// Per-token OPD loss and student-logit gradient: compaction of supervised
+// tokens, the portable one-CTA-per-row kernel, masked-row zero fill and the
+// fixed-order loss sum (sm_103a).  The cluster-resident row kernel used for
+// aligned bf16 rows lives in rowkl_cluster.cu.
+//
+// Per supervised token (Eq. opd-rkl), from one read of each logit row:
+//   m, S = sum exp(z - m) for both models by an online (rescaling) pass,
+//   A = sum exp(z_s - m_s) (z_s - z_t)  ->  KL = A/S_s - (LSE_s - LSE_t),
+// then the gradient pass g_v = w p_v ((z_s - z_t)_v - (LSE_s - LSE_t) - KL)
+// (full vocabulary) or g_v = w l (delta_vy - p_v) (sampled token).
+
+#include <algorithm>
+
+#include "common.cuh"
+#include "kernels.h"
+
+namespace turnopd {
+
+size_t loss_workspace_bytes(int64_t T)
+{
+    const int64_t nblk = (T + kCompactBlock - 1) / kCompactBlock;
+    return align256(sizeof(int4) * (size_t)T) + align256(sizeof(int32_t) * (size_t)(nblk + 1)) +
+           align256(sizeof(int32_t)) + align256(sizeof(double) * (size_t)T) + 256;
+}
+
+LossWorkspace loss_workspace_layout(void *ws, int64_t T)
+{
+    const int64_t nblk = (T + kCompactBlock - 1) / kCompactBlock;
+    char *p = static_cast<char *>(ws);
+    LossWorkspace l;
+    l.rows = reinterpret_cast<int4 *>(p);
+    p += align256(sizeof(int4) * (size_t)T);
+    l.blk_count = reinterpret_cast<int32_t *>(p);
+    p += align256(sizeof(int32_t) * (size_t)(nblk + 1));
+    l.nvalid = reinterpret_cast<int32_t *>(p);
+    p += align256(sizeof(int32_t));
+    l.row_wl = reinterpret_cast<double *>(p);
+    return l;
+}
+
+// ---------------------------------------------------------------- compaction
+
+struct CompactIn {
+    const uint8_t *mask;
+    const int32_t *row_of_token;
+    const int32_t *sampled_ids;
+    const float *w;
+    int64_t num_rows;
+    int64_t vocab;
+    int64_t T;
+    int32_t mode;
+    float *token_loss;
+    int32_t *status;
+};
+
+// Token i enters the row list iff it is supervised and its row (and sampled
+// id) are in range; otherwise its loss is 0 (and a range error is recorded).
+__device__ __forceinline__ bool token_valid(const CompactIn &c, int64_t i, bool record)
+{
+    if (!c.mask[i])
+        return false;
+    const int64_t r = c.row_of_token ? (int64_t)c.row_of_token[i] : i;
+    bool ok = r >= 0 && r < c.num_rows;
+    if (ok && c.mode == TURNOPD_SAMPLED_TOKEN) {
+        const int32_t y = c.sampled_ids[i];
+        ok = y >= 0 && y < c.vocab;
+    }
+    if (!ok && record)
+        set_status(c.status, TURNOPD_ERR_TOKEN_RANGE);
+    return ok;
+}
+
+constexpr int kCompactThreads = 256;
+constexpr int kPerThread = kCompactBlock / kCompactThreads;  // 16 contiguous tokens
+
+__global__ void k_compact_count(CompactIn c, int32_t *__restrict__ blk_count)
+{
+    __shared__ int warp_tot[kCompactThreads / 32];
+    const int64_t i0 = (int64_t)blockIdx.x * kCompactBlock + (int64_t)threadIdx.x * kPerThread;
+    int n = 0;
+    for (int k = 0; k < kPerThread; ++k) {
+        const int64_t i = i0 + k;
+        if (i >= c.T)
+            break;
+        if (token_valid(c, i, true))
+            ++n;
+        else
+            c.token_loss[i] = 0.f;
+    }
+    n = warp_sum_i32(n);
+    if ((threadIdx.x & 31) == 0)
+        warp_tot[threadIdx.x >> 5] = n;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int tot = 0;
+        for (int wi = 0; wi < kCompactThreads / 32; ++wi)
+            tot += warp_tot[wi];
+        blk_count[blockIdx.x] = tot;
+    }
+}
+
+__global__ void k_compact_scatter(CompactIn c, const int32_t *__restrict__ blk_count,
+                                  int4 *__restrict__ rows, int32_t *__restrict__ nvalid)
+{
+    __shared__ int warp_tot[kCompactThreads / 32];
+    __shared__ int warp_off[kCompactThreads / 32];
+    __shared__ int64_t base_s;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    // exclusive prefix over the preceding blocks
+    int64_t pre = 0;
+    for (int k = threadIdx.x; k < (int)blockIdx.x; k += kCompactThreads)
+        pre += blk_count[k];
+    pre = warp_sum_i64(pre);
+    if (lane == 0)
+        warp_tot[warp] = (int)pre;  // fits: a prefix never exceeds T < 2^31
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int64_t s = 0;
+        for (int wi = 0; wi < kCompactThreads / 32; ++wi)
+            s += warp_tot[wi];
+        base_s = s;
+    }
+    __syncthreads();
+    const int64_t base = base_s;
+
+    const int64_t i0 = (int64_t)blockIdx.x * kCompactBlock + (int64_t)threadIdx.x * kPerThread;
+    uint32_t bits = 0;
+    for (int k = 0; k < kPerThread; ++k) {
+        const int64_t i = i0 + k;
+        if (i < c.T && token_valid(c, i, false))
+            bits |= 1u << k;
+    }
+    const int n = __popc(bits);
+    // exclusive scan of n across the block (thread order = token order)
+    int incl = n;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o)
+            incl += y;
+    }
+    __syncthreads();  // warp_tot reuse
+    if (lane == 31)
+        warp_tot[warp] = incl;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        int s = 0;
+        for (int wi = 0; wi < kCompactThreads / 32; ++wi) {
+            warp_off[wi] = s;
+            s += warp_tot[wi];
+        }
+        if (blockIdx.x == gridDim.x - 1)
+            *nvalid = (int32_t)(base + s);
+    }
+    __syncthreads();
+    int64_t pos = base + warp_off[warp] + (incl - n);
+    for (int k = 0; k < kPerThread; ++k) {
+        if (bits & (1u << k)) {
+            const int64_t i = i0 + k;
+            const int32_t r = c.row_of_token ? c.row_of_token[i] : (int32_t)i;
+            const int32_t y = c.mode == TURNOPD_SAMPLED_TOKEN ? c.sampled_ids[i] : -1;
+            rows[pos++] = make_int4((int32_t)i, r, y, __float_as_int(c.w[i]));
+        }
+    }
+}
+
+// ---------------------------------------------------------------- row kernel
+
+template <typename TIn> struct Vec;
+template <> struct Vec<__nv_bfloat16> {
+    static constexpr int N = 8;
+    __device__ static void load(const void *p, float *x)
+    {
+        const uint4 u = __ldg(reinterpret_cast<const uint4 *>(p));
+        x[0] = bf16lo(u.x), x[1] = bf16hi(u.x), x[2] = bf16lo(u.y), x[3] = bf16hi(u.y);
+        x[4] = bf16lo(u.z), x[5] = bf16hi(u.z), x[6] = bf16lo(u.w), x[7] = bf16hi(u.w);
+    }
+};
+template <> struct Vec<float> {
+    static constexpr int N = 4;
+    __device__ static void load(const void *p, float *x)
+    {
+        const float4 u = __ldg(reinterpret_cast<const float4 *>(p));
+        x[0] = u.x, x[1] = u.y, x[2] = u.z, x[3] = u.w;
+    }
+};
+
+template <typename TOut, int N> __device__ __forceinline__ void store_vec(TOut *p, const float *g);
+template <> __device__ __forceinline__ void store_vec<__nv_bfloat16, 8>(__nv_bfloat16 *p, const float *g)
+{
+    uint4 u;
+    u.x = pack_bf16x2(g[0], g[1]);
+    u.y = pack_bf16x2(g[2], g[3]);
+    u.z = pack_bf16x2(g[4], g[5]);
+    u.w = pack_bf16x2(g[6], g[7]);
+    *reinterpret_cast<uint4 *>(p) = u;
+}
+template <> __device__ __forceinline__ void store_vec<__nv_bfloat16, 4>(__nv_bfloat16 *p, const float *g)
+{
+    uint2 u;
+    u.x = pack_bf16x2(g[0], g[1]);
+    u.y = pack_bf16x2(g[2], g[3]);
+    *reinterpret_cast<uint2 *>(p) = u;
+}
+template <> __device__ __forceinline__ void store_vec<float, 8>(float *p, const float *g)
+{
+    reinterpret_cast<float4 *>(p)[0] = make_float4(g[0], g[1], g[2], g[3]);
+    reinterpret_cast<float4 *>(p)[1] = make_float4(g[4], g[5], g[6], g[7]);
+}
+template <> __device__ __forceinline__ void store_vec<float, 4>(float *p, const float *g)
+{
+    *reinterpret_cast<float4 *>(p) = make_float4(g[0], g[1], g[2], g[3]);
+}
+
+// Fold n student/teacher values into the online accumulators.
+template <int N>
+__device__ __forceinline__ void accumulate(Student &s, Teacher &t, const float *a, const float *b)
+{
+    float mx = a[0], xd = a[0] - b[0], my = b[0];
+#pragma unroll
+    for (int k = 1; k < N; ++k) {
+        if (a[k] > mx) {
+            mx = a[k];
+            xd = a[k] - b[k];
+        }
+        my = fmaxf(my, b[k]);
+    }
+    if (mx > s.m) {
+        const float f = ex2((s.m - mx) * kLog2e);
+        s.a = fmaf(s.s, s.d - xd, s.a) * f;
+        s.s *= f;
+        s.m = mx;
+        s.d = xd;
+    }
+    if (my > t.m) {
+        t.s *= ex2((t.m - my) * kLog2e);
+        t.m = my;
+    }
+    const float ns = -s.m * kLog2e, nt = -t.m * kLog2e;
+#pragma unroll
+    for (int k = 0; k < N; ++k) {
+        const float e = ex2(fmaf(a[k], kLog2e, ns));
+        s.s += e;
+        s.a = fmaf(e, (a[k] - b[k]) - s.d, s.a);
+        t.s += ex2(fmaf(b[k], kLog2e, nt));
+    }
+}
+
+constexpr int kRowThreads = 256;
+
+template <typename TIn, typename TOut, bool VEC>
+__global__ void __launch_bounds__(kRowThreads)
+k_row_portable(RowIn p)
+{
+    __shared__ Student red_s[kRowThreads / 32];
+    __shared__ Teacher red_t[kRowThreads / 32];
+    __shared__ float bc[5];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int nvalid = *p.nvalid;
+    const TIn *zs = static_cast<const TIn *>(p.zs);
+    const TIn *zt = static_cast<const TIn *>(p.zt);
+    TOut *grad = static_cast<TOut *>(p.grad);
+    constexpr int N = Vec<TIn>::N;
+    const int64_t V = p.vocab;
+    const int64_t nvec = VEC ? V / N : 0;
+
+    for (int j = blockIdx.x; j < nvalid; j += gridDim.x) {
+        const int4 meta = p.rows[j];
+        const int i = meta.x;
+        const int64_t r = meta.y;
+        const TIn *rs = zs + r * p.ld;
+        const TIn *rt = zt + r * p.ld;
+        Student s = student_empty();
+        Teacher t = teacher_empty();
+        if (VEC) {
+            for (int64_t q = threadIdx.x; q < nvec; q += kRowThreads) {
+                float a[N], b[N];
+                Vec<TIn>::load(rs + q * N, a);
+                Vec<TIn>::load(rt + q * N, b);
+                accumulate<N>(s, t, a, b);
+            }
+        }
+        for (int64_t v = nvec * N + threadIdx.x; v < V; v += kRowThreads) {
+            float a = to_float(rs[v]), b = to_float(rt[v]);
+            accumulate<1>(s, t, &a, &b);
+        }
+        s = warp_merge(s);
+        t = warp_merge(t);
+        if (lane == 0) {
+            red_s[warp] = s;
+            red_t[warp] = t;
+        }
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            Student S = red_s[0];
+            Teacher U = red_t[0];
+            for (int k = 1; k < kRowThreads / 32; ++k) {
+                S = student_merge(S, red_s[k]);
+                U = teacher_merge(U, red_t[k]);
+            }
+            const RowConst rc = row_const(S, U);
+            float ell = rc.kl;
+            if (p.mode == TURNOPD_SAMPLED_TOKEN) {
+                const int32_t y = meta.z;
+                ell = (to_float(rs[y]) - to_float(rt[y])) - rc.dl;
+            }
+            const float wi = __int_as_float(meta.w);
+            if (!isfinite(rc.lse_s) || !isfinite(rc.lse_t) || !isfinite(ell))
+                set_status(p.status, TURNOPD_ERR_NONFINITE);
+            p.token_loss[i] = ell;
+            p.row_wl[j] = (double)wi * (double)ell;
+            bc[0] = rc.lse_s;
+            bc[1] = rc.d;
+            bc[2] = rc.cp;  // g = w p (((z_s - z_t) - d) - cp)
+            bc[3] = wi;
+            bc[4] = wi * ell;
+        }
+        __syncthreads();
+        if (grad) {
+            const float nl = -bc[0] * kLog2e, d = bc[1], cp = bc[2], wi = bc[3], wl = bc[4];
+            const bool sampled = p.mode == TURNOPD_SAMPLED_TOKEN;
+            const int64_t y = sampled ? (int64_t)meta.z : -1;
+            TOut *gr = grad + r * p.ld;
+            if (VEC) {
+                for (int64_t q = threadIdx.x; q < nvec; q += kRowThreads) {
+                    float a[N], b[N], g[N];
+                    Vec<TIn>::load(rs + q * N, a);
+                    Vec<TIn>::load(rt + q * N, b);
+#pragma unroll
+                    for (int k = 0; k < N; ++k) {
+                        const float pv = ex2(fmaf(a[k], kLog2e, nl));
+                        g[k] = sampled ? (((q * N + k) == y ? wl : 0.f) - wl * pv)
+                                       : wi * pv * (((a[k] - b[k]) - d) - cp);
+                    }
+                    store_vec<TOut, N>(gr + q * N, g);
+                }
+            }
+            for (int64_t v = nvec * N + threadIdx.x; v < V; v += kRowThreads) {
+                const float a = to_float(rs[v]), b = to_float(rt[v]);
+                const float pv = ex2(fmaf(a, kLog2e, nl));
+                const float g = sampled ? ((v == y ? wl : 0.f) - wl * pv) : wi * pv * (((a - b) - d) - cp);
+                gr[v] = from_float<TOut>(g);
+            }
+        }
+        __syncthreads();  // bc / red reuse by the next row
+    }
+}
+
+// ---------------------------------------------------------------- zero fill
+
+template <typename TOut>
+__global__ void k_zero_masked(const uint8_t *__restrict__ mask, const int32_t *__restrict__ rot,
+                              int64_t T, int64_t num_rows, int64_t ld, int64_t vocab, TOut *grad)
+{
+    for (int64_t i = blockIdx.x; i < T; i += gridDim.x) {
+        if (mask[i])
+            continue;
+        const int64_t r = rot ? (int64_t)rot[i] : i;
+        if (r < 0 || r >= num_rows)
+            continue;
+        TOut *g = grad + r * ld;
+        for (int64_t v = threadIdx.x; v < vocab; v += blockDim.x)
+            g[v] = from_float<TOut>(0.f);
+    }
+}
+
+// ---------------------------------------------------------------- loss sum
+
+// loss = sum_j row_wl[j] over the compacted rows (= token order), fixed tree.
+__global__ void k_loss_sum(const double *__restrict__ row_wl, const int32_t *__restrict__ nvalid,
+                           double *__restrict__ loss, int32_t *status)
+{
+    __shared__ double part[32];
+    const int n = *nvalid;
+    double s = 0.0;
+    for (int j = threadIdx.x; j < n; j += blockDim.x)
+        s += row_wl[j];
+    s = warp_sum_f64(s);
+    if ((threadIdx.x & 31) == 0)
+        part[threadIdx.x >> 5] = s;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        double tot = 0.0;
+        for (int k = 0; k < (int)(blockDim.x >> 5); ++k)
+            tot += part[k];
+        if (!isfinite(tot))
+            set_status(status, TURNOPD_ERR_NONFINITE);
+        *loss = tot;
+    }
+}
+
+// ---------------------------------------------------------------- launcher
+
+
+template <typename TIn, typename TOut>
+static cudaError_t launch_portable(const RowIn &p, bool vec, int grid, cudaStream_t stream)
+{
+    if (vec)
+        k_row_portable<TIn, TOut, true><<<grid, kRowThreads, 0, stream>>>(p);
+    else
+        k_row_portable<TIn, TOut, false><<<grid, kRowThreads, 0, stream>>>(p);
+    return cudaGetLastError();
+}
+
+static bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+cudaError_t launch_loss(const LossArgs &a, const LossWorkspace &ws, cudaStream_t stream)
+{
+    const int nblk = (int)((a.T + kCompactBlock - 1) / kCompactBlock);
+    CompactIn c{a.mask, a.row_of_token, a.sampled_ids, a.w, a.num_rows, a.vocab, a.T, a.mode,
+                a.token_loss, a.status};
+    k_compact_count<<<nblk, kCompactThreads, 0, stream>>>(c, ws.blk_count);
+    k_compact_scatter<<<nblk, kCompactThreads, 0, stream>>>(c, ws.blk_count, ws.rows, ws.nvalid);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess)
+        return e;
+
+    const int sms = device_sm_count();
+    if (a.grad && (a.flags & TURNOPD_ZERO_MASKED_GRAD)) {
+        const int grid = (int)std::min<int64_t>(a.T, (int64_t)sms * 8);
+        if (a.grad_dtype == TURNOPD_BF16)
+            k_zero_masked<__nv_bfloat16><<<grid, 256, 0, stream>>>(
+                a.mask, a.row_of_token, a.T, a.num_rows, a.ld, a.vocab,
+                static_cast<__nv_bfloat16 *>(a.grad));
+        else
+            k_zero_masked<float><<<grid, 256, 0, stream>>>(a.mask, a.row_of_token, a.T, a.num_rows,
+                                                            a.ld, a.vocab, static_cast<float *>(a.grad));
+    }
+
+    RowIn p{a.zs, a.zt, a.ld, a.vocab, a.row_of_token, a.sampled_ids, a.w, a.mode, a.grad,
+            a.token_loss, ws.row_wl, ws.rows, ws.nvalid, a.status};
+    bool done = false;
+    if (a.in_dtype == TURNOPD_BF16 && !(a.flags & TURNOPD_FORCE_PORTABLE)) {
+        e = launch_row_cluster(p, a.grad_dtype == TURNOPD_F32, stream, &done);
+        if (e != cudaSuccess)
+            return e;
+    }
+    if (!done) {
+        const size_t esz = a.in_dtype == TURNOPD_BF16 ? 2 : 4;
+        const bool vec = aligned16(a.zs) && aligned16(a.zt) && (!a.grad || aligned16(a.grad)) &&
+                         ((size_t)a.ld * esz) % 16 == 0;
+        const int grid = (int)std::min<int64_t>(std::max<int64_t>(a.T, 1), (int64_t)sms * 8);
+        const bool g32 = a.grad_dtype == TURNOPD_F32;
+        if (a.in_dtype == TURNOPD_BF16)
+            e = g32 ? launch_portable<__nv_bfloat16, float>(p, vec, grid, stream)
+                    : launch_portable<__nv_bfloat16, __nv_bfloat16>(p, vec, grid, stream);
+        else
+            e = g32 ? launch_portable<float, float>(p, vec, grid, stream)
+                    : launch_portable<float, __nv_bfloat16>(p, vec, grid, stream);
+        if (e != cudaSuccess)
+            return e;
+    }
+    k_loss_sum<<<1, 1024, 0, stream>>>(ws.row_wl, ws.nvalid, a.loss, a.status);
+    return cudaGetLastError();
+}
+
+}  // namespace turnopd

@@ -1,0 +1,119 @@
+"""The C-ABI library loads and exports every symbol include/turnopd.h declares,
+and its host-side argument checks answer without a GPU (they return before any
+CUDA call).  No compute call is made here."""
+import ctypes
+import math
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "turnopd.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2607_05804_gb300 import build as B
+
+    B.build()
+    import paper_2607_05804_gb300 as P
+
+    return P.load()
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"^[A-Za-z_][\w \*]*?\b(turnopd_\w+)\s*\(", src, flags=re.M)))
+
+
+def test_header_declares_the_entry_points():
+    names = declared_functions()
+    for n in ("turnopd_turn_counts", "turnopd_weights", "turnopd_loss_fwd_bwd",
+              "turnopd_turn_stats", "turnopd_alpha_schedule", "turnopd_status_string",
+              "turnopd_weights_workspace_bytes", "turnopd_loss_workspace_bytes"):
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(lib):
+    missing = [n for n in declared_functions() if not hasattr(lib, n)]
+    assert not missing, missing
+
+
+def test_binding_names_match_header():
+    import paper_2607_05804_gb300 as P
+
+    for n in declared_functions():
+        assert hasattr(P, n), n
+
+
+FAKE = ctypes.c_void_p(0x10000)  # never dereferenced: every call below fails validation first
+
+
+def test_loss_host_validation(lib):
+    P = ctypes.c_void_p
+    f = lib.turnopd_loss_fwd_bwd
+    ws_need = lib.turnopd_loss_workspace_bytes(64)
+    assert ws_need > 0
+
+    def call(zs=FAKE, ld=1024, vocab=1024, rows=64, T=64, mode=0, grad_dtype=0, in_dtype=1,
+             flags=0, ws=FAKE, wsb=None, loss=FAKE, status=FAKE, y=FAKE, grad=FAKE):
+        return f(zs, FAKE, in_dtype, ld, vocab, rows, None, y, FAKE, FAKE, T, mode, grad,
+                 grad_dtype, flags, FAKE, loss, ws, ws_need if wsb is None else wsb, status, None)
+
+    assert call(zs=None) == 1
+    assert call(loss=None) == 1
+    assert call(status=None) == 1
+    assert call(mode=1, y=None) == 1
+    assert call(ld=100, vocab=101) == 2
+    assert call(vocab=0) == 2
+    assert call(rows=10) == 2          # dense rows need num_rows >= num_tokens
+    assert call(mode=7) == 6
+    assert call(in_dtype=5) == 6
+    assert call(grad_dtype=3) == 6
+    assert call(flags=0x8000) == 6
+    assert call(ws=None) == 10
+    assert call(wsb=ws_need - 1) == 10
+    assert call(ws=ctypes.c_void_p(0x10010)) == 10  # not 256-byte aligned
+    assert call(zs=ctypes.c_void_p(0x10001)) == 2   # misaligned bf16 pointer
+
+
+def test_structure_host_validation(lib):
+    f = lib.turnopd_weights
+    need = lib.turnopd_weights_workspace_bytes(4, 8)
+    base = dict(tid=FAKE, msk=FAKE, off=FAKE, B=4, T=100, Tm=8, alpha=0.5, scope=0, n_min=0,
+                w=FAKE, ws=FAKE, wsb=need, st=FAKE)
+
+    def call(**kw):
+        a = dict(base, **kw)
+        return f(a["tid"], a["msk"], a["off"], a["B"], a["T"], a["Tm"], a["alpha"], a["scope"],
+                 a["n_min"], None, a["w"], a["ws"], a["wsb"], a["st"], None)
+
+    assert call(off=None) == 1
+    assert call(st=None) == 1
+    assert call(w=None) == 1
+    assert call(Tm=0) == 2
+    assert call(Tm=5000) == 2
+    assert call(B=-1) == 2
+    assert call(alpha=1.5) == 2
+    assert call(alpha=float("nan")) == 2
+    assert call(scope=9) == 6
+    assert call(wsb=need - 1) == 10
+    g = lib.turnopd_turn_stats
+    assert g(None, FAKE, FAKE, FAKE, 4, 100, 8, FAKE, FAKE, FAKE, FAKE, FAKE, FAKE, None) == 1
+    assert g(FAKE, FAKE, FAKE, FAKE, 4, 100, 8, FAKE, FAKE, None, FAKE, FAKE, FAKE, None) == 1
+    h = lib.turnopd_turn_counts
+    assert h(FAKE, FAKE, FAKE, 4, 100, 8, FAKE, None, FAKE, None) == 1
+
+
+def test_alpha_schedule_and_status_strings(lib, oracle):
+    import paper_2607_05804_gb300 as P
+
+    for k in range(0, 101, 7):
+        assert P.turnopd_alpha_schedule(k, 100) == oracle.alpha_schedule(k, 100)
+    assert math.isnan(P.turnopd_alpha_schedule(1, 0))
+    assert math.isnan(P.turnopd_alpha_schedule(1, 10, 0.5, 0.5))
+    for code in range(11):
+        assert P.turnopd_status_string(code)
+    assert P.turnopd_status_string(0) == "ok"

@@ -1,0 +1,417 @@
+"""GPU parity: libturnopd (through its C ABI) against the fp64 CPU oracle on the
+same seeded inputs, element by element, within the tolerances in parity.py.
+
+Sizes: the tiny batch (V = 1024, fp32) exhaustively over alpha x mode x kernel;
+packed batches at a reduced vocabulary that spans many tiles and a ragged tail
+(every row checked); the three agent-shaped batches at the full V = 151,936 in
+bf16 with the benchmark's launch configuration (sampled rows checked against
+the oracle, all rows against size-free properties); edge and error cases.
+"""
+import numpy as np
+import pytest
+
+import workloads as W
+from parity import (assert_grad_rows, assert_loss, assert_stats, assert_token_loss,
+                    assert_weights)
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+FORCE_PORTABLE = 0x100
+ZERO_MASKED = 0x1
+
+
+@pytest.fixture(scope="module")
+def P():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2607_05804_gb300 as P
+
+    P.load()
+    return P
+
+
+def make_step(P, b, V, *, compact, mode=0, alpha=0.5, flags=0, y=None, scope=0, n_min=0):
+    from paper_2607_05804_gb300.step import LossStep, to_device
+
+    tid, msk, off, rot = to_device(b, "cuda", compact)
+    return LossStep(tid, msk, off, b.max_turns, V, row_of_token=rot, sampled_ids=y, mode=mode,
+                    alpha=alpha, scope=scope, n_min=n_min, flags=flags)
+
+
+def per_token_ids(b, y_rows, compact):
+    """Sampled ids are per token; for compact rows, row k belongs to the k-th supervised token."""
+    if not compact:
+        return y_rows
+    y = torch.zeros(b.num_tokens, dtype=torch.int32, device=y_rows.device)
+    idx = torch.from_numpy(np.nonzero(b.loss_mask)[0]).to(y_rows.device)
+    y[idx] = y_rows
+    return y
+
+
+def bits_or_f32(z):
+    return W.bf16_bits(z) if z.dtype == torch.bfloat16 else z.detach().cpu().numpy()
+
+
+def run_chain(P, oracle, b, V, zs, zt, *, mode, alpha, flags=0, grad_dtype=None, compact=False,
+              scope=0, n_min=0, seed_y=1):
+    """GPU chain vs oracle chain on every row of the batch."""
+    y = per_token_ids(b, W.sample_ids(zs, seed_y, V), compact) if mode == 1 else None
+    step = make_step(P, b, V, compact=compact, mode=mode, alpha=alpha, flags=flags, y=y,
+                     scope=scope, n_min=n_min)
+    gdt = zs.dtype if grad_dtype is None else grad_dtype
+    grad = torch.full(zs.shape, 7.0, dtype=gdt, device="cuda")
+    step.run(zs, zt, grad)
+    torch.cuda.synchronize()
+    assert step.status() == 0
+    T = b.num_tokens
+    w_ref = oracle.weights(b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns, alpha, scope, n_min)
+    w_gpu = step.w[:T].cpu().numpy()
+    assert_weights(w_gpu, w_ref)
+    rot = b.compact_rows() if compact else None
+    ynp = y.cpu().numpy() if y is not None else None
+    g_ref, tl_ref, loss_ref = oracle.loss_fwd_bwd(
+        bits_or_f32(zs), bits_or_f32(zt), V, b.loss_mask, w_ref.astype(np.float32), mode=mode,
+        row_of_token=rot, sampled_ids=ynp)
+    tl = step.token_loss[:T].cpu().numpy()
+    assert_token_loss(tl, tl_ref, b.loss_mask)
+    assert_loss(step.loss.item(), loss_ref)
+    rows = np.nonzero(b.loss_mask)[0] if not compact else np.arange(b.num_valid)
+    toks = np.nonzero(b.loss_mask)[0]
+    g = grad.float().cpu().numpy().astype(np.float64)
+    extra = dict(ell=tl_ref[toks], w=w_ref[toks]) if mode == 1 else {}
+    assert_grad_rows(g[rows][:, :V], g_ref[rows], bf16=(gdt == torch.bfloat16), **extra)
+    st_ref = oracle.turn_stats(tl_ref, b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns)
+    st = {k: v.cpu().numpy() for k, v in step.stats().items()}
+    assert_stats(st, st_ref, tl_ref, b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns)
+    return step, grad
+
+
+# ---------------------------------------------------------------- tiny batch, exhaustive
+
+@pytest.mark.parametrize("flags", [0, FORCE_PORTABLE], ids=["default", "portable"])
+@pytest.mark.parametrize("mode", [0, 1], ids=["full", "sampled"])
+@pytest.mark.parametrize("alpha", [0.0, 0.5, 1.0])
+def test_tiny_exhaustive(P, oracle, alpha, mode, flags):
+    b = W.tiny()
+    zs, zt = W.make_logits(b.num_tokens, 1024, "tiny", torch.float32, seed=0, device="cuda")
+    run_chain(P, oracle, b, 1024, zs, zt, mode=mode, alpha=alpha, flags=flags)
+
+
+# ---------------------------------------------------------------- reduced vocabulary, all rows
+
+@pytest.mark.parametrize("V,ld", [(4099, 4104), (4099, 4099), (16384, 16384)])
+@pytest.mark.parametrize("gdt", ["bf16", "f32"])
+@pytest.mark.parametrize("flags", [0, FORCE_PORTABLE], ids=["default", "portable"])
+def test_packed_reduced_vocab(P, oracle, V, ld, gdt, flags):
+    b = W.packed(seed=2, num_traj=4, traj_len=1024)
+    zs, zt = W.make_logits(b.num_tokens, V, "agent", torch.bfloat16, seed=3, device="cuda", ld=ld)
+    run_chain(P, oracle, b, V, zs, zt, mode=0, alpha=0.5, flags=flags,
+              grad_dtype=torch.bfloat16 if gdt == "bf16" else torch.float32)
+
+
+@pytest.mark.parametrize("mode", [0, 1], ids=["full", "sampled"])
+def test_household_compact_reduced_vocab(P, oracle, mode):
+    b = W.household(seed=5, num_traj=4, traj_len=4096)
+    V = 8192
+    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=6, device="cuda")
+    run_chain(P, oracle, b, V, zs, zt, mode=mode, alpha=0.25, compact=True)
+
+
+@pytest.mark.parametrize("scope,n_min", [(0, 2), (1, 0), (1, 3)])
+def test_scopes_and_floor(P, oracle, scope, n_min):
+    b = W.multihop(seed=7, num_traj=6, min_len=256, max_len=2048)
+    V = 2048
+    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=8, device="cuda")
+    run_chain(P, oracle, b, V, zs, zt, mode=0, alpha=0.7, compact=True, scope=scope, n_min=n_min)
+
+
+# ---------------------------------------------------------------- cluster kernel, all rows
+
+@pytest.mark.parametrize("V", [50000, W.V_QWEN])
+@pytest.mark.parametrize("mode", [0, 1], ids=["full", "sampled"])
+@pytest.mark.parametrize("gdt", ["bf16", "f32"])
+def test_cluster_kernel_all_rows(P, oracle, V, mode, gdt):
+    """The cluster-resident kernel (vocabularies >= 32768, multiple of 8) on every row:
+    V = 50,000 gives a ragged last slice (6250 vectors over 8 CTAs)."""
+    b = W.packed(seed=11, num_traj=2, traj_len=256)
+    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=12, device="cuda")
+    run_chain(P, oracle, b, V, zs, zt, mode=mode, alpha=0.5, compact=True,
+              grad_dtype=torch.bfloat16 if gdt == "bf16" else torch.float32)
+
+
+def test_cluster_matches_portable(P, oracle):
+    """Both kernels agree with each other to within the oracle tolerances."""
+    b = W.packed(seed=13, num_traj=2, traj_len=512)
+    V = W.V_QWEN
+    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=13, device="cuda")
+    out = []
+    for flags in (0, FORCE_PORTABLE):
+        step = make_step(P, b, V, compact=True, flags=flags)
+        g = torch.empty(zs.shape, dtype=torch.float32, device="cuda")
+        step.run(zs, zt, g)
+        torch.cuda.synchronize()
+        assert step.status() == 0
+        out.append((g, step.token_loss[:b.num_tokens].clone(), step.loss.item()))
+    (g0, t0, l0), (g1, t1, l1) = out
+    assert abs(l0 - l1) <= 2e-5 * abs(l0)
+    assert ((t0 - t1).abs() <= 2e-4 * t0.abs().clamp(min=1)).all()
+    rowmax = g0.abs().amax(dim=1, keepdim=True)
+    assert ((g0 - g1).abs() <= 2e-4 * rowmax).all()
+
+
+# ---------------------------------------------------------------- full vocabulary, sampled rows
+
+FULL_V = W.V_QWEN
+
+
+def full_size_check(P, oracle, b, mode, alpha, n_rows=12, seed=0):
+    V = FULL_V
+    R = b.num_valid
+    zs, zt = W.make_logits(R, V, "agent", torch.bfloat16, seed=seed, device="cuda")
+    y_rows = W.sample_ids(zs, seed + 1) if mode == 1 else None
+    y = per_token_ids(b, y_rows, True) if mode == 1 else None
+    step = make_step(P, b, V, compact=True, mode=mode, alpha=alpha, y=y)
+    grad = torch.empty_like(zs)
+    step.run(zs, zt, grad)
+    torch.cuda.synchronize()
+    assert step.status() == 0
+    T = b.num_tokens
+    w_ref = oracle.weights(b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns, alpha)
+    assert_weights(step.w[:T].cpu().numpy(), w_ref)
+    rng = np.random.default_rng(seed)
+    rows = np.unique(np.concatenate([[0, R - 1], rng.integers(0, R, n_rows)]))
+    toks = np.nonzero(b.loss_mask)[0][rows]
+    tl = step.token_loss[:T].cpu().numpy()
+    w32 = w_ref.astype(np.float32)
+    zsr, ztr = W.bf16_bits(zs[rows]), W.bf16_bits(zt[rows])
+    gg = grad[rows].float().cpu().numpy().astype(np.float64)
+    for k, (r, i) in enumerate(zip(rows, toks)):
+        yy = int(y_rows[r]) if y_rows is not None else 0
+        _, _, ell, _, g = oracle.row(zsr[k], ztr[k], mode=mode, y=yy, w=float(w32[i]))
+        assert_token_loss(tl[i:i + 1], [ell])
+        extra = dict(ell=[ell], w=[w32[i]]) if mode == 1 else {}
+        assert_grad_rows(gg[k:k + 1], g[None, :], bf16=True, **extra)
+    # size-free properties over every row
+    wl = np.dot(w32.astype(np.float64), tl.astype(np.float64))
+    assert abs(step.loss.item() - wl) <= 1e-9 * abs(wl)
+    assert (tl[b.loss_mask == 0] == 0).all()
+    if mode == 0:
+        assert (tl[b.loss_mask == 1] >= -1e-4).all()
+    # every row's gradient sums to 0; bf16 rounding moves each term by <= 2^-9 of itself
+    for r0 in range(0, R, 2048):
+        chunk = grad[r0:r0 + 2048]
+        s = torch.sum(chunk, dim=1, dtype=torch.float32).abs()
+        a = torch.sum(chunk.abs(), dim=1, dtype=torch.float32)
+        assert (s <= 2.0 ** -8 * a + 1e-30).all()
+    st = step.stats()
+    n_bt, counts = oracle.turn_counts(b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns)
+    assert np.array_equal(st["traj_turn_cnt"].cpu().numpy(), n_bt)
+    assert np.array_equal(st["turn_surv"].cpu().numpy(), counts[:b.max_turns])
+    assert abs(st["turn_sum"].sum().item() - tl.astype(np.float64).sum()) <= 1e-9 * max(1, abs(tl).sum())
+
+
+def test_full_packed(P, oracle):
+    full_size_check(P, oracle, W.packed(0), mode=0, alpha=0.5)
+
+
+def test_full_household(P, oracle):
+    for alpha in (0.0, 0.25, 0.5, 0.75, 1.0):
+        b = W.household(0)
+        V = FULL_V
+        # weights over the full batch for every alpha of the sweep
+        step = make_step(P, b, V, compact=True, alpha=alpha)
+        step.weights()
+        torch.cuda.synchronize()
+        assert step.status() == 0
+        assert_weights(step.w[:b.num_tokens].cpu().numpy(),
+                       oracle.weights(b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns, alpha))
+    full_size_check(P, oracle, W.household(0), mode=0, alpha=0.5, seed=3)
+
+
+@pytest.mark.parametrize("mode", [0, 1], ids=["full", "sampled"])
+def test_full_multihop(P, oracle, mode):
+    full_size_check(P, oracle, W.multihop(0), mode=mode, alpha=0.5, seed=5)
+
+
+# ---------------------------------------------------------------- turn stats in isolation
+
+def test_turn_stats_full_size(P, oracle):
+    from paper_2607_05804_gb300.step import to_device
+
+    for b in (W.household(0), W.multihop(0)):
+        rng = np.random.default_rng(3)
+        tl = (rng.gamma(2.0, 1.0, b.num_tokens) * b.loss_mask).astype(np.float32)
+        step = make_step(P, b, 8, compact=True)
+        step.token_loss[:b.num_tokens] = torch.from_numpy(tl).cuda()
+        step.turn_stats()
+        torch.cuda.synchronize()
+        assert step.status() == 0
+        st_ref = oracle.turn_stats(tl.astype(np.float64), b.turn_id, b.loss_mask, b.traj_offsets,
+                                   b.max_turns)
+        st = {k: v.cpu().numpy() for k, v in step.stats().items()}
+        assert np.array_equal(st["traj_turn_cnt"], st_ref["traj_turn_cnt"])
+        assert np.array_equal(st["turn_cnt"], st_ref["turn_cnt"])
+        assert np.array_equal(st["turn_surv"], st_ref["turn_surv"])
+        np.testing.assert_allclose(st["traj_turn_sum"], st_ref["traj_turn_sum"], rtol=1e-12, atol=1e-9)
+        np.testing.assert_allclose(st["turn_sum"], st_ref["turn_sum"], rtol=1e-12, atol=1e-9)
+
+
+# ---------------------------------------------------------------- edge and error cases
+
+def test_empty_and_all_masked(P, oracle):
+    from paper_2607_05804_gb300.step import LossStep
+
+    # empty batch
+    e = lambda dt: torch.zeros(0, dtype=dt, device="cuda")
+    off = torch.zeros(2, dtype=torch.int64, device="cuda")
+    step = LossStep(e(torch.int32), e(torch.uint8), off, 3, 16)
+    z = torch.zeros((0, 16), dtype=torch.bfloat16, device="cuda")
+    step.loss.fill_(5.0)
+    step.run(z, z, torch.zeros_like(z))
+    torch.cuda.synchronize()
+    assert step.status() == 0 and step.loss.item() == 0.0
+    # all-masked batch with empty trajectories
+    b = W._from_spans("masked", [[("o", 40)], [], [("o", 7), ("p", 3)]], max_turns=2)
+    zs, zt = W.make_logits(b.num_tokens, 64, "tiny", torch.float32, seed=0, device="cuda")
+    step = make_step(P, b, 64, compact=False)
+    step.token_loss.fill_(3.0)
+    step.run(zs, zt, torch.zeros_like(zs))
+    torch.cuda.synchronize()
+    assert step.status() == 0
+    assert step.loss.item() == 0.0
+    assert not step.w.any() and not step.token_loss.any()
+    assert not step.turn_cnt.any()
+
+
+def test_random_structures_with_empty_trajectories(P, oracle):
+    rng = np.random.default_rng(42)
+    for k in range(6):
+        b = W.random_structure(rng, num_traj=int(rng.integers(1, 9)), max_len=80,
+                               max_turns=int(rng.integers(1, 7)))
+        zs, zt = W.make_logits(b.num_tokens, 40, "agent", torch.bfloat16, seed=k, device="cuda",
+                               ld=48)
+        if b.num_tokens == 0:
+            continue
+        run_chain(P, oracle, b, 40, zs, zt, mode=k % 2, alpha=0.3 * (k % 4))
+
+
+def test_zero_masked_grad_and_untouched_rows(P, oracle):
+    b = W.packed(seed=4, num_traj=2, traj_len=512)
+    V = 1000
+    zs, zt = W.make_logits(b.num_tokens, V, "agent", torch.bfloat16, seed=4, device="cuda", ld=1024)
+    for flags in (0, ZERO_MASKED):
+        step = make_step(P, b, V, compact=False, flags=flags)
+        grad = torch.full(zs.shape, 3.0, dtype=torch.bfloat16, device="cuda")
+        step.run(zs, zt, grad)
+        torch.cuda.synchronize()
+        masked = torch.from_numpy(b.loss_mask == 0).cuda()
+        g = grad[masked]
+        if flags:
+            assert not g[:, :V].any()
+        else:
+            assert (g[:, :V] == 3.0).all()
+        assert (grad[:, V:] == 3.0).all()  # padding columns never written
+
+
+def test_padding_never_read(P, oracle):
+    b = W.packed(seed=6, num_traj=2, traj_len=256)
+    V = 500
+    zs, zt = W.make_logits(b.num_tokens, V, "agent", torch.bfloat16, seed=6, device="cuda", ld=512)
+    ref_step, ref_grad = run_chain(P, oracle, b, V, zs, zt, mode=0, alpha=0.5)
+    zs[:, V:] = float("nan")
+    zt[:, V:] = float("inf")
+    step = make_step(P, b, V, compact=False)
+    grad = torch.full(zs.shape, 7.0, dtype=torch.bfloat16, device="cuda")
+    step.run(zs, zt, grad)
+    torch.cuda.synchronize()
+    assert step.status() == 0
+    assert torch.equal(grad, ref_grad) and step.loss.item() == ref_step.loss.item()
+
+
+def test_deterministic(P, oracle):
+    b = W.packed(seed=1, num_traj=4, traj_len=2048)
+    V = FULL_V
+    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=1, device="cuda")
+    outs = []
+    for _ in range(2):
+        step = make_step(P, b, V, compact=True)
+        grad = torch.empty_like(zs)
+        step.run(zs, zt, grad)
+        torch.cuda.synchronize()
+        outs.append((grad.clone(), step.token_loss.clone(), step.loss.item(), step.turn_sum.clone()))
+    assert torch.equal(outs[0][0], outs[1][0]) and torch.equal(outs[0][1], outs[1][1])
+    assert outs[0][2] == outs[1][2] and torch.equal(outs[0][3], outs[1][3])
+
+
+def test_device_errors(P, oracle):
+    b = W.tiny()
+    V = 64
+    zs, zt = W.make_logits(b.num_tokens, V, "tiny", torch.float32, seed=0, device="cuda")
+    valid = np.nonzero(b.loss_mask)[0]
+    # row index out of range -> TOKEN_RANGE, that token's loss is 0, the rest unaffected
+    step = make_step(P, b, V, compact=True)
+    step.row_of_token[int(valid[5])] = b.num_valid + 3
+    step.run(zs[:b.num_valid], zt[:b.num_valid], torch.zeros_like(zs[:b.num_valid]))
+    torch.cuda.synchronize()
+    assert step.status() == 5
+    assert step.token_loss[int(valid[5])].item() == 0.0
+    # sampled id out of range
+    y = torch.zeros(b.num_tokens, dtype=torch.int32, device="cuda")
+    y[int(valid[2])] = V
+    step = make_step(P, b, V, compact=False, mode=1, y=y)
+    step.run(zs, zt, torch.zeros_like(zs))
+    torch.cuda.synchronize()
+    assert step.status() == 5
+    # supervised token with a turn id out of range
+    step = make_step(P, b, V, compact=False)
+    step.turn_id[int(valid[0])] = b.max_turns
+    step.run(zs, zt, torch.zeros_like(zs))
+    torch.cuda.synchronize()
+    assert step.status() == 4
+    # bad offsets
+    step = make_step(P, b, V, compact=False)
+    step.traj_offsets[1] = b.num_tokens + 5
+    step.weights()
+    torch.cuda.synchronize()
+    assert step.status() == 3
+    # non-finite logits
+    step = make_step(P, b, V, compact=False)
+    zs2 = zs.clone()
+    zs2[int(valid[1]), 3] = float("inf")
+    step.run(zs2, zt, torch.zeros_like(zs))
+    torch.cuda.synchronize()
+    assert step.status() == 9
+
+
+def test_virtual_ranks_merge(P, oracle):
+    """Data-parallel by whole trajectories, emulated on one GPU: each 'rank' runs its
+    own trajectories with the rank-summed count vector; merged results equal one call."""
+    b = W.packed(seed=9, num_traj=6, traj_len=1024)
+    V = 3000
+    zs, zt = W.make_logits(b.num_tokens, V, "agent", torch.bfloat16, seed=9, device="cuda")
+    whole = make_step(P, b, V, compact=False, alpha=0.6, scope=0, n_min=2)
+    gw = torch.zeros_like(zs)
+    whole.run(zs, zt, gw)
+    parts, steps = [(0, 2), (2, 6)], []
+    for lo, hi in parts:
+        a, z = int(b.traj_offsets[lo]), int(b.traj_offsets[hi])
+        sub = W.Batch("part", b.turn_id[a:z], b.loss_mask[a:z], b.traj_offsets[lo:hi + 1] - a,
+                      b.max_turns)
+        steps.append((make_step(P, sub, V, compact=False, alpha=0.6, scope=0, n_min=2), a, z))
+    g_counts = sum(s.local_counts().clone() for s, _, _ in steps)
+    grads = []
+    for s, a, z in steps:
+        g = torch.zeros_like(zs[a:z])
+        s.run(zs[a:z], zt[a:z], g, global_counts=g_counts)
+        grads.append(g)
+    torch.cuda.synchronize()
+    assert whole.status() == 0 and all(s.status() == 0 for s, _, _ in steps)
+    assert torch.equal(torch.cat([s.w[:s.T] for s, _, _ in steps]), whole.w[:whole.T])
+    assert torch.equal(torch.cat(grads), gw)
+    loss = sum(s.loss.item() for s, _, _ in steps)
+    assert abs(loss - whole.loss.item()) <= 1e-12 * abs(whole.loss.item())
+    assert torch.equal(sum(s.turn_cnt for s, _, _ in steps), whole.turn_cnt)
+    assert torch.equal(sum(s.turn_surv for s, _, _ in steps), whole.turn_surv)
+    torch.testing.assert_close(sum(s.turn_sum for s, _, _ in steps), whole.turn_sum,
+                               rtol=1e-12, atol=1e-12)
