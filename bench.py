@@ -173,10 +173,10 @@ def build_inputs(args, rank, device):
 
 
 def run_step(step, zs, zt, grad, world, dist, ev_pair=None):
+    from paper_2607_05804_gb300 import dp
+
     if world > 1:
-        counts = step.local_counts().clone()
-        dist.all_reduce(counts)
-        step.weights(counts)
+        step.weights(dp.global_counts(step.local_counts()))
     else:
         step.weights()
     if ev_pair is not None:
@@ -186,7 +186,7 @@ def run_step(step, zs, zt, grad, world, dist, ev_pair=None):
         ev_pair[1].record()
     step.turn_stats()
     if world > 1:
-        dist.all_reduce(step.loss)
+        dp.reduce_step(step.loss, step.turn_sum, step.turn_cnt, step.turn_surv)
 
 
 def cpu_baseline(b, zs, zt, V, alpha, mode, rows_override=0, budget_s=15.0):
