@@ -183,6 +183,47 @@ turnopd_status turnopd_loss_fwd_bwd(const void *z_student, const void *z_teacher
 size_t turnopd_loss_workspace_bytes(int64_t num_tokens);
 
 /*
+ * turnopd_loss_fwd_bwd_static -- turnopd_loss_fwd_bwd for callers that cannot
+ * allocate device memory.  The paper has no counterpart: this is an addition
+ * of the library, not a step of the method.
+ *
+ * Who needs it: a caller whose device memory is owned by someone else -- a
+ * framework's caching allocator or a fixed arena that forbids raw cudaMalloc,
+ * a C host with no allocator of its own to hand out a workspace, or a
+ * latency-bound loop that must never reach cudaMalloc/cudaFree (cudaFree
+ * synchronises the whole device, and cudaMalloc can fail or stall once a pool
+ * has reserved the memory).  Such a caller still passes its inputs and
+ * outputs; only the scratch space moves into the library.
+ *
+ * Scratch: one file-scope device array of TURNOPD_STATIC_SCRATCH_BYTES,
+ * enough for TURNOPD_STATIC_MAX_TOKENS tokens.  Every GPU on which the
+ * library is loaded holds this array until the process exits.
+ * Limits: num_tokens > TURNOPD_STATIC_MAX_TOKENS returns TURNOPD_ERR_WORKSPACE
+ * before anything is launched.
+ * Set-up: the first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current).  Make that first call
+ * before any stream capture.
+ * Sharing: all calls use the one array.  Calls that can overlap on the GPU
+ * (different streams, or several host threads) race on it and may return
+ * wrong results: issue them on one stream.  The array keeps whatever the last
+ * call left there; nothing in it needs to start at zero, because every call
+ * writes each scratch word before reading it.
+ * Allocation: none -- no cudaMalloc, cudaFree or allocating library call.
+ * Arguments, outputs, errors and precision: as turnopd_loss_fwd_bwd, without
+ * the workspace arguments.
+ */
+#define TURNOPD_STATIC_MAX_TOKENS 65536
+#define TURNOPD_STATIC_SCRATCH_BYTES 1573632u
+turnopd_status turnopd_loss_fwd_bwd_static(const void *z_student, const void *z_teacher,
+                                           int32_t in_dtype, int64_t ld, int64_t vocab,
+                                           int64_t num_rows, const int32_t *row_of_token,
+                                           const int32_t *sampled_ids, const uint8_t *loss_mask,
+                                           const float *w, int64_t num_tokens, int32_t mode,
+                                           void *grad_student, int32_t grad_dtype, uint32_t flags,
+                                           float *token_loss_out, double *loss_out,
+                                           int32_t *dev_status, turnopd_stream_t stream);
+
+/*
  * turnopd_turn_stats -- turn statistics of the per-token losses
  * (Eq. observed-turn-kl: K_t is the mean per-token reverse KL over the
  * supervised tokens at turn t, over trajectories that reach t; the survivor

@@ -21,7 +21,8 @@ __all__ = [
     "TURNOPD_FORCE_PORTABLE", "TURNOPD_MAX_TURNS",
     "turnopd_turn_counts", "turnopd_weights", "turnopd_weights_workspace_bytes",
     "turnopd_loss_fwd_bwd", "turnopd_loss_workspace_bytes", "turnopd_turn_stats",
-    "turnopd_alpha_schedule", "turnopd_status_string",
+    "turnopd_alpha_schedule", "turnopd_status_string", "turnopd_loss_fwd_bwd_static",
+    "TURNOPD_STATIC_MAX_TOKENS",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -33,6 +34,7 @@ TURNOPD_SCOPE_TRAJ, TURNOPD_SCOPE_BATCH = 0, 1
 TURNOPD_ZERO_MASKED_GRAD = 0x1
 TURNOPD_FORCE_PORTABLE = 0x100
 TURNOPD_MAX_TURNS = 4096
+TURNOPD_STATIC_MAX_TOKENS = 65536
 
 STATUS_NAMES = {
     0: "TURNOPD_OK", 1: "TURNOPD_ERR_NULL", 2: "TURNOPD_ERR_SHAPE", 3: "TURNOPD_ERR_OFFSETS",
@@ -73,6 +75,8 @@ def load():
         "turnopd_loss_fwd_bwd": [P, P, i32, i64, i64, i64, P, P, P, P, i64, i32, P, i32, u32,
                                  P, P, P, sz, P, P],
         "turnopd_turn_stats": [P, P, P, P, i32, i64, i32, P, P, P, P, P, P, P],
+        "turnopd_loss_fwd_bwd_static": [P, P, i32, i64, i64, i64, P, P, P, P, i64, i32, P, i32,
+                                        u32, P, P, P, P],
     }
     for name, args in sig.items():
         fn = getattr(lib, name)
@@ -243,3 +247,38 @@ def turnopd_turn_stats(token_loss, turn_id, loss_mask, traj_offsets, max_turns, 
                                      _ptr(traj_turn_cnt), _ptr(turn_sum), _ptr(turn_cnt),
                                      _ptr(turn_surv), _ptr(dev_status), _stream(stream)),
            "turnopd_turn_stats")
+
+
+def turnopd_loss_fwd_bwd_static(z_student, z_teacher, vocab, row_of_token, sampled_ids, loss_mask,
+                                w, mode, grad_student, flags, token_loss_out, loss_out, dev_status,
+                                stream=None):
+    """turnopd_loss_fwd_bwd without a workspace argument, for callers that cannot
+    allocate device memory: the library's own static device scratch is used instead
+    (at most TURNOPD_STATIC_MAX_TOKENS tokens; calls must not overlap on the GPU)."""
+    import torch
+
+    T = loss_mask.numel()
+    for name, z in (("z_student", z_student), ("z_teacher", z_teacher)):
+        if not z.is_cuda or z.dim() != 2 or z.stride(1) != 1:
+            raise ValueError(f"{name} must be a 2-D CUDA tensor with unit column stride")
+    if z_teacher.shape != z_student.shape or z_teacher.stride() != z_student.stride() \
+            or z_teacher.dtype != z_student.dtype:
+        raise ValueError("z_teacher must match z_student in shape, stride and dtype")
+    ld = z_student.stride(0)
+    if grad_student is not None and (grad_student.shape != z_student.shape
+                                     or grad_student.stride(0) != ld or grad_student.stride(1) != 1
+                                     or not grad_student.is_cuda):
+        raise ValueError("grad_student must match z_student in shape and row stride")
+    _need(row_of_token, "row_of_token", torch.int32, T)
+    _need(sampled_ids, "sampled_ids", torch.int32, T)
+    _need(loss_mask, "loss_mask", torch.uint8)
+    _need(w, "w", torch.float32, T)
+    _need(token_loss_out, "token_loss_out", torch.float32, T)
+    _need(loss_out, "loss_out", torch.float64, 1)
+    _need(dev_status, "dev_status", torch.int32, 1)
+    gdt = _dtype_code(grad_student, "grad_student") if grad_student is not None else TURNOPD_F32
+    _check(load().turnopd_loss_fwd_bwd_static(
+        _ptr(z_student), _ptr(z_teacher), _dtype_code(z_student, "z_student"), ld, int(vocab),
+        z_student.shape[0], _ptr(row_of_token), _ptr(sampled_ids), _ptr(loss_mask), _ptr(w), T,
+        int(mode), _ptr(grad_student), gdt, int(flags), _ptr(token_loss_out), _ptr(loss_out),
+        _ptr(dev_status), _stream(stream)), "turnopd_loss_fwd_bwd_static")
