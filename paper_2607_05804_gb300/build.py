@@ -21,6 +21,8 @@ LIB = os.path.join(HERE, "libturnopd.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
          "-Xptxas", "-warn-spills"]
+# Extra nvcc flags (e.g. tuning macros such as -DTURNOPD_ROW_THREADS=384) for experiments.
+EXTRA = os.environ.get("TURNOPD_NVCC_FLAGS", "").split()
 
 
 def _nvcc():
@@ -51,7 +53,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
     try:
         def compile_one(src):
             obj = os.path.join(tmp, os.path.basename(src) + ".o")
-            cmd = [nvcc, *ARCH, *FLAGS, "-I", INCLUDE, "-I", CSRC, "-c", src, "-o", obj]
+            cmd = [nvcc, *ARCH, *FLAGS, *EXTRA, "-I", INCLUDE, "-I", CSRC, "-c", src, "-o", obj]
             r = subprocess.run(cmd, capture_output=True, text=True)
             if r.returncode != 0:
                 raise RuntimeError(f"nvcc failed on {src}:\n{r.stdout}\n{r.stderr}")

@@ -9,19 +9,23 @@
 //
 // Per CTA (persistent, one per SM, rows cid, cid + nclusters, ...):
 //   * thread 0 streams slices into a 3-stage ring with bulk asynchronous
-//     copies (cp.async.bulk, completion on an mbarrier, L2 evict-first);
-//   * stats(k+1): each thread takes the max over its vectors, then sums
-//     exp(z - m) for both models and A = sum exp(z_s - m_s)((z_s - z_t) - d);
-//     the CTA's partial goes to every CTA of the cluster through distributed
-//     shared memory (one 32-byte record per CTA per row);
-//   * barrier.cluster arrive, grad(k) from the resident slice of the previous
-//     row, barrier.cluster wait: the exchange latency of row k+1 hides behind
-//     the gradient pass of row k;
-//   * every CTA merges the CS records in rank order (identical arithmetic in
-//     every CTA, deterministic), so all slices use the same LSE and KL.
-// No CTA spins on another CTA's memory; the only waits are the hardware
-// cluster barrier (all CTAs of a cluster run the same row count) and
-// mbarrier waits on this CTA's own copies, bounded with an error status.
+//     copies (cp.async.bulk, completion on a "full" mbarrier, L2 evict-first);
+//     a stage is refilled once every warp has arrived on its "empty" mbarrier;
+//   * stats(k+1): per thread a max pass (packed bf16x2 max) and a sum pass
+//     (packed f32x2 arithmetic): S = sum exp(z - m) for both models and
+//     A = sum exp(z_s - m_s)((z_s - z_t) - d), d taken at the student's max.
+//     The CTA's partial is pushed to every CTA of the cluster with st.async
+//     into a 4-slot record ring; completion lands on the receiver's mbarrier
+//     (32 bytes per sender), so no cluster-wide barrier runs per row;
+//   * grad(k) from the resident slice of the previous row, overlapping the
+//     record exchange of row k+1;
+//   * every warp merges the CS records by the same fixed 8-lane tree, so all
+//     CTAs use bit-identical LSE and KL (deterministic).
+// Each thread reads its vectors of a row from shared memory twice: once into
+// registers for the maxima and sums, once for the gradient (3 exponentials
+// per element in all).
+// Waits are bounded: on timeout the kernel records TURNOPD_ERR_TIMEOUT, stops
+// computing and runs its remaining barriers without waiting, so it terminates.
 
 #include <algorithm>
 
@@ -32,7 +36,7 @@ namespace turnopd {
 namespace {
 
 constexpr int kStages = 3;
-constexpr uint32_t kCopyChunk = 16384;       // bytes per bulk copy instruction
+constexpr uint32_t kCopyChunk = 65536;       // bytes per bulk copy instruction
 constexpr uint32_t kWaitLimit = 1u << 22;    // mbarrier polls before giving up
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p)
@@ -61,19 +65,19 @@ __device__ __forceinline__ uint32_t cluster_count()
     return r;
 }
 
-__device__ __forceinline__ void cluster_arrive()
+__device__ __forceinline__ void cluster_sync()
 {
-    asm volatile("barrier.cluster.arrive.release;" ::: "memory");
-}
-
-__device__ __forceinline__ void cluster_wait()
-{
-    asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
+    asm volatile("barrier.cluster.arrive.release;\n\tbarrier.cluster.wait.acquire;" ::: "memory");
 }
 
 __device__ __forceinline__ void mbar_init(uint64_t *bar, uint32_t count)
 {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *bar)
+{
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t bytes)
@@ -83,12 +87,27 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *bar, uint32_t by
                  : "memory");
 }
 
+// Wait on a barrier completed by this CTA's threads or its own bulk copies.
 __device__ __forceinline__ bool mbar_try_wait(uint64_t *bar, uint32_t parity)
 {
     uint32_t ok;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(bar)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait on a barrier completed by other CTAs' st.async records.
+__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t *bar, uint32_t parity)
+{
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
         : "r"(smem_u32(bar)), "r"(parity)
@@ -113,64 +132,165 @@ __device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t by
         : "memory");
 }
 
-// Store 16 bytes into the shared memory of CTA `rank` of this cluster at the
-// address that `local` has in this CTA.
-__device__ __forceinline__ void st_cluster(const void *local, uint32_t rank, float4 v)
+__device__ __forceinline__ uint32_t mapa(uint32_t addr, uint32_t rank)
 {
-    uint32_t raddr;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(raddr) : "r"(smem_u32(local)), "r"(rank));
-    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(raddr), "f"(v.x), "f"(v.y),
-                 "f"(v.z), "f"(v.w)
-                 : "memory");
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(addr), "r"(rank));
+    return r;
 }
 
-__device__ __forceinline__ void unpack8(const uint4 u, float *x)
+// 16 bytes into another CTA's shared memory; completion counted on its mbarrier.
+__device__ __forceinline__ void st_async16(uint32_t raddr, uint32_t rbar, float4 v)
 {
-    x[0] = bf16lo(u.x), x[1] = bf16hi(u.x), x[2] = bf16lo(u.y), x[3] = bf16hi(u.y);
-    x[4] = bf16lo(u.z), x[5] = bf16hi(u.z), x[6] = bf16lo(u.w), x[7] = bf16hi(u.w);
+    asm volatile(
+        "st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.f32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+            raddr),
+        "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w), "r"(rbar)
+        : "memory");
 }
 
-struct Smem {
-    unsigned char *stage;  // kStages x [zs slice | zt slice]
-    float *rec;            // [2 slots][CS][8]
-    int4 *meta;            // [kStages] row records
-    uint64_t *full;        // [kStages] mbarriers
-    float *red;            // [warps][8]
-};
+// ---- packed f32x2 arithmetic (two fp32 lanes per instruction) -----------
 
-template <int CS, int NT, int VPT, bool G32>
-__global__ void __launch_bounds__(NT, 1) k_row_cluster(RowIn p, int slice_vec, int nvec)
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c)
 {
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+        "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+    return d;
+}
+
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b)
+{
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+
+__device__ __forceinline__ float2 fsub2(float2 a, float2 b)
+{
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "sub.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b)
+{
+    float2 d;
+    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+        "mul.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
+        : "=f"(d.x), "=f"(d.y)
+        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+    return d;
+}
+
+__device__ __forceinline__ float2 unpack2(uint32_t u) { return make_float2(bf16lo(u), bf16hi(u)); }
+__device__ __forceinline__ float2 splat(float x) { return make_float2(x, x); }
+__device__ __forceinline__ float2 ex2x2(float2 x) { return make_float2(ex2(x.x), ex2(x.y)); }
+
+__device__ __forceinline__ uint32_t hmax2u(uint32_t a, uint32_t b)
+{
+    uint32_t d;
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
+    return d;
+}
+
+__device__ __forceinline__ uint32_t word(const uint4 &v, int j)
+{
+    return j == 0 ? v.x : (j == 1 ? v.y : (j == 2 ? v.z : v.w));
+}
+
+// Merge per-lane partial statistics across the first `width` lanes of a warp
+// (lanes beyond hold empty partials): exact max by butterfly, one rescale
+// exponential per lane, then butterfly sums.  Lane 0's result is used; its
+// association order is fixed, so every warp and CTA gets the same bits.
+template <int WIDTH>
+__device__ __forceinline__ void lane_merge(Student &S, Teacher &T)
+{
+    float m = S.m, mt = T.m;
+#pragma unroll
+    for (int o = 1; o < WIDTH; o <<= 1) {
+        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
+    }
+    // reference difference of the lowest lane holding the max
+    const unsigned own = __ballot_sync(0xffffffffu, S.m == m && m != -INFINITY);
+    const int src = own ? __ffs(own) - 1 : 0;
+    const float d = __shfl_sync(0xffffffffu, S.d, src);
+    const float f = m == -INFINITY ? 0.f : ex2((S.m - m) * kLog2e);
+    const float ft = mt == -INFINITY ? 0.f : ex2((T.m - mt) * kLog2e);
+    float s = S.s * f, a = fmaf(S.s, S.d - d, S.a) * f, t = T.s * ft;
+    if (S.m == -INFINITY)
+        s = 0.f, a = 0.f;
+    if (T.m == -INFINITY)
+        t = 0.f;
+#pragma unroll
+    for (int o = 1; o < WIDTH; o <<= 1) {
+        s += __shfl_xor_sync(0xffffffffu, s, o);
+        a += __shfl_xor_sync(0xffffffffu, a, o);
+        t += __shfl_xor_sync(0xffffffffu, t, o);
+    }
+    S = Student{m, s, a, d};
+    T = Teacher{mt, t};
+}
+
+// G groups of NT threads per CTA take the rows of the cluster in turn (row k
+// to group k % G).  Record slots: 2G, so a slot is reused by the same group
+// two rows later, after that group has read it (a peer can run at most G rows
+// ahead of the slowest CTA in sending records).
+template <int CS, int NT, int VPT, int G, bool G32>
+__global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_vec, int nvec)
+{
+    constexpr int kSlots = 2 * G;
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ int s_dead;
-    constexpr int NW = NT / 32;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    constexpr int NWG = NT / 32;  // warps per group
+    const int tid = threadIdx.x, lane = tid & 31;
+    const int group = tid / NT, gtid = tid % NT, gwarp = gtid >> 5;
     const uint32_t rank = cluster_ctarank();
     const int cid = (int)cluster_id(), ncl = (int)cluster_count();
     const uint32_t slice_bytes = (uint32_t)slice_vec * 16u;
     const uint32_t stage_bytes = 2u * slice_bytes;
-    const int v0 = (int)rank * slice_vec;                       // first vector of my slice
+    const int v0 = (int)rank * slice_vec;  // first vector of my slice
     const int my_vec = max(0, min(slice_vec, nvec - v0));
     const uint32_t my_bytes = (uint32_t)my_vec * 16u;
 
-    Smem sm;
-    sm.stage = smem;
-    sm.rec = reinterpret_cast<float *>(smem + kStages * stage_bytes);
-    sm.meta = reinterpret_cast<int4 *>(sm.rec + 2 * CS * 8);
-    sm.full = reinterpret_cast<uint64_t *>(sm.meta + kStages);
-    sm.red = reinterpret_cast<float *>(sm.full + kStages);
+    unsigned char *stage = smem;
+    float *rec = reinterpret_cast<float *>(smem + kStages * stage_bytes);  // [kSlots][CS][8]
+    int4 *meta = reinterpret_cast<int4 *>(rec + kSlots * CS * 8);          // [kStages]
+    uint64_t *full = reinterpret_cast<uint64_t *>(meta + kStages);         // [kStages]
+    uint64_t *empty = full + kStages;                                      // [kStages]
+    uint64_t *recv = empty + kStages;                                      // [kSlots]
+    float *red = reinterpret_cast<float *>(recv + kSlots);                 // [G][NWG][8]
+    int *srow = reinterpret_cast<int *>(red + G * NWG * 8);                // [kStages] row in stage
 
     if (tid == 0) {
         s_dead = 0;
-        for (int s = 0; s < kStages; ++s)
-            mbar_init(&sm.full[s], 1);
+        for (int s = 0; s < kStages; ++s) {
+            mbar_init(&full[s], 1);
+            mbar_init(&empty[s], NWG);
+            srow[s] = -1;
+        }
+        for (int s = 0; s < kSlots; ++s)
+            mbar_init(&recv[s], 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        for (int s = 0; s < kSlots; ++s)
+            mbar_arrive_expect_tx(&recv[s], CS * 32u);  // first record of each slot
     }
     __syncthreads();
-    // every CTA of the cluster is resident before any distributed-shared write
-    cluster_arrive();
-    cluster_wait();
+    cluster_sync();  // peers' barriers are initialised before any record is sent
 
     const int nvalid = *p.nvalid;
     const int n = nvalid > cid ? (nvalid - cid + ncl - 1) / ncl : 0;  // same for the whole cluster
@@ -179,125 +299,183 @@ __global__ void __launch_bounds__(NT, 1) k_row_cluster(RowIn p, int slice_vec, i
 
     const __nv_bfloat16 *zs = static_cast<const __nv_bfloat16 *>(p.zs);
     const __nv_bfloat16 *zt = static_cast<const __nv_bfloat16 *>(p.zt);
-    const uint64_t pol = evict_first_policy();
 
-    // thread 0: stream row k of this cluster into stage k % kStages
-    auto issue = [&](int k, int4 m) {
-        const int s = k % kStages;
-        sm.meta[s] = m;
-        const size_t off = (size_t)m.y * (size_t)p.ld + (size_t)v0 * 8;
-        const char *gs = reinterpret_cast<const char *>(zs + off);
-        const char *gt = reinterpret_cast<const char *>(zt + off);
-        unsigned char *ds = sm.stage + s * stage_bytes;
-        mbar_arrive_expect_tx(&sm.full[s], 2u * my_bytes);
-        for (uint32_t o = 0; o < my_bytes; o += kCopyChunk) {
-            const uint32_t sz = min(kCopyChunk, my_bytes - o);
-            bulk_g2s(ds + o, gs + o, sz, &sm.full[s], pol);
-            bulk_g2s(ds + slice_bytes + o, gt + o, sz, &sm.full[s], pol);
-        }
-    };
-
-    auto wait_full = [&](int k) {
-        const int s = k % kStages;
-        const uint32_t parity = (uint32_t)((k / kStages) & 1);
-        if (*(volatile int *)&s_dead)
+    auto dead = [&]() { return *(volatile int *)&s_dead != 0; };
+    auto wait_bar = [&](uint64_t *bar, uint32_t parity, bool cluster_scope) {
+        if (dead())
             return;
         for (uint32_t it = 0; it < kWaitLimit; ++it)
-            if (mbar_try_wait(&sm.full[s], parity))
+            if (cluster_scope ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity))
                 return;
         s_dead = 1;
         set_status(p.status, TURNOPD_ERR_TIMEOUT);
     };
+    auto group_sync = [&]() { asm volatile("bar.sync %0, %1;" ::"r"(1 + group), "r"(NT) : "memory"); };
 
-    // statistics of the resident slice of row k -> record into every CTA's slot k & 1
-    auto stats = [&](int k) {
+    // Data of row k: wait until the stage has been armed for row k, then for
+    // its phase.  (A parity wait alone would also accept the phase of the
+    // stage's previous row, k - kStages, when a group reaches row k early.)
+    auto wait_full = [&](int k) {
         const int s = k % kStages;
-        const uint4 *vs = reinterpret_cast<const uint4 *>(sm.stage + s * stage_bytes);
-        const uint4 *vt = reinterpret_cast<const uint4 *>(sm.stage + s * stage_bytes + slice_bytes);
-        float ms = -INFINITY, xd = 0.f, mt = -INFINITY;
-#pragma unroll
-        for (int u = 0; u < VPT; ++u) {
-            const int q = tid + u * NT;
-            if (q < my_vec) {
-                float a[8], b[8];
-                unpack8(vs[q], a);
-                unpack8(vt[q], b);
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    if (a[e] > ms) {
-                        ms = a[e];
-                        xd = a[e] - b[e];
-                    }
-                    mt = fmaxf(mt, b[e]);
-                }
-            }
+        if (dead())
+            return;
+        uint32_t it = 0;
+        while (*(volatile int *)&srow[s] != k && ++it < kWaitLimit) {
         }
-        const float ns = -ms * kLog2e, nt = -mt * kLog2e;
-        float ss = 0.f, aa = 0.f, st = 0.f;
-#pragma unroll
-        for (int u = 0; u < VPT; ++u) {
-            const int q = tid + u * NT;
-            if (q < my_vec) {
-                float a[8], b[8];
-                unpack8(vs[q], a);
-                unpack8(vt[q], b);
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float es = ex2(fmaf(a[e], kLog2e, ns));
-                    ss += es;
-                    aa = fmaf(es, (a[e] - b[e]) - xd, aa);
-                    st += ex2(fmaf(b[e], kLog2e, nt));
-                }
-            }
+        if (it >= kWaitLimit) {
+            s_dead = 1;
+            set_status(p.status, TURNOPD_ERR_TIMEOUT);
+            return;
         }
-        Student S = ms == -INFINITY ? student_empty() : Student{ms, ss, aa, xd};
-        Teacher U = mt == -INFINITY ? teacher_empty() : Teacher{mt, st};
-        S = warp_merge(S);
-        U = warp_merge(U);
-        if (lane == 0) {
-            float *r = sm.red + warp * 8;
-            r[0] = S.m, r[1] = S.s, r[2] = S.a, r[3] = S.d, r[4] = U.m, r[5] = U.s;
-        }
-        __syncthreads();
-        if (warp == 0 && lane < CS) {
-            Student A = Student{sm.red[0], sm.red[1], sm.red[2], sm.red[3]};
-            Teacher B = Teacher{sm.red[4], sm.red[5]};
-            for (int w2 = 1; w2 < NW; ++w2) {
-                const float *r = sm.red + w2 * 8;
-                A = student_merge(A, Student{r[0], r[1], r[2], r[3]});
-                B = teacher_merge(B, Teacher{r[4], r[5]});
-            }
-            // sampled-token logits, from the CTA whose slice holds y
-            float ys = 0.f, yt = 0.f;
-            const int y = sm.meta[s].z;
-            if (y >= 0 && y / 8 >= v0 && y / 8 < v0 + my_vec) {
-                const int e = y - v0 * 8;
-                ys = to_float(reinterpret_cast<const __nv_bfloat16 *>(vs)[e]);
-                yt = to_float(reinterpret_cast<const __nv_bfloat16 *>(vt)[e]);
-            }
-            float *slot = sm.rec + ((k & 1) * CS + (int)rank) * 8;
-            st_cluster(slot, (uint32_t)lane, make_float4(A.m, A.s, A.a, A.d));
-            st_cluster(slot + 4, (uint32_t)lane, make_float4(B.m, B.s, ys, yt));
+        wait_bar(&full[s], (uint32_t)((k / kStages) & 1), false);
+    };
+
+    // stream row k of this cluster into stage k % kStages (after the stage's
+    // previous row is done with it)
+    auto issue = [&](int k, int4 m) {
+        const int s = k % kStages;
+        meta[s] = m;
+        *(volatile int *)&srow[s] = k;
+        const size_t off = (size_t)m.y * (size_t)p.ld + (size_t)v0 * 8;
+        const char *gs = reinterpret_cast<const char *>(zs + off);
+        const char *gt = reinterpret_cast<const char *>(zt + off);
+        unsigned char *ds = stage + s * stage_bytes;
+        const uint64_t pol = evict_first_policy();
+        mbar_arrive_expect_tx(&full[s], 2u * my_bytes);
+        for (uint32_t o = 0; o < my_bytes; o += kCopyChunk) {
+            const uint32_t sz = min(kCopyChunk, my_bytes - o);
+            bulk_g2s(ds + o, gs + o, sz, &full[s], pol);
+            bulk_g2s(ds + slice_bytes + o, gt + o, sz, &full[s], pol);
         }
     };
 
-    // row constants of row k from the CS records (same order in every CTA)
-    auto combine = [&](int k, float &ell) {
-        const float *slot = sm.rec + (k & 1) * CS * 8;
-        Student A = Student{slot[0], slot[1], slot[2], slot[3]};
-        Teacher B = Teacher{slot[4], slot[5]};
+    // statistics of row k: this CTA's record into slot k % kSlots of every CTA
+    auto stats = [&](int k) {
+        const int s = k % kStages;
+        const uint4 *vs = reinterpret_cast<const uint4 *>(stage + s * stage_bytes);
+        const uint4 *vt = reinterpret_cast<const uint4 *>(stage + s * stage_bytes + slice_bytes);
+        // max pass (packed bf16); remember the vector holding the student max
+        uint32_t tmax = 0xff80ff80u;  // (-inf, -inf)
+        float best = -INFINITY;
+        int bq = -1;
 #pragma unroll
-        for (int c = 1; c < CS; ++c) {
-            const float *r = slot + c * 8;
-            A = student_merge(A, Student{r[0], r[1], r[2], r[3]});
-            B = teacher_merge(B, Teacher{r[4], r[5]});
+        for (int u = 0; u < VPT; ++u) {
+            const int q = gtid + u * NT;
+            if (q < my_vec) {
+                const uint4 a = vs[q], b = vt[q];
+                const uint32_t m = hmax2u(hmax2u(a.x, a.y), hmax2u(a.z, a.w));
+                const float v = fmaxf(bf16lo(m), bf16hi(m));
+                if (v > best) {
+                    best = v;
+                    bq = q;
+                }
+                tmax = hmax2u(tmax, hmax2u(hmax2u(b.x, b.y), hmax2u(b.z, b.w)));
+            }
         }
+        const float ms = best, mt = fmaxf(bf16lo(tmax), bf16hi(tmax));
+        float xd = 0.f;
+        if (bq >= 0) {  // reference difference at the first element equal to the max
+            const uint4 a = vs[bq], b = vt[bq];
+            bool found = false;
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const float2 x = unpack2(word(a, j)), y = unpack2(word(b, j));
+                if (!found && x.x == ms) {
+                    xd = x.x - y.x;
+                    found = true;
+                }
+                if (!found && x.y == ms) {
+                    xd = x.y - y.y;
+                    found = true;
+                }
+            }
+        }
+        // sum pass (packed pairs)
+        const float2 L2 = splat(kLog2e), NS = splat(-ms * kLog2e), NTT = splat(-mt * kLog2e);
+        const float2 D = splat(xd);
+        float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
+#pragma unroll
+        for (int u = 0; u < VPT; ++u) {
+            const int q = gtid + u * NT;
+            if (q < my_vec) {
+                const uint4 a = vs[q], b = vt[q];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float2 a2 = unpack2(word(a, j)), b2 = unpack2(word(b, j));
+                    const float2 es = ex2x2(ffma2(a2, L2, NS));
+                    S2 = fadd2(S2, es);
+                    A2 = ffma2(es, fsub2(fsub2(a2, b2), D), A2);
+                    T2 = fadd2(T2, ex2x2(ffma2(b2, L2, NTT)));
+                }
+            }
+        }
+        Student S = ms == -INFINITY ? student_empty() : Student{ms, S2.x + S2.y, A2.x + A2.y, xd};
+        Teacher U = mt == -INFINITY ? teacher_empty() : Teacher{mt, T2.x + T2.y};
+        lane_merge<32>(S, U);
+        float *rg = red + group * NWG * 8;
+        if (lane == 0) {
+            float *rw = rg + gwarp * 8;
+            rw[0] = S.m, rw[1] = S.s, rw[2] = S.a, rw[3] = S.d, rw[4] = U.m, rw[5] = U.s;
+        }
+        group_sync();
+        if (gwarp == 0) {
+            Student A = student_empty();
+            Teacher B = teacher_empty();
+            if (lane < NWG) {
+                const float *r = rg + lane * 8;
+                A = Student{r[0], r[1], r[2], r[3]};
+                B = Teacher{r[4], r[5]};
+            }
+            lane_merge<NWG>(A, B);
+            A.m = __shfl_sync(0xffffffffu, A.m, 0);
+            A.s = __shfl_sync(0xffffffffu, A.s, 0);
+            A.a = __shfl_sync(0xffffffffu, A.a, 0);
+            A.d = __shfl_sync(0xffffffffu, A.d, 0);
+            B.m = __shfl_sync(0xffffffffu, B.m, 0);
+            B.s = __shfl_sync(0xffffffffu, B.s, 0);
+            if (lane < CS) {
+                float ys = 0.f, yt = 0.f;  // sampled-token logits, from the CTA holding y
+                const int y = meta[s].z;
+                if (y >= 0 && y / 8 >= v0 && y / 8 < v0 + my_vec) {
+                    const int e = y - v0 * 8;
+                    ys = to_float(reinterpret_cast<const __nv_bfloat16 *>(vs)[e]);
+                    yt = to_float(reinterpret_cast<const __nv_bfloat16 *>(vt)[e]);
+                }
+                const int slot = k % kSlots;
+                const uint32_t ra = mapa(smem_u32(rec + (slot * CS + (int)rank) * 8), (uint32_t)lane);
+                const uint32_t rbar = mapa(smem_u32(&recv[slot]), (uint32_t)lane);
+                st_async16(ra, rbar, make_float4(A.m, A.s, A.a, A.d));
+                st_async16(ra + 16, rbar, make_float4(B.m, B.s, ys, yt));
+            }
+        }
+    };
+
+    // row constants of row k from the CS records (identical in every warp/CTA)
+    auto combine = [&](int k, float &ell) {
+        const int slot = k % kSlots;
+        wait_bar(&recv[slot], (uint32_t)((k / kSlots) & 1), true);
+        const float *r = rec + slot * CS * 8;
+        Student A = student_empty();
+        Teacher B = teacher_empty();
+        if (lane < CS) {
+            const float4 x = *reinterpret_cast<const float4 *>(r + lane * 8);
+            const float4 y = *reinterpret_cast<const float4 *>(r + lane * 8 + 4);
+            A = Student{x.x, x.y, x.z, x.w};
+            B = Teacher{y.x, y.y};
+        }
+        lane_merge<CS>(A, B);
+        A.m = __shfl_sync(0xffffffffu, A.m, 0);
+        A.s = __shfl_sync(0xffffffffu, A.s, 0);
+        A.a = __shfl_sync(0xffffffffu, A.a, 0);
+        A.d = __shfl_sync(0xffffffffu, A.d, 0);
+        B.m = __shfl_sync(0xffffffffu, B.m, 0);
+        B.s = __shfl_sync(0xffffffffu, B.s, 0);
         const RowConst rc = row_const(A, B);
         ell = rc.kl;
-        const int y = sm.meta[k % kStages].z;
+        const int y = meta[k % kStages].z;
         if (y >= 0) {
             const int owner = (y / 8) / slice_vec;
-            ell = (slot[owner * 8 + 6] - slot[owner * 8 + 7]) - rc.dl;
+            ell = (r[owner * 8 + 6] - r[owner * 8 + 7]) - rc.dl;
         }
         return rc;
     };
@@ -306,39 +484,52 @@ __global__ void __launch_bounds__(NT, 1) k_row_cluster(RowIn p, int slice_vec, i
         if (!p.grad)
             return;
         const int s = k % kStages;
-        const int4 m = sm.meta[s];
-        const uint4 *vs = reinterpret_cast<const uint4 *>(sm.stage + s * stage_bytes);
-        const uint4 *vt = reinterpret_cast<const uint4 *>(sm.stage + s * stage_bytes + slice_bytes);
+        const int4 m = meta[s];
+        const uint4 *vs = reinterpret_cast<const uint4 *>(stage + s * stage_bytes);
+        const uint4 *vt = reinterpret_cast<const uint4 *>(stage + s * stage_bytes + slice_bytes);
         const float wi = __int_as_float(m.w), wl = wi * ell;
-        const float nl = -rc.lse_s * kLog2e, d = rc.d, cp = rc.cp;
         const int y = m.z;
         const size_t row_off = (size_t)m.y * (size_t)p.ld + (size_t)v0 * 8;
+        const float2 L2 = splat(kLog2e), D = splat(rc.d), CP = splat(rc.cp);
+        const float2 NL = splat(-rc.lse_s * kLog2e);
+        const float2 W = splat(wi), NWL = splat(-wl);
 #pragma unroll
         for (int u = 0; u < VPT; ++u) {
-            const int q = tid + u * NT;
+            const int q = gtid + u * NT;
             if (q < my_vec) {
-                float a[8], b[8], g[8];
-                unpack8(vs[q], a);
-                unpack8(vt[q], b);
+                float2 g[4];
+                if (y < 0) {  // full vocabulary: g = w p ((z_s - z_t) - d - cp)
+                    const uint4 a = vs[q], b = vt[q];
 #pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float pv = ex2(fmaf(a[e], kLog2e, nl));
-                    if (y < 0)
-                        g[e] = wi * pv * (((a[e] - b[e]) - d) - cp);
-                    else
-                        g[e] = ((v0 + q) * 8 + e == y ? wl : 0.f) - wl * pv;
+                    for (int j = 0; j < 4; ++j) {
+                        const float2 a2 = unpack2(word(a, j)), b2 = unpack2(word(b, j));
+                        const float2 pv = ex2x2(ffma2(a2, L2, NL));
+                        g[j] = fmul2(fmul2(pv, W), fsub2(fsub2(fsub2(a2, b2), D), CP));
+                    }
+                } else {  // sampled token: g = w l (e_y - p)
+                    const uint4 a = vs[q];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const float2 pv = ex2x2(ffma2(unpack2(word(a, j)), L2, NL));
+                        g[j] = fmul2(pv, NWL);
+                        const int e = ((v0 + q) * 8 + 2 * j) - y;
+                        if (e == 0)
+                            g[j].x += wl;
+                        else if (e == -1)
+                            g[j].y += wl;
+                    }
                 }
                 if (G32) {
                     float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(p.grad) + row_off +
                                                              (size_t)q * 8);
-                    __stcs(dst, make_float4(g[0], g[1], g[2], g[3]));
-                    __stcs(dst + 1, make_float4(g[4], g[5], g[6], g[7]));
+                    __stcs(dst, make_float4(g[0].x, g[0].y, g[1].x, g[1].y));
+                    __stcs(dst + 1, make_float4(g[2].x, g[2].y, g[3].x, g[3].y));
                 } else {
                     uint4 o;
-                    o.x = pack_bf16x2(g[0], g[1]);
-                    o.y = pack_bf16x2(g[2], g[3]);
-                    o.z = pack_bf16x2(g[4], g[5]);
-                    o.w = pack_bf16x2(g[6], g[7]);
+                    o.x = pack_bf16x2(g[0].x, g[0].y);
+                    o.y = pack_bf16x2(g[1].x, g[1].y);
+                    o.z = pack_bf16x2(g[2].x, g[2].y);
+                    o.w = pack_bf16x2(g[3].x, g[3].y);
                     __stcs(reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.grad) + row_off +
                                                      (size_t)q * 8),
                            o);
@@ -347,66 +538,76 @@ __global__ void __launch_bounds__(NT, 1) k_row_cluster(RowIn p, int slice_vec, i
         }
     };
 
-    // prologue: rows 0..2 in flight, statistics of row 0 exchanged
+    // The groups take rows in turn: while one waits for its row's records or
+    // data, the others compute.
     if (tid == 0)
         for (int k = 0; k < kStages && k < n; ++k)
             issue(k, p.rows[cid + k * ncl]);
-    wait_full(0);
-    stats(0);
-    cluster_arrive();
-    cluster_wait();
-
-    for (int k = 0; k < n; ++k) {
+    for (int k = group; k < n; k += G) {
         int4 ahead = make_int4(0, 0, -1, 0);
-        if (tid == 0 && k + kStages < n)
-            ahead = p.rows[cid + (k + kStages) * ncl];  // consumed at the end of this iteration
+        if (gtid == 0 && k + kStages < n)
+            ahead = p.rows[cid + (k + kStages) * ncl];  // used at the end of the iteration
+        wait_full(k);
+        stats(k);
         float ell;
         const RowConst rc = combine(k, ell);
-        if (rank == 0 && tid == 0) {
-            const int4 m = sm.meta[k % kStages];
+        if (gtid == 0)
+            mbar_arrive_expect_tx(&recv[k % kSlots], CS * 32u);  // re-arm for row k + kSlots
+        if (rank == 0 && gtid == 0) {
+            const int4 m = meta[k % kStages];
             if (!isfinite(rc.lse_s) || !isfinite(rc.lse_t) || !isfinite(ell))
                 set_status(p.status, TURNOPD_ERR_NONFINITE);
             p.token_loss[m.x] = ell;
             p.row_wl[cid + k * ncl] = (double)__int_as_float(m.w) * (double)ell;
         }
-        if (k + 1 < n) {
-            wait_full(k + 1);
-            stats(k + 1);
-        }
-        cluster_arrive();
-        grad(k, rc, ell);
-        cluster_wait();
-        __syncthreads();  // every thread is done with stage k % kStages
-        if (tid == 0 && k + kStages < n) {
+        if (!dead())
+            grad(k, rc, ell);
+        __syncwarp();
+        if (lane == 0)
+            mbar_arrive(&empty[k % kStages]);
+        if (gtid == 0 && k + kStages < n) {
+            wait_bar(&empty[k % kStages], (uint32_t)((k / kStages) & 1), false);
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             issue(k + kStages, ahead);
         }
     }
 
-    // after a timeout, let this CTA's own copies land before the CTA exits
-    if (tid == 0 && s_dead) {
+    // after a timeout, let this CTA's own copies land before it exits
+    if (tid == 0 && dead()) {
         for (int k = max(0, n - kStages); k < n; ++k)
             for (uint32_t it = 0; it < kWaitLimit; ++it)
-                if (mbar_try_wait(&sm.full[k % kStages], (uint32_t)((k / kStages) & 1)))
+                if (mbar_try_wait(&full[k % kStages], (uint32_t)((k / kStages) & 1)))
                     break;
     }
+    cluster_sync();  // no CTA leaves while a peer may still address its shared memory
 }
 
+// Threads per row group and groups per CTA (tuning knobs).
+#ifndef TURNOPD_ROW_THREADS
+#define TURNOPD_ROW_THREADS 384
+#endif
+#ifndef TURNOPD_ROW_GROUPS
+#define TURNOPD_ROW_GROUPS 2
+#endif
 constexpr int kCS = 8;
-constexpr int kNT = 256;
-constexpr int kVPT = 10;
+constexpr int kNT = TURNOPD_ROW_THREADS;
+constexpr int kG = TURNOPD_ROW_GROUPS;
+constexpr int kMaxSlice = 2400;                      // vectors per CTA: 3 stages fit 227 KB
+constexpr int kVPT = (kMaxSlice + kNT - 1) / kNT;    // vectors per thread
 constexpr int64_t kMinVocab = 32768;  // below this the portable kernel is faster
 
 size_t cluster_smem_bytes(int slice_vec)
 {
-    return (size_t)kStages * 2 * slice_vec * 16 + 2 * kCS * 8 * sizeof(float) +
-           kStages * sizeof(int4) + kStages * sizeof(uint64_t) + (kNT / 32) * 8 * sizeof(float);
+    return (size_t)kStages * 2 * slice_vec * 16 + 2 * kG * kCS * 8 * sizeof(float) +
+           kStages * sizeof(int4) + (2 * kStages + 2 * kG) * sizeof(uint64_t) +
+           kG * (kNT / 32) * 8 * sizeof(float) +  // per-group warp partials
+           kStages * sizeof(int);                   // row held by each stage
 }
 
 template <bool G32>
 cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaStream_t stream)
 {
-    auto kern = k_row_cluster<kCS, kNT, kVPT, G32>;
+    auto kern = k_row_cluster<kCS, kNT, kVPT, kG, G32>;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess)
@@ -431,7 +632,7 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    cfg.blockDim = dim3(kNT);
+    cfg.blockDim = dim3(kG * kNT);
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     if (grid_cache[dev][gi] == 0) {
@@ -459,7 +660,7 @@ cudaError_t launch_row_cluster(const RowIn &p, bool fp32_grad, cudaStream_t stre
         return cudaSuccess;
     const int nvec = (int)(p.vocab / 8);
     const int slice_vec = (nvec + kCS - 1) / kCS;
-    if (slice_vec > kVPT * kNT)
+    if (slice_vec > kMaxSlice)
         return cudaSuccess;
     const size_t smem = cluster_smem_bytes(slice_vec);
     int dev = 0, optin = 0;
@@ -469,8 +670,7 @@ cudaError_t launch_row_cluster(const RowIn &p, bool fp32_grad, cudaStream_t stre
     e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
     if (e != cudaSuccess)
         return e;
-    // leave room for the kernel's static shared memory
-    if (smem + 64 > (size_t)optin)
+    if (smem + 64 > (size_t)optin)  // room for the kernel's static shared memory
         return cudaSuccess;
     *used = true;
     return fp32_grad ? launch_t<true>(p, slice_vec, nvec, smem, stream)
