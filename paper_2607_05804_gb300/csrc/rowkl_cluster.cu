@@ -150,49 +150,14 @@ __device__ __forceinline__ void st_async16(uint32_t raddr, uint32_t rbar, float4
 }
 
 // ---- packed f32x2 arithmetic (two fp32 lanes per instruction) -----------
+// The sm_100-family paired-fp32 builtins; subtraction as an exact fma by -1.
 
-__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c)
-{
-    float2 d;
-    asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
-        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
-        "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-        : "=f"(d.x), "=f"(d.y)
-        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
-    return d;
-}
-
-__device__ __forceinline__ float2 fadd2(float2 a, float2 b)
-{
-    float2 d;
-    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
-        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
-        "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-        : "=f"(d.x), "=f"(d.y)
-        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-    return d;
-}
-
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) { return __fadd2_rn(a, b); }
+__device__ __forceinline__ float2 fmul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
 __device__ __forceinline__ float2 fsub2(float2 a, float2 b)
 {
-    float2 d;
-    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
-        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
-        "sub.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-        : "=f"(d.x), "=f"(d.y)
-        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-    return d;
-}
-
-__device__ __forceinline__ float2 fmul2(float2 a, float2 b)
-{
-    float2 d;
-    asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
-        "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
-        "mul.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n\t}"
-        : "=f"(d.x), "=f"(d.y)
-        : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
-    return d;
+    return __ffma2_rn(b, make_float2(-1.f, -1.f), a);
 }
 
 __device__ __forceinline__ float2 unpack2(uint32_t u) { return make_float2(bf16lo(u), bf16hi(u)); }
@@ -245,6 +210,17 @@ __device__ __forceinline__ void lane_merge(Student &S, Teacher &T)
     T = Teacher{mt, t};
 }
 
+// Per-row constants the gradient pass needs (computed once per row).
+struct GradConst {
+    float lse_s, lse_t, kl;
+    float nlw;        // -LSE_s log2e + log2 |w| (full) or log2 |w l| (sampled)
+    float sg;         // sign of w
+    float nd, ncp;    // -sg d, -sg cp
+    float nc;         // -sg (d + cp)
+    float sgl;        // sign of -w l (sampled)
+    float wl;         // w l
+};
+
 // G groups of NT threads per CTA take the rows of the cluster in turn (row k
 // to group k % G).  Record slots: 2G, so a slot is reused by the same group
 // two rows later, after that group has read it (a peer can run at most G rows
@@ -274,6 +250,7 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
     uint64_t *recv = empty + kStages;                                      // [kSlots]
     float *red = reinterpret_cast<float *>(recv + kSlots);                 // [G][NWG][8]
     int *srow = reinterpret_cast<int *>(red + G * NWG * 8);                // [kStages] row in stage
+    float *rcs = reinterpret_cast<float *>(srow + 4);                       // [G][16] row constants
 
     if (tid == 0) {
         s_dead = 0;
@@ -354,27 +331,30 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
         const int s = k % kStages;
         const uint4 *vs = reinterpret_cast<const uint4 *>(stage + s * stage_bytes);
         const uint4 *vt = reinterpret_cast<const uint4 *>(stage + s * stage_bytes + slice_bytes);
-        // max pass (packed bf16); remember the vector holding the student max
-        uint32_t tmax = 0xff80ff80u;  // (-inf, -inf)
-        float best = -INFINITY;
-        int bq = -1;
+        // max pass (packed bf16): running maxima, plus each vector's student
+        // maximum kept packed so the argmax vector is found after the loop
+        uint32_t smax = 0xff80ff80u, tmax = 0xff80ff80u;  // (-inf, -inf)
+        uint32_t vmax[VPT];
 #pragma unroll
         for (int u = 0; u < VPT; ++u) {
             const int q = gtid + u * NT;
+            vmax[u] = 0xff80ff80u;
             if (q < my_vec) {
                 const uint4 a = vs[q], b = vt[q];
-                const uint32_t m = hmax2u(hmax2u(a.x, a.y), hmax2u(a.z, a.w));
-                const float v = fmaxf(bf16lo(m), bf16hi(m));
-                if (v > best) {
-                    best = v;
-                    bq = q;
-                }
+                vmax[u] = hmax2u(hmax2u(a.x, a.y), hmax2u(a.z, a.w));
+                smax = hmax2u(smax, vmax[u]);
                 tmax = hmax2u(tmax, hmax2u(hmax2u(b.x, b.y), hmax2u(b.z, b.w)));
             }
         }
-        const float ms = best, mt = fmaxf(bf16lo(tmax), bf16hi(tmax));
+        const float ms = fmaxf(bf16lo(smax), bf16hi(smax)), mt = fmaxf(bf16lo(tmax), bf16hi(tmax));
+        // reference difference at the first element equal to the student max
         float xd = 0.f;
-        if (bq >= 0) {  // reference difference at the first element equal to the max
+        if (ms != -INFINITY) {
+            int bq = gtid;
+#pragma unroll
+            for (int u = VPT - 1; u >= 0; --u)
+                if (bf16lo(vmax[u]) == ms || bf16hi(vmax[u]) == ms)
+                    bq = gtid + u * NT;
             const uint4 a = vs[bq], b = vt[bq];
             bool found = false;
 #pragma unroll
@@ -450,49 +430,71 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
         }
     };
 
-    // row constants of row k from the CS records (identical in every warp/CTA)
+    // row constants of row k from the CS records, computed by the group's
+    // first warp (fixed merge order: identical in every CTA) and shared with
+    // the group through shared memory
     auto combine = [&](int k, float &ell) {
         const int slot = k % kSlots;
-        wait_bar(&recv[slot], (uint32_t)((k / kSlots) & 1), true);
-        const float *r = rec + slot * CS * 8;
-        Student A = student_empty();
-        Teacher B = teacher_empty();
-        if (lane < CS) {
-            const float4 x = *reinterpret_cast<const float4 *>(r + lane * 8);
-            const float4 y = *reinterpret_cast<const float4 *>(r + lane * 8 + 4);
-            A = Student{x.x, x.y, x.z, x.w};
-            B = Teacher{y.x, y.y};
+        float *bc = rcs + group * 16;
+        if (gwarp == 0) {
+            wait_bar(&recv[slot], (uint32_t)((k / kSlots) & 1), true);
+            const float *r = rec + slot * CS * 8;
+            Student A = student_empty();
+            Teacher B = teacher_empty();
+            if (lane < CS) {
+                const float4 x = *reinterpret_cast<const float4 *>(r + lane * 8);
+                const float4 y = *reinterpret_cast<const float4 *>(r + lane * 8 + 4);
+                A = Student{x.x, x.y, x.z, x.w};
+                B = Teacher{y.x, y.y};
+            }
+            lane_merge<CS>(A, B);
+            if (lane == 0) {
+                const RowConst rc = row_const(A, B);
+                float e = rc.kl;
+                const int y = meta[k % kStages].z;
+                if (y >= 0) {
+                    const int owner = (y / 8) / slice_vec;
+                    e = (r[owner * 8 + 6] - r[owner * 8 + 7]) - rc.dl;
+                }
+                // gradient constants of the row (see grad): p w = 2^(z_s log2e + nlw),
+                // sign sg of w applied through fma by (sg, sg)
+                const float wi = __int_as_float(meta[k % kStages].w), wl = wi * e;
+                const float sg = wi < 0.f ? -1.f : 1.f;
+                bc[0] = rc.lse_s, bc[1] = rc.lse_t, bc[2] = rc.kl, bc[3] = e;
+                bc[4] = -rc.lse_s * kLog2e + log2f(fabsf(y < 0 ? wi : wl));  // nlw
+                bc[5] = sg;
+                bc[6] = -sg * rc.d;
+                bc[7] = -sg * rc.cp;
+                bc[8] = -sg * (rc.d + rc.cp);     // bf16 output: one rounding of d + cp
+                bc[9] = wl > 0.f ? -1.f : 1.f;    // sampled: sign of -w l
+                bc[10] = wl;
+                mbar_arrive_expect_tx(&recv[slot], CS * 32u);  // re-arm for row k + kSlots
+            }
         }
-        lane_merge<CS>(A, B);
-        A.m = __shfl_sync(0xffffffffu, A.m, 0);
-        A.s = __shfl_sync(0xffffffffu, A.s, 0);
-        A.a = __shfl_sync(0xffffffffu, A.a, 0);
-        A.d = __shfl_sync(0xffffffffu, A.d, 0);
-        B.m = __shfl_sync(0xffffffffu, B.m, 0);
-        B.s = __shfl_sync(0xffffffffu, B.s, 0);
-        const RowConst rc = row_const(A, B);
-        ell = rc.kl;
-        const int y = meta[k % kStages].z;
-        if (y >= 0) {
-            const int owner = (y / 8) / slice_vec;
-            ell = (r[owner * 8 + 6] - r[owner * 8 + 7]) - rc.dl;
-        }
-        return rc;
+        group_sync();
+        GradConst gc;
+        gc.lse_s = bc[0], gc.lse_t = bc[1], gc.kl = bc[2];
+        ell = bc[3];
+        gc.nlw = bc[4], gc.sg = bc[5], gc.nd = bc[6], gc.ncp = bc[7], gc.nc = bc[8], gc.sgl = bc[9];
+        gc.wl = bc[10];
+        return gc;
     };
 
-    auto grad = [&](int k, const RowConst &rc, float ell) {
+    auto grad = [&](int k, const GradConst &gc) {
         if (!p.grad)
             return;
         const int s = k % kStages;
         const int4 m = meta[s];
         const uint4 *vs = reinterpret_cast<const uint4 *>(stage + s * stage_bytes);
         const uint4 *vt = reinterpret_cast<const uint4 *>(stage + s * stage_bytes + slice_bytes);
-        const float wi = __int_as_float(m.w), wl = wi * ell;
         const int y = m.z;
+        const float wl = gc.wl;
         const size_t row_off = (size_t)m.y * (size_t)p.ld + (size_t)v0 * 8;
-        const float2 L2 = splat(kLog2e), D = splat(rc.d), CP = splat(rc.cp);
-        const float2 NL = splat(-rc.lse_s * kLog2e);
-        const float2 W = splat(wi), NWL = splat(-wl);
+        // p |w| = 2^(z_s log2e - LSE_s log2e + log2 |w|); the sign of w enters through an
+        // fma by (sg, sg), which is exact on z_s - z_t
+        const float2 L2 = splat(kLog2e), NLW = splat(gc.nlw);
+        const float2 SG = splat(gc.sg), ND = splat(gc.nd), NCP = splat(gc.ncp), NC = splat(gc.nc);
+        const float2 SGL = splat(gc.sgl);
 #pragma unroll
         for (int u = 0; u < VPT; ++u) {
             const int q = gtid + u * NT;
@@ -503,15 +505,16 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         const float2 a2 = unpack2(word(a, j)), b2 = unpack2(word(b, j));
-                        const float2 pv = ex2x2(ffma2(a2, L2, NL));
-                        g[j] = fmul2(fmul2(pv, W), fsub2(fsub2(fsub2(a2, b2), D), CP));
+                        const float2 pw = ex2x2(ffma2(a2, L2, NLW));
+                        // sg ((z_s - z_t) - c) with one rounding; sg (z_s - z_t) is exact
+                        const float2 x = fsub2(a2, b2);
+                        g[j] = G32 ? fmul2(pw, fadd2(ffma2(x, SG, ND), NCP)) : fmul2(pw, ffma2(x, SG, NC));
                     }
                 } else {  // sampled token: g = w l (e_y - p)
                     const uint4 a = vs[q];
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
-                        const float2 pv = ex2x2(ffma2(unpack2(word(a, j)), L2, NL));
-                        g[j] = fmul2(pv, NWL);
+                        g[j] = fmul2(ex2x2(ffma2(unpack2(word(a, j)), L2, NLW)), SGL);
                         const int e = ((v0 + q) * 8 + 2 * j) - y;
                         if (e == 0)
                             g[j].x += wl;
@@ -550,18 +553,16 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
         wait_full(k);
         stats(k);
         float ell;
-        const RowConst rc = combine(k, ell);
-        if (gtid == 0)
-            mbar_arrive_expect_tx(&recv[k % kSlots], CS * 32u);  // re-arm for row k + kSlots
+        const GradConst gc = combine(k, ell);
         if (rank == 0 && gtid == 0) {
             const int4 m = meta[k % kStages];
-            if (!isfinite(rc.lse_s) || !isfinite(rc.lse_t) || !isfinite(ell))
+            if (!isfinite(gc.lse_s) || !isfinite(gc.lse_t) || !isfinite(ell))
                 set_status(p.status, TURNOPD_ERR_NONFINITE);
             p.token_loss[m.x] = ell;
             p.row_wl[cid + k * ncl] = (double)__int_as_float(m.w) * (double)ell;
         }
         if (!dead())
-            grad(k, rc, ell);
+            grad(k, gc);
         __syncwarp();
         if (lane == 0)
             mbar_arrive(&empty[k % kStages]);
@@ -601,7 +602,8 @@ size_t cluster_smem_bytes(int slice_vec)
     return (size_t)kStages * 2 * slice_vec * 16 + 2 * kG * kCS * 8 * sizeof(float) +
            kStages * sizeof(int4) + (2 * kStages + 2 * kG) * sizeof(uint64_t) +
            kG * (kNT / 32) * 8 * sizeof(float) +  // per-group warp partials
-           kStages * sizeof(int);                   // row held by each stage
+           4 * sizeof(int) +                        // row held by each stage
+           kG * 16 * sizeof(float);                 // broadcast row constants
 }
 
 template <bool G32>
