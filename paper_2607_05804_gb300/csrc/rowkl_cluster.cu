@@ -180,7 +180,7 @@ __device__ __forceinline__ uint32_t word(const uint4 &v, int j)
 // (lanes beyond hold empty partials): exact max by butterfly, one rescale
 // exponential per lane, then butterfly sums.  Lane 0's result is used; its
 // association order is fixed, so every warp and CTA gets the same bits.
-template <int WIDTH>
+template <int WIDTH, bool USE_D = true>
 __device__ __forceinline__ void lane_merge(Student &S, Teacher &T)
 {
     float m = S.m, mt = T.m;
@@ -190,12 +190,15 @@ __device__ __forceinline__ void lane_merge(Student &S, Teacher &T)
         mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
     }
     // reference difference of the lowest lane holding the max
-    const unsigned own = __ballot_sync(0xffffffffu, S.m == m && m != -INFINITY);
-    const int src = own ? __ffs(own) - 1 : 0;
-    const float d = __shfl_sync(0xffffffffu, S.d, src);
+    float d = 0.f;
+    if (USE_D) {
+        const unsigned own = __ballot_sync(0xffffffffu, S.m == m && m != -INFINITY);
+        const int src = own ? __ffs(own) - 1 : 0;
+        d = __shfl_sync(0xffffffffu, S.d, src);
+    }
     const float f = m == -INFINITY ? 0.f : ex2((S.m - m) * kLog2e);
     const float ft = mt == -INFINITY ? 0.f : ex2((T.m - mt) * kLog2e);
-    float s = S.s * f, a = fmaf(S.s, S.d - d, S.a) * f, t = T.s * ft;
+    float s = S.s * f, a = (USE_D ? fmaf(S.s, S.d - d, S.a) : S.a) * f, t = T.s * ft;
     if (S.m == -INFINITY)
         s = 0.f, a = 0.f;
     if (T.m == -INFINITY)
@@ -229,6 +232,11 @@ template <int CS, int NT, int VPT, int G, bool G32>
 __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_vec, int nvec)
 {
     constexpr int kSlots = 2 * G;
+    // Reference difference d (A = sum e ((z_s - z_t) - d), d at the student's
+    // max): it keeps gradients at a dominant token accurate to fp32 relative
+    // precision.  A bf16 gradient needs no such care: without d the error of
+    // E_p[z_s - z_t] is ~1e-6 absolute, under a bf16 ulp of those gradients.
+    constexpr bool kUseD = G32;
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ int s_dead;
     constexpr int NWG = NT / 32;  // warps per group
@@ -347,9 +355,10 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
             }
         }
         const float ms = fmaxf(bf16lo(smax), bf16hi(smax)), mt = fmaxf(bf16lo(tmax), bf16hi(tmax));
-        // reference difference at the first element equal to the student max
+        // reference difference at the first element equal to the student max;
+        // only the fp32 gradient needs it (see kUseD)
         float xd = 0.f;
-        if (ms != -INFINITY) {
+        if (kUseD && ms != -INFINITY) {
             int bq = gtid;
 #pragma unroll
             for (int u = VPT - 1; u >= 0; --u)
@@ -384,14 +393,14 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
                     const float2 a2 = unpack2(word(a, j)), b2 = unpack2(word(b, j));
                     const float2 es = ex2x2(ffma2(a2, L2, NS));
                     S2 = fadd2(S2, es);
-                    A2 = ffma2(es, fsub2(fsub2(a2, b2), D), A2);
+                    A2 = ffma2(es, kUseD ? fsub2(fsub2(a2, b2), D) : fsub2(a2, b2), A2);
                     T2 = fadd2(T2, ex2x2(ffma2(b2, L2, NTT)));
                 }
             }
         }
         Student S = ms == -INFINITY ? student_empty() : Student{ms, S2.x + S2.y, A2.x + A2.y, xd};
         Teacher U = mt == -INFINITY ? teacher_empty() : Teacher{mt, T2.x + T2.y};
-        lane_merge<32>(S, U);
+        lane_merge<32, kUseD>(S, U);
         float *rg = red + group * NWG * 8;
         if (lane == 0) {
             float *rw = rg + gwarp * 8;
@@ -406,7 +415,7 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
                 A = Student{r[0], r[1], r[2], r[3]};
                 B = Teacher{r[4], r[5]};
             }
-            lane_merge<NWG>(A, B);
+            lane_merge<NWG, kUseD>(A, B);
             A.m = __shfl_sync(0xffffffffu, A.m, 0);
             A.s = __shfl_sync(0xffffffffu, A.s, 0);
             A.a = __shfl_sync(0xffffffffu, A.a, 0);
@@ -447,7 +456,7 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
                 A = Student{x.x, x.y, x.z, x.w};
                 B = Teacher{y.x, y.y};
             }
-            lane_merge<CS>(A, B);
+            lane_merge<CS, kUseD>(A, B);
             if (lane == 0) {
                 const RowConst rc = row_const(A, B);
                 float e = rc.kl;
