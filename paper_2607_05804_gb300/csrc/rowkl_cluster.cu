@@ -594,7 +594,7 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
 
 // Threads per row group and groups per CTA (tuning knobs).
 #ifndef TURNOPD_ROW_THREADS
-#define TURNOPD_ROW_THREADS 384
+#define TURNOPD_ROW_THREADS 512
 #endif
 #ifndef TURNOPD_ROW_GROUPS
 #define TURNOPD_ROW_GROUPS 2
