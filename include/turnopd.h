@@ -224,6 +224,39 @@ turnopd_status turnopd_loss_fwd_bwd_static(const void *z_student, const void *z_
                                            int32_t *dev_status, turnopd_stream_t stream);
 
 /*
+ * turnopd_fused_lmhead_fwd_bwd -- the OPD loss with the two LM heads fused in:
+ * student logits z_s = h_s W_s^T and teacher logits z_t = h_t W_t^T of the
+ * supervised tokens are formed tile by tile on the tensor cores and consumed
+ * by the loss without ever being stored (Eq. opd-rkl, full vocabulary).
+ * Outputs l_i, L = sum_i w_i l_i and dL/dh_s = G W_s with G = dL/dz_s (the
+ * chain rule through z_s = h_s W_s^T; G is formed in fp32 and rounded to bf16
+ * for the second tensor-core product).
+ * Inputs (device, row-major, bf16):
+ *   h_s [num_tokens, d_s], W_s [vocab, d_s], h_t [num_tokens, d_t], W_t [vocab, d_t]
+ *   loss_mask uint8[num_tokens], w float32[num_tokens] (turnopd_weights).
+ *   d_s must be a multiple of 256, d_t of 64; every pointer 16-byte aligned.
+ *   mode: TURNOPD_FULL_VOCAB only (others return TURNOPD_ERR_UNSUPPORTED).
+ * Outputs:
+ *   dh_s_out  float32[num_tokens, d_s] or NULL (forward only); rows of masked
+ *             tokens are zero.
+ *   token_loss_out float32[num_tokens] (0 for masked tokens), loss_out double.
+ * Workspace: turnopd_fused_workspace_bytes(num_tokens, vocab, d_s, d_t) bytes
+ *   (gathered hidden rows, per-row partial statistics, the transposed W_s and
+ *   G in bf16: about 2 num_tokens vocab + 2 d_s vocab bytes).
+ * Device errors: TURNOPD_ERR_NONFINITE, TURNOPD_ERR_TIMEOUT (bounded waits).
+ */
+turnopd_status turnopd_fused_lmhead_fwd_bwd(const void *h_s, const void *W_s, int64_t d_s,
+                                            const void *h_t, const void *W_t, int64_t d_t,
+                                            int64_t vocab, const uint8_t *loss_mask,
+                                            const float *w, int64_t num_tokens, int32_t mode,
+                                            float *dh_s_out, float *token_loss_out,
+                                            double *loss_out, void *workspace,
+                                            size_t workspace_bytes, int32_t *dev_status,
+                                            turnopd_stream_t stream);
+
+size_t turnopd_fused_workspace_bytes(int64_t num_tokens, int64_t vocab, int64_t d_s, int64_t d_t);
+
+/*
  * turnopd_turn_stats -- turn statistics of the per-token losses
  * (Eq. observed-turn-kl: K_t is the mean per-token reverse KL over the
  * supervised tokens at turn t, over trajectories that reach t; the survivor

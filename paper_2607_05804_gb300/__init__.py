@@ -22,7 +22,7 @@ __all__ = [
     "turnopd_turn_counts", "turnopd_weights", "turnopd_weights_workspace_bytes",
     "turnopd_loss_fwd_bwd", "turnopd_loss_workspace_bytes", "turnopd_turn_stats",
     "turnopd_alpha_schedule", "turnopd_status_string", "turnopd_loss_fwd_bwd_static",
-    "TURNOPD_STATIC_MAX_TOKENS",
+    "TURNOPD_STATIC_MAX_TOKENS", "turnopd_fused_lmhead_fwd_bwd", "turnopd_fused_workspace_bytes",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -77,6 +77,8 @@ def load():
         "turnopd_turn_stats": [P, P, P, P, i32, i64, i32, P, P, P, P, P, P, P],
         "turnopd_loss_fwd_bwd_static": [P, P, i32, i64, i64, i64, P, P, P, P, i64, i32, P, i32,
                                         u32, P, P, P, P],
+        "turnopd_fused_lmhead_fwd_bwd": [P, P, i64, P, P, i64, i64, P, P, i64, i32, P, P, P, P, sz,
+                                         P, P],
     }
     for name, args in sig.items():
         fn = getattr(lib, name)
@@ -86,6 +88,8 @@ def load():
     lib.turnopd_weights_workspace_bytes.restype = sz
     lib.turnopd_loss_workspace_bytes.argtypes = [i64]
     lib.turnopd_loss_workspace_bytes.restype = sz
+    lib.turnopd_fused_workspace_bytes.argtypes = [i64, i64, i64, i64]
+    lib.turnopd_fused_workspace_bytes.restype = sz
     lib.turnopd_alpha_schedule.argtypes = [i64, i64, f64, f64]
     lib.turnopd_alpha_schedule.restype = f64
     lib.turnopd_status_string.argtypes = [ctypes.c_int]
@@ -154,6 +158,38 @@ def turnopd_weights_workspace_bytes(num_traj: int, max_turns: int) -> int:
 
 def turnopd_loss_workspace_bytes(num_tokens: int) -> int:
     return int(load().turnopd_loss_workspace_bytes(int(num_tokens)))
+
+
+def turnopd_fused_workspace_bytes(num_tokens: int, vocab: int, d_s: int, d_t: int) -> int:
+    return int(load().turnopd_fused_workspace_bytes(int(num_tokens), int(vocab), int(d_s), int(d_t)))
+
+
+def turnopd_fused_lmhead_fwd_bwd(h_s, W_s, h_t, W_t, loss_mask, w, mode, dh_s_out, token_loss_out,
+                                 loss_out, workspace, dev_status, stream=None):
+    """h_s [T, d_s], W_s [V, d_s], h_t [T, d_t], W_t [V, d_t] bf16; dh_s_out [T, d_s] fp32 or None."""
+    import torch
+
+    T, d_s = h_s.shape
+    d_t = h_t.shape[1]
+    V = W_s.shape[0]
+    _need(h_s, "h_s", torch.bfloat16)
+    _need(W_s, "W_s", torch.bfloat16)
+    _need(h_t, "h_t", torch.bfloat16, T * d_t)
+    _need(W_t, "W_t", torch.bfloat16, V * d_t)
+    if W_s.shape[1] != d_s or W_t.shape[0] != V or h_t.shape[0] != T:
+        raise ValueError("shape mismatch between hidden states and heads")
+    _need(loss_mask, "loss_mask", torch.uint8, T)
+    _need(w, "w", torch.float32, T)
+    _need(dh_s_out, "dh_s_out", torch.float32, T * d_s)
+    _need(token_loss_out, "token_loss_out", torch.float32, T)
+    _need(loss_out, "loss_out", torch.float64, 1)
+    _need(workspace, "workspace")
+    _need(dev_status, "dev_status", torch.int32, 1)
+    _check(load().turnopd_fused_lmhead_fwd_bwd(
+        _ptr(h_s), _ptr(W_s), d_s, _ptr(h_t), _ptr(W_t), d_t, V, _ptr(loss_mask), _ptr(w), T,
+        int(mode), _ptr(dh_s_out), _ptr(token_loss_out), _ptr(loss_out), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream)),
+        "turnopd_fused_lmhead_fwd_bwd")
 
 
 def turnopd_turn_counts(turn_id, loss_mask, traj_offsets, max_turns, traj_turn_cnt, counts,

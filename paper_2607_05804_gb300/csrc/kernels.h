@@ -81,6 +81,29 @@ struct RowIn {
 
 int device_sm_count();
 
+// Pieces of the loss path reused by the fused LM-head path.
+cudaError_t launch_compaction(const LossArgs &a, int4 *rows, int32_t *blk_count, int32_t *nvalid,
+                              cudaStream_t stream);
+void launch_loss_sum(const double *row_wl, const int32_t *nvalid, double *loss, int32_t *status,
+                     cudaStream_t stream);
+// Zero rows i (of d fp32 values) of out where mask[i] == 0.
+void launch_zero_masked_f32(const uint8_t *mask, int64_t T, int64_t d, float *out, cudaStream_t stream);
+
+// Fused LM heads (bf16 hidden states and heads) + loss + dL/dh_s.
+struct FusedCall {
+    const void *h_s, *W_s, *h_t, *W_t;
+    int64_t d_s, d_t, vocab, T;
+    const uint8_t *mask;
+    const float *w;
+    float *dh_s;
+    float *token_loss;
+    double *loss;
+    void *workspace;
+    int32_t *status;
+};
+size_t fused_workspace_bytes(int64_t T, int64_t V, int64_t d_s, int64_t d_t);
+cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream);
+
 // Cluster-resident kernel for aligned bf16 rows; sets *used = false (and
 // launches nothing) when the shape does not fit it.
 cudaError_t launch_row_cluster(const RowIn &p, bool fp32_grad, cudaStream_t stream, bool *used);

@@ -404,14 +404,32 @@ static cudaError_t launch_portable(const RowIn &p, bool vec, int grid, cudaStrea
 
 static bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
-cudaError_t launch_loss(const LossArgs &a, const LossWorkspace &ws, cudaStream_t stream)
+cudaError_t launch_compaction(const LossArgs &a, int4 *rows, int32_t *blk_count, int32_t *nvalid,
+                              cudaStream_t stream)
 {
     const int nblk = (int)((a.T + kCompactBlock - 1) / kCompactBlock);
     CompactIn c{a.mask, a.row_of_token, a.sampled_ids, a.w, a.num_rows, a.vocab, a.T, a.mode,
                 a.token_loss, a.status};
-    k_compact_count<<<nblk, kCompactThreads, 0, stream>>>(c, ws.blk_count);
-    k_compact_scatter<<<nblk, kCompactThreads, 0, stream>>>(c, ws.blk_count, ws.rows, ws.nvalid);
-    cudaError_t e = cudaGetLastError();
+    k_compact_count<<<nblk, kCompactThreads, 0, stream>>>(c, blk_count);
+    k_compact_scatter<<<nblk, kCompactThreads, 0, stream>>>(c, blk_count, rows, nvalid);
+    return cudaGetLastError();
+}
+
+void launch_loss_sum(const double *row_wl, const int32_t *nvalid, double *loss, int32_t *status,
+                     cudaStream_t stream)
+{
+    k_loss_sum<<<1, 1024, 0, stream>>>(row_wl, nvalid, loss, status);
+}
+
+void launch_zero_masked_f32(const uint8_t *mask, int64_t T, int64_t d, float *out, cudaStream_t stream)
+{
+    const int grid = (int)std::min<int64_t>(std::max<int64_t>(T, 1), (int64_t)device_sm_count() * 8);
+    k_zero_masked<float><<<grid, 256, 0, stream>>>(mask, nullptr, T, T, d, d, out);
+}
+
+cudaError_t launch_loss(const LossArgs &a, const LossWorkspace &ws, cudaStream_t stream)
+{
+    cudaError_t e = launch_compaction(a, ws.rows, ws.blk_count, ws.nvalid, stream);
     if (e != cudaSuccess)
         return e;
 
@@ -450,7 +468,7 @@ cudaError_t launch_loss(const LossArgs &a, const LossWorkspace &ws, cudaStream_t
         if (e != cudaSuccess)
             return e;
     }
-    k_loss_sum<<<1, 1024, 0, stream>>>(ws.row_wl, ws.nvalid, a.loss, a.status);
+    launch_loss_sum(ws.row_wl, ws.nvalid, a.loss, a.status, stream);
     return cudaGetLastError();
 }
 

@@ -194,6 +194,45 @@ turnopd_status turnopd_loss_fwd_bwd(const void *z_student, const void *z_teacher
     return cuda_status(launch_loss(a, loss_workspace_layout(workspace, num_tokens), s));
 }
 
+size_t turnopd_fused_workspace_bytes(int64_t num_tokens, int64_t vocab, int64_t d_s, int64_t d_t)
+{
+    if (num_tokens < 0 || vocab < 1 || d_s < 1 || d_t < 1)
+        return 0;
+    return fused_workspace_bytes(num_tokens, vocab, d_s, d_t);
+}
+
+turnopd_status turnopd_fused_lmhead_fwd_bwd(const void *h_s, const void *W_s, int64_t d_s,
+                                            const void *h_t, const void *W_t, int64_t d_t,
+                                            int64_t vocab, const uint8_t *loss_mask,
+                                            const float *w, int64_t num_tokens, int32_t mode,
+                                            float *dh_s_out, float *token_loss_out,
+                                            double *loss_out, void *workspace,
+                                            size_t workspace_bytes, int32_t *dev_status,
+                                            turnopd_stream_t stream)
+{
+    if (!loss_out || !dev_status || !W_s || !W_t)
+        return TURNOPD_ERR_NULL;
+    if (num_tokens > 0 && (!h_s || !h_t || !loss_mask || !w || !token_loss_out))
+        return TURNOPD_ERR_NULL;
+    if (mode != TURNOPD_FULL_VOCAB)
+        return TURNOPD_ERR_UNSUPPORTED;
+    if (num_tokens < 0 || num_tokens > INT32_MAX || vocab < 1 || vocab > INT32_MAX || d_s < 256 ||
+        d_s % 256 != 0 || d_t < 64 || d_t % 64 != 0 || d_s > 65536 || d_t > 65536)
+        return TURNOPD_ERR_SHAPE;
+    if (misaligned(h_s, 16) || misaligned(W_s, 16) || misaligned(h_t, 16) || misaligned(W_t, 16) ||
+        (dh_s_out && misaligned(dh_s_out, 16)) || misaligned(loss_out, 8))
+        return TURNOPD_ERR_SHAPE;
+    if (!workspace || misaligned(workspace, 256) ||
+        workspace_bytes < fused_workspace_bytes(num_tokens, vocab, d_s, d_t))
+        return TURNOPD_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (num_tokens == 0)
+        return cuda_status(cudaMemsetAsync(loss_out, 0, sizeof(double), s));
+    FusedCall c{h_s, W_s, h_t, W_t, d_s, d_t, vocab, num_tokens, loss_mask, w, dh_s_out,
+                token_loss_out, loss_out, workspace, dev_status};
+    return cuda_status(launch_fused(c, s));
+}
+
 turnopd_status turnopd_turn_stats(const float *token_loss, const int32_t *turn_id,
                                   const uint8_t *loss_mask, const int64_t *traj_offsets,
                                   int32_t num_traj, int64_t num_tokens, int32_t max_turns,

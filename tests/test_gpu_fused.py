@@ -1,0 +1,126 @@
+"""GPU parity of the fused LM-head path (turnopd_fused_lmhead_fwd_bwd) against
+the fp64 oracle.
+
+Tolerances: per-token loss and total loss as for the logit path (the logits are
+fp32 tensor-core sums of exact bf16 products instead of fp64 sums: relative
+error ~1e-6).  dL/dh_s = G W_s with G rounded to bf16 (2^-9 relative) before
+the second product: per element within 1e-2 of its row's maximum |dh|, and a
+relative Frobenius error within 4e-3 per row.
+"""
+import numpy as np
+import pytest
+
+import workloads as W
+from parity import assert_loss, assert_token_loss
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def P():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2607_05804_gb300 as P
+
+    P.load()
+    return P
+
+
+def assert_dh(dh_gpu, dh_ref):
+    dh_gpu = np.asarray(dh_gpu, np.float64)
+    dh_ref = np.asarray(dh_ref, np.float64)
+    rowmax = np.abs(dh_ref).max(axis=1, keepdims=True)
+    err = np.abs(dh_gpu - dh_ref)
+    bad = np.argwhere(err > 1e-2 * rowmax + 1e-30)
+    assert bad.size == 0, f"{len(bad)} dh elements off, first {bad[:3].tolist()}"
+    fro = np.linalg.norm(dh_gpu - dh_ref, axis=1) / np.maximum(np.linalg.norm(dh_ref, axis=1), 1e-30)
+    assert (fro <= 4e-3).all(), fro.max()
+
+
+def run_fused(P, b, d_s, d_t, V, seed, alpha=1.0, grad=True):
+    from paper_2607_05804_gb300.step import LossStep, to_device
+
+    T = b.num_tokens
+    h_s, W_s, h_t, W_t = W.make_fused(T, d_s, d_t, V, seed=seed, device="cuda")
+    tid, msk, off, _ = to_device(b, "cuda", compact=False)
+    step = LossStep(tid, msk, off, b.max_turns, V, alpha=alpha)
+    w = step.weights()
+    ws = torch.empty(P.turnopd_fused_workspace_bytes(T, V, d_s, d_t), dtype=torch.uint8, device="cuda")
+    dh = torch.full((T, d_s), 3.0, dtype=torch.float32, device="cuda") if grad else None
+    tl = torch.full((T,), 7.0, dtype=torch.float32, device="cuda")
+    loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+    P.turnopd_fused_lmhead_fwd_bwd(h_s, W_s, h_t, W_t, msk, w, 0, dh, tl, loss, ws, step.dev_status)
+    torch.cuda.synchronize()
+    assert step.status() == 0
+    return (h_s, W_s, h_t, W_t), w.cpu().numpy(), dh, tl.cpu().numpy(), loss.item()
+
+
+def test_fused_small_all_rows(P, oracle):
+    """Ragged vocabulary (1000: last 256-tile partial, padded K 1024) and
+    several 128-row tiles with a ragged last tile."""
+    b = W.packed(seed=3, num_traj=2, traj_len=160)
+    d_s, d_t, V = 256, 192, 1000
+    heads, w, dh, tl, loss = run_fused(P, b, d_s, d_t, V, seed=4)
+    bits = [W.bf16_bits(x) for x in heads]
+    dh_ref, tl_ref, loss_ref = oracle.fused_lmhead(*bits, b.loss_mask, w)
+    assert_token_loss(tl, tl_ref, b.loss_mask)
+    assert_loss(loss, loss_ref)
+    g = dh.cpu().numpy()
+    m = b.loss_mask == 1
+    assert (g[~m] == 0).all()
+    assert_dh(g[m], dh_ref[m])
+
+
+def test_fused_forward_only(P, oracle):
+    b = W.packed(seed=5, num_traj=1, traj_len=300)
+    d_s, d_t, V = 512, 256, 4100
+    heads, w, _, tl, loss = run_fused(P, b, d_s, d_t, V, seed=6, grad=False)
+    bits = [W.bf16_bits(x) for x in heads]
+    _, tl_ref, loss_ref = oracle.fused_lmhead(*bits, b.loss_mask, w)
+    assert_token_loss(tl, tl_ref, b.loss_mask)
+    assert_loss(loss, loss_ref)
+
+
+def test_fused_full_heads_sampled_tokens(P, oracle):
+    """Full-size heads (d_s = 4096, d_t = 5120, V = 151,936) on a 600-token batch;
+    the oracle recomputes a few supervised tokens, all rows checked by properties."""
+    b = W.packed(seed=7, num_traj=1, traj_len=600)
+    d_s, d_t, V = 4096, 5120, W.V_QWEN
+    heads, w, dh, tl, loss = run_fused(P, b, d_s, d_t, V, seed=8)
+    bits = [W.bf16_bits(x) for x in heads]
+    valid = np.nonzero(b.loss_mask)[0]
+    rng = np.random.default_rng(0)
+    pick = np.unique(np.concatenate([valid[:1], valid[-1:], rng.choice(valid, 4, replace=False)]))
+    dh_ref, tl_ref, _ = oracle.fused_lmhead(*bits, b.loss_mask, w, subset=pick)
+    assert_token_loss(tl[pick], tl_ref[pick])
+    g = dh.cpu().numpy()
+    assert_dh(g[pick], dh_ref[pick])
+    assert (g[b.loss_mask == 0] == 0).all()
+    assert (tl[b.loss_mask == 0] == 0).all()
+    assert (tl[valid] >= -1e-4).all()
+    wl = float(np.dot(w.astype(np.float64), tl.astype(np.float64)))
+    assert abs(loss - wl) <= 1e-9 * abs(wl)
+
+
+def test_fused_errors(P):
+    T, d_s, d_t, V = 8, 256, 64, 512
+    z = lambda *s: torch.zeros(s, dtype=torch.bfloat16, device="cuda")
+    msk = torch.ones(T, dtype=torch.uint8, device="cuda")
+    w = torch.ones(T, dtype=torch.float32, device="cuda")
+    tl = torch.zeros(T, dtype=torch.float32, device="cuda")
+    loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ws = torch.empty(P.turnopd_fused_workspace_bytes(T, V, d_s, d_t), dtype=torch.uint8, device="cuda")
+    with pytest.raises(P.TurnopdError) as e:  # d_s not a multiple of 256
+        P.turnopd_fused_lmhead_fwd_bwd(z(T, 128), z(V, 128), z(T, d_t), z(V, d_t), msk, w, 0, None, tl,
+                                       loss, ws, st)
+    assert e.value.code == 2
+    with pytest.raises(P.TurnopdError) as e:  # sampled mode not offered here
+        P.turnopd_fused_lmhead_fwd_bwd(z(T, d_s), z(V, d_s), z(T, d_t), z(V, d_t), msk, w, 1, None, tl,
+                                       loss, ws, st)
+    assert e.value.code == 6
+    with pytest.raises(P.TurnopdError) as e:  # small workspace
+        P.turnopd_fused_lmhead_fwd_bwd(z(T, d_s), z(V, d_s), z(T, d_t), z(V, d_t), msk, w, 0, None, tl,
+                                       loss, ws[:1024], st)
+    assert e.value.code == 10
