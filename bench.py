@@ -47,7 +47,7 @@ def parse():
     p.add_argument("--steps", type=int, default=20)
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["native", "reference"], default="native")
-    p.add_argument("--workload", default="packed", choices=["packed", "household", "multihop"])
+    p.add_argument("--workload", default="packed", choices=["packed", "household", "multihop", "fused"])
     p.add_argument("--mode", default="full", choices=["full", "sampled"])
     p.add_argument("--alpha", type=float, default=0.5)
     p.add_argument("--no-e2e", action="store_true")
@@ -258,11 +258,123 @@ def reference_arm(args, world, rank):
     print(json.dumps(out), flush=True)
 
 
+# weights (3) + fused call (compaction 2, gathers 2, W_s transpose, statistics pass,
+# merge, gradient pass, masked-row zeroing, dL/dh_s, loss sum) + turn statistics (2)
+FUSED_KERNELS_PER_STEP = 16
+
+
+def fused_cpu_baseline(b, heads, w, budget_s=12.0):
+    """The fp64 oracle on a bounded sample of supervised tokens of the fused
+    workload (each token: both heads' logits over the whole vocabulary, the KL,
+    and dL/dh_s), scaled to supervised tokens/s."""
+    import numpy as np
+
+    import oracle
+    import workloads as W
+
+    bits = [W.bf16_bits(x) for x in heads]
+    wn = w.cpu().numpy()
+    valid = np.nonzero(b.loss_mask)[0]
+    n, spent = 4, 0.0
+    while True:
+        pick = valid[:: max(1, len(valid) // n)][:n]
+        t0 = time.perf_counter()
+        oracle.fused_lmhead(*bits, b.loss_mask, wn, subset=pick)
+        spent = time.perf_counter() - t0
+        if spent > budget_s / 4 or n >= len(valid):
+            break
+        n = min(len(valid), int(n * max(2.0, budget_s / 2 / max(spent, 1e-3))))
+    return {"value": len(pick) / spent, "unit": "tokens/s", "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": f"{len(pick)} of {len(valid)} supervised tokens, full heads, fp64, {spent:.1f} s"}
+
+
+def fused_bench(args, world, rank, local):
+    """Fused LM-head step: 8 x 2048 tokens (packed turn structure), student head
+    4096 x 151,936, teacher head 5120 x 151,936 (bf16), alpha = 1, full vocabulary:
+    weights, fused forward + backward (dL/dh_s), turn statistics."""
+    import torch
+
+    import workloads as W
+    import paper_2607_05804_gb300 as P
+    from paper_2607_05804_gb300.step import LossStep, to_device
+
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    P.load()
+    b = W.fused(seed=rank)
+    d_s, d_t, V = 4096, 5120, W.V_QWEN
+    T = b.num_tokens
+    h_s, W_s, h_t, W_t = W.make_fused(T, d_s, d_t, V, seed=3000 + rank, device=device)
+    tid, msk, off, _ = to_device(b, device, compact=False)
+    step = LossStep(tid, msk, off, b.max_turns, V, alpha=1.0)
+    ws = torch.empty(P.turnopd_fused_workspace_bytes(T, V, d_s, d_t), dtype=torch.uint8, device=device)
+    dh = torch.empty((T, d_s), dtype=torch.float32, device=device)
+
+    def one(ev=None):
+        step.weights()
+        if ev is not None:
+            ev[0].record()
+        P.turnopd_fused_lmhead_fwd_bwd(h_s, W_s, h_t, W_t, msk, step.w[:T], 0, dh,
+                                       step.token_loss[:T], step.loss, ws, step.dev_status)
+        if ev is not None:
+            ev[1].record()
+        step.turn_stats()
+
+    for _ in range(max(args.warmup, 3)):
+        one()
+    torch.cuda.synchronize()
+    if step.status() != 0:
+        raise RuntimeError(f"device status {step.status()}")
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local)
+    torch.cuda.synchronize()
+    sampler.start()
+    a.record()
+    for k in range(args.steps):
+        one(evs[k])
+    z.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    ms = a.elapsed_time(z)
+    call_ms = statistics.mean(x.elapsed_time(y) for x, y in evs)
+    Tv = b.num_valid
+    flops = 2.0 * Tv * V * (d_s + d_t) * 2 + 2.0 * Tv * V * d_s  # forward, recompute, dH
+    peak = 1715.8
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as fh:
+            peak = float(json.load(fh)["bf16_tflops_sustained"])
+        peak_kind = "measured (sustained)"
+    except Exception:
+        peak_kind = "fallback"
+    tflops = flops / (call_ms / 1e3) / 1e12
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = fused_cpu_baseline(b, (h_s, W_s, h_t, W_t), step.w[:T])
+    out = {"metric": "fused LM-head loss fwd+bwd supervised tokens/s", "value": Tv * args.steps / (ms / 1e3),
+           "unit": "tokens/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+           "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+           "config": {"workload": f"{b.name}_V{V}_ds{d_s}_dt{d_t}", "tokens": T, "supervised_tokens": Tv,
+                      "alpha": 1.0, "mode": "full", "flops_per_step": flops},
+           "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s",
+                        "frac": tflops / peak, "peak_kind": peak_kind,
+                        "kernel": "turnopd_fused_lmhead_fwd_bwd launch sequence", "launch_ms": call_ms,
+                        "traffic": None},
+           "gpu_launches": FUSED_KERNELS_PER_STEP * args.steps, "clocks": clocks, "e2e": None,
+           "cpu_baseline": cpu}
+    print(json.dumps(out), flush=True)
+
+
 def main():
     args = parse()
     world, rank, local = dist_env()
     if args.impl == "reference":
         reference_arm(args, world, rank)
+        return
+    if args.workload == "fused":
+        fused_bench(args, world, rank, local)
         return
     import torch
 
