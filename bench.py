@@ -54,8 +54,8 @@ def parse():
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-sample-rows", type=int, default=0, help="0 = size to ~15 s of oracle work")
     p.add_argument("--num-traj", type=int, default=0,
-                   help="packed workload only: trajectories (0 = 8); smaller cases serve profiling")
-    p.add_argument("--traj-len", type=int, default=0, help="packed workload only: tokens per trajectory")
+                   help="packed and fused workloads: trajectories (0 = 8); smaller cases serve profiling")
+    p.add_argument("--traj-len", type=int, default=0, help="packed and fused workloads: tokens per trajectory (0 = the workload's own)")
     return p.parse_args()
 
 
@@ -301,7 +301,7 @@ def fused_bench(args, world, rank, local):
     device = torch.device("cuda", local)
     torch.cuda.set_device(device)
     P.load()
-    b = W.fused(seed=rank)
+    b = W.fused(seed=rank, num_traj=args.num_traj or 8, traj_len=args.traj_len or 2048)
     d_s, d_t, V = 4096, 5120, W.V_QWEN
     T = b.num_tokens
     h_s, W_s, h_t, W_t = W.make_fused(T, d_s, d_t, V, seed=3000 + rank, device=device)

@@ -240,9 +240,10 @@ turnopd_status turnopd_loss_fwd_bwd_static(const void *z_student, const void *z_
  *   dh_s_out  float32[num_tokens, d_s] or NULL (forward only); rows of masked
  *             tokens are zero.
  *   token_loss_out float32[num_tokens] (0 for masked tokens), loss_out double.
- * Workspace: turnopd_fused_workspace_bytes(num_tokens, vocab, d_s, d_t) bytes
- *   (gathered hidden rows, per-row partial statistics, the transposed W_s and
- *   G in bf16: about 2 num_tokens vocab + 2 d_s vocab bytes).
+ * Workspace: turnopd_fused_workspace_bytes(num_tokens, vocab, d_s, d_t) bytes,
+ *   queried with the device that will run the call current (gathered hidden
+ *   rows, per-row partial statistics, G in bf16 and per-SM partial dH tiles:
+ *   about 2 num_tokens vocab bytes + 256 KiB per SM).
  * Device errors: TURNOPD_ERR_NONFINITE, TURNOPD_ERR_TIMEOUT (bounded waits).
  */
 turnopd_status turnopd_fused_lmhead_fwd_bwd(const void *h_s, const void *W_s, int64_t d_s,

@@ -2,25 +2,30 @@
 // supervised tokens are produced tile by tile on the tensor cores and consumed
 // in the epilogue, never stored.
 //
-//   forward   Z_s = H_s W_s^T (K = d_s), Z_t = H_t W_t^T (K = d_t) per 128-row x
-//             256-vocab tile, accumulated in tensor memory (512 fp32 columns:
-//             Z_s in [0,256), Z_t in [256,512)); the epilogue folds each tile
-//             into per-row online statistics (max, sum exp, sum exp (z_s - z_t))
-//             for both models over a group of vocabulary tiles;
+//   forward   Z_t = H_t W_t^T (K = d_t), then Z_s = H_s W_s^T (K = d_s), per
+//             128-row x 256-vocab tile, accumulated in tensor memory (512 fp32
+//             columns: Z_t in [0,256), Z_s in [256,512)); the epilogue folds
+//             each tile into per-row online statistics (max, sum exp,
+//             sum exp (z_s - z_t)) for both models over a group of tiles;
 //   merge     per row: LSE_s, LSE_t, KL = E_p[z_s - z_t] - (LSE_s - LSE_t);
 //   backward  the same tiles are recomputed; the epilogue forms
 //             G = w p_s ((z_s - z_t) - E_p[z_s - z_t]) = dL/dz_s and stores it in
 //             bf16 (the gradient w.r.t. the logits, not the logits);
-//   dH_s      = G W_s by a second tensor-core GEMM over the vocabulary.
+//   dH_s      = G W_s by a second tensor-core GEMM over the vocabulary, W_s read
+//             in place as an MN-major operand.
 //
 // GEMM structure (persistent, one CTA per SM): warp 0 streams 128x64 A and
 // 256x64 B bf16 tiles with TMA (128-byte swizzle) into a 4-stage ring, warp 1
-// allocates tensor memory and issues tcgen05.mma (one thread), warps 2..9
-// read the accumulator back (tcgen05.ld) for the epilogue.  Stage and
-// accumulator hand-offs are mbarriers completed by TMA transaction counts and
-// tcgen05.commit.  Every wait is bounded; on timeout the kernel records
-// TURNOPD_ERR_TIMEOUT, keeps its hand-off sequence without waiting, and
-// releases its tensor memory before it exits.
+// allocates tensor memory and issues tcgen05.mma (one thread), warps 2..17
+// read the accumulator back (tcgen05.ld) for the epilogue.  The two halves of
+// the accumulator are released separately: the epilogue copies Z_t of tile j
+// into registers while Z_s of tile j is computed, and reads Z_s of tile j
+// while Z_t of tile j+1 is computed, so the tensor pipe does not wait for the
+// epilogue.  Hand-offs are mbarriers completed by TMA transaction counts,
+// tcgen05.commit and epilogue-warp arrivals.  Every wait is bounded; on
+// timeout the kernel records TURNOPD_ERR_TIMEOUT, keeps its hand-off sequence
+// without waiting, drains its own in-flight copies and tensor-core work with
+// bounded waits, and releases its tensor memory before it exits.
 
 #include <cudaTypedefs.h>
 
@@ -35,10 +40,13 @@ namespace {
 
 constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2, B_BYTES = BN * BK * 2, STAGE_BYTES = A_BYTES + B_BYTES;
-constexpr int kEpiWarps = 8;
+constexpr int kEpiWarps = 16;                    // 4 per tensor-memory lane quarter
+constexpr int kColQuarters = kEpiWarps / 4;      // column slices of a tile
+constexpr int kEpiCols = BN / kColQuarters;      // 64 columns per epilogue thread
 constexpr int kThreads = 32 * (2 + kEpiWarps);
 constexpr uint32_t kLimit = 1u << 24;
 constexpr int kTilesPerGroup = 10;  // vocabulary tiles one work unit folds into one partial
+constexpr uint32_t kColT = 0, kColS = 256;  // tensor-memory columns of Z_t and Z_s
 
 struct FusedArgs {
     int64_t vocab;
@@ -47,7 +55,7 @@ struct FusedArgs {
     const int4 *rows;      // compacted supervised rows {token, row, y, w bits}
     const int32_t *nvalid;
     int n_groups;          // vocabulary groups (units per M tile)
-    float *part;           // [n_groups][2 halves][cap rows][8] partial statistics
+    float *part;           // [n_groups][kColQuarters][cap rows][8] partial statistics
     int64_t cap;           // row capacity of the gathered buffers
     const float *rowc;     // [cap][4]: lse_s * log2e - log2 |w|, E_p[z_s - z_t], sign w, -
     __nv_bfloat16 *G;      // [cap][vpad] backward output
@@ -66,28 +74,78 @@ __device__ __forceinline__ bool wait_lim(uint64_t *bar, uint32_t parity, int32_t
     return false;
 }
 
+// Bounded wait used while draining at exit (also after a timeout).
+__device__ __forceinline__ void wait_drain(uint64_t *bar, uint32_t parity)
+{
+    for (uint32_t i = 0; i < kLimit; ++i)
+        if (mbar_try_wait(bar, parity))
+            return;
+}
+
 // Shared memory: ring of STAGES x (A tile | B tile), then barriers.
 struct FusedSmem {
     uint8_t *a, *b;
-    uint64_t *full, *empty, *accf, *acce;
+    uint64_t *full, *empty;
+    uint64_t *acc_t, *acc_s;    // tensor core -> epilogue: Z_t / Z_s of a tile complete
+    uint64_t *free_t, *free_s;  // epilogue -> tensor core: Z_t / Z_s columns read
+    uint64_t *drain;
     uint32_t *tslot;
 };
 
-__device__ __forceinline__ FusedSmem carve(uint8_t *raw)
+__device__ __forceinline__ FusedSmem carve(uint8_t *raw, int b_bytes_padded)
 {
     FusedSmem s;
     uint8_t *base = raw + ((1024 - (smem_u32(raw) & 1023)) & 1023);
     s.a = base;
     s.b = base + STAGES * A_BYTES;
-    s.full = reinterpret_cast<uint64_t *>(s.b + STAGES * B_BYTES);
+    s.full = reinterpret_cast<uint64_t *>(s.b + b_bytes_padded);
     s.empty = s.full + STAGES;
-    s.accf = s.empty + STAGES;
-    s.acce = s.accf + 1;
-    s.tslot = reinterpret_cast<uint32_t *>(s.acce + 1);
+    s.acc_t = s.empty + STAGES;
+    s.acc_s = s.acc_t + 1;
+    s.free_t = s.acc_s + 1;
+    s.free_s = s.free_t + 1;
+    s.drain = s.free_s + 1;
+    s.tslot = reinterpret_cast<uint32_t *>(s.drain + 1);
     return s;
 }
 
-constexpr size_t kFusedSmem = STAGES * STAGE_BYTES + 1024 + 256;
+constexpr int kLmBRegion = STAGES * B_BYTES;
+// The dH kernel reads B as an MN-major operand; 32 KB of slack after the ring
+// keeps every address its descriptors can form inside the allocation.
+constexpr int kDhBRegion = STAGES * B_BYTES + 32768;
+constexpr size_t kFusedSmem = STAGES * A_BYTES + kLmBRegion + 1024 + 256;
+constexpr size_t kDhSmem = STAGES * A_BYTES + kDhBRegion + 1024 + 256;
+static_assert(kDhSmem <= 232448, "shared memory per CTA");
+
+__device__ __forceinline__ void init_barriers(const FusedSmem &sm)
+{
+    for (int s = 0; s < STAGES; ++s) {
+        mbar_init(&sm.full[s], 1);
+        mbar_init(&sm.empty[s], 1);
+    }
+    mbar_init(sm.acc_t, 1);
+    mbar_init(sm.acc_s, 1);
+    mbar_init(sm.free_t, kEpiWarps);
+    mbar_init(sm.free_s, kEpiWarps);
+    mbar_init(sm.drain, 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Producer exit: wait (bounded) for the last copy issued into every stage.
+__device__ __forceinline__ void drain_loads(const FusedSmem &sm, uint32_t issued)
+{
+    const uint32_t first = issued > STAGES ? issued - STAGES : 0;
+    for (uint32_t j = first; j < issued; ++j)
+        wait_drain(&sm.full[j % STAGES], (j / STAGES) & 1);
+}
+
+// MMA issuer exit: wait (bounded) until every tcgen05 operation it issued is done.
+__device__ __forceinline__ void drain_mma(const FusedSmem &sm)
+{
+    tc_commit(sm.drain);
+    wait_drain(sm.drain, 0);
+}
 
 // ----------------------------------------------------------------------------
 // Forward statistics (MODE 0) / backward logit gradient (MODE 1).
@@ -101,24 +159,17 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ int s_dead;
-    FusedSmem sm = carve(smem_raw);
+    FusedSmem sm = carve(smem_raw, kLmBRegion);
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
     const int nvalid = *a.nvalid;
     const int m_tiles = (nvalid + BM - 1) / BM;
     const int n_tiles = (int)((a.vocab + BN - 1) / BN);
     const int units = m_tiles * a.n_groups;
-    const int kb_s = a.d_s / BK, kb_t = a.d_t / BK, kb_tile = kb_s + kb_t;
+    const int kb_s = a.d_s / BK, kb_t = a.d_t / BK;
 
     if (threadIdx.x == 0) {
         s_dead = 0;
-        for (int s = 0; s < STAGES; ++s) {
-            mbar_init(&sm.full[s], 1);
-            mbar_init(&sm.empty[s], 1);
-        }
-        mbar_init(sm.accf, 1);
-        mbar_init(sm.acce, kEpiWarps);
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        init_barriers(sm);
     }
     if (warp == 1) {
         tmem_alloc(sm.tslot, 512);
@@ -130,7 +181,7 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
     const uint32_t tmem = *sm.tslot;
 
     if (warp == 0 && lane == 0) {
-        // ---------------- producer: k-blocks of every tile of every unit
+        // ---------------- producer: per tile the teacher k-blocks, then the student's
         tma_prefetch_desc(&tHs);
         tma_prefetch_desc(&tWs);
         tma_prefetch_desc(&tHt);
@@ -140,62 +191,69 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
             const int mt = u % m_tiles, g = u / m_tiles;
             const int t0 = g * kTilesPerGroup, t1 = min(n_tiles, t0 + kTilesPerGroup);
             for (int nt = t0; nt < t1; ++nt) {
-                for (int kb = 0; kb < kb_tile; ++kb, ++it) {
+                for (int kb = 0; kb < kb_t + kb_s; ++kb, ++it) {
                     const int s = it % STAGES;
                     if (it >= STAGES)
                         wait_lim(&sm.empty[s], ((it / STAGES) - 1) & 1, a.status, &s_dead);
                     mbar_arrive_expect_tx(&sm.full[s], STAGE_BYTES);
-                    if (kb < kb_s) {
-                        tma_load_2d(sm.a + s * A_BYTES, &tHs, kb * BK, mt * BM, &sm.full[s]);
-                        tma_load_2d(sm.b + s * B_BYTES, &tWs, kb * BK, nt * BN, &sm.full[s]);
+                    if (kb < kb_t) {
+                        tma_load_2d(sm.a + s * A_BYTES, &tHt, kb * BK, mt * BM, &sm.full[s]);
+                        tma_load_2d(sm.b + s * B_BYTES, &tWt, kb * BK, nt * BN, &sm.full[s]);
                     } else {
-                        tma_load_2d(sm.a + s * A_BYTES, &tHt, (kb - kb_s) * BK, mt * BM, &sm.full[s]);
-                        tma_load_2d(sm.b + s * B_BYTES, &tWt, (kb - kb_s) * BK, nt * BN, &sm.full[s]);
+                        tma_load_2d(sm.a + s * A_BYTES, &tHs, (kb - kb_t) * BK, mt * BM, &sm.full[s]);
+                        tma_load_2d(sm.b + s * B_BYTES, &tWs, (kb - kb_t) * BK, nt * BN, &sm.full[s]);
                     }
                 }
             }
         }
+        drain_loads(sm, it);
     } else if (warp == 1 && lane == 0) {
-        // ---------------- MMA issuer: Z_s into columns [0,256), Z_t into [256,512)
+        // ---------------- MMA issuer
         constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
         uint32_t it = 0, tile = 0;
+        auto run_k = [&](uint32_t dcol, int nkb) {
+            for (int kb = 0; kb < nkb; ++kb, ++it) {
+                const int s = it % STAGES;
+                wait_lim(&sm.full[s], (it / STAGES) & 1, a.status, &s_dead);
+                tc_fence_after();
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k) {
+                    const uint64_t ad = smem_desc_sw128(smem_u32(sm.a + s * A_BYTES) + k * 32);
+                    const uint64_t bd = smem_desc_sw128(smem_u32(sm.b + s * B_BYTES) + k * 32);
+                    tc_mma(tmem + dcol, ad, bd, idesc, kb > 0 || k > 0);
+                }
+                tc_commit(&sm.empty[s]);
+            }
+        };
         for (int u = blockIdx.x; u < units; u += gridDim.x) {
             const int g = u / m_tiles;
             const int t0 = g * kTilesPerGroup, t1 = min(n_tiles, t0 + kTilesPerGroup);
             for (int nt = t0; nt < t1; ++nt, ++tile) {
-                if (tile > 0)  // the epilogue has read the previous tile's accumulators
-                    wait_lim(sm.acce, (tile - 1) & 1, a.status, &s_dead);
+                if (tile > 0)  // the epilogue holds Z_t of the previous tile in registers
+                    wait_lim(sm.free_t, (tile - 1) & 1, a.status, &s_dead);
                 tc_fence_after();
-                for (int kb = 0; kb < kb_tile; ++kb, ++it) {
-                    const int s = it % STAGES;
-                    wait_lim(&sm.full[s], (it / STAGES) & 1, a.status, &s_dead);
-                    tc_fence_after();
-                    const bool teacher = kb >= kb_s;
-                    const uint32_t d = tmem + (teacher ? 256u : 0u);
-                    const int kk = teacher ? kb - kb_s : kb;
-#pragma unroll
-                    for (int k = 0; k < BK / 16; ++k) {
-                        const uint64_t ad = smem_desc_sw128(smem_u32(sm.a + s * A_BYTES) + k * 32);
-                        const uint64_t bd = smem_desc_sw128(smem_u32(sm.b + s * B_BYTES) + k * 32);
-                        tc_mma(d, ad, bd, idesc, kk > 0 || k > 0);
-                    }
-                    tc_commit(&sm.empty[s]);
-                }
-                tc_commit(sm.accf);
+                run_k(kColT, kb_t);
+                tc_commit(sm.acc_t);
+                if (tile > 0)  // the epilogue has read Z_s of the previous tile
+                    wait_lim(sm.free_s, (tile - 1) & 1, a.status, &s_dead);
+                tc_fence_after();
+                run_k(kColS, kb_s);
+                tc_commit(sm.acc_s);
             }
         }
+        drain_mma(sm);
     } else if (warp >= 2) {
-        // ---------------- epilogue: warp pair (q, half) owns rows q*32.. and 128 columns
+        // ---------------- epilogue: warp (q, cq) owns rows q*32.. and columns cq*64..
         const int ew = warp - 2;
-        const int q = warp % 4;             // tensor-memory lane quarter this warp may read
-        const int half = ew / 4;            // columns [half*128, half*128 + 128) of the tile
+        const int q = warp % 4;              // tensor-memory lane quarter this warp may read
+        const int cq = ew / 4;               // column slice [cq*64, cq*64 + 64) of the tile
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+        const uint32_t col0 = (uint32_t)(cq * kEpiCols);
         uint32_t tile = 0;
         for (int u = blockIdx.x; u < units; u += gridDim.x) {
             const int mt = u % m_tiles, g = u / m_tiles;
             const int t0 = g * kTilesPerGroup, t1 = min(n_tiles, t0 + kTilesPerGroup);
-            const int rloc = q * 32 + lane;
-            const int row = mt * BM + rloc;
+            const int row = mt * BM + q * 32 + lane;
             const bool valid_row = row < nvalid;
             float ms = -INFINITY, ss = 0.f, sa = 0.f, mt_ = -INFINITY, st = 0.f;
             float nl = 0.f, cp = 0.f, sg = 1.f;
@@ -204,122 +262,168 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
                 nl = c.x, cp = c.y, sg = c.z;
             }
             for (int nt = t0; nt < t1; ++nt, ++tile) {
-                wait_lim(sm.accf, tile & 1, a.status, &s_dead);
+                const int64_t vbase = (int64_t)nt * BN + col0;   // vocabulary id of column 0 here
+                const int64_t left = a.vocab - vbase;
+                const int nv = left <= 0 ? 0 : (left >= kEpiCols ? kEpiCols : (int)left);
+                // Z_t: 64 columns into registers, then release them to the next tile
+                float zt[kEpiCols];
+                wait_lim(sm.acc_t, tile & 1, a.status, &s_dead);
                 tc_fence_after();
-#pragma unroll 1
-                for (int ch = 0; ch < 4; ++ch) {
-                    const int c0 = half * 128 + ch * 32;
-                    float zs[32], zt[32];
-                    tmem_ld32(tmem + lane_off + (uint32_t)c0, zs);
-                    tmem_ld32(tmem + lane_off + 256u + (uint32_t)c0, zt);
+                tmem_ld32(tmem + lane_off + kColT + col0, *reinterpret_cast<float(*)[32]>(&zt[0]));
+                tmem_ld32(tmem + lane_off + kColT + col0 + 32, *reinterpret_cast<float(*)[32]>(&zt[32]));
+                tmem_ld_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(sm.free_t);
+                if (MODE == 0 && nv > 0) {
+                    float cmt = -INFINITY;
+#pragma unroll
+                    for (int j = 0; j < kEpiCols; ++j)
+                        if (j < nv)
+                            cmt = fmaxf(cmt, zt[j]);
+                    if (cmt > mt_) {
+                        st *= ex2((mt_ - cmt) * kLog2e);
+                        mt_ = cmt;
+                    }
+                    const float ntt = -mt_ * kLog2e;
+#pragma unroll
+                    for (int j = 0; j < kEpiCols; ++j)
+                        if (j < nv)
+                            st += ex2(fmaf(zt[j], kLog2e, ntt));
+                }
+                // Z_s: 16 columns at a time
+                wait_lim(sm.acc_s, tile & 1, a.status, &s_dead);
+                tc_fence_after();
+#pragma unroll
+                for (int ch = 0; ch < kEpiCols / 16; ++ch) {
+                    float zs[16];
+                    tmem_ld16(tmem + lane_off + kColS + col0 + ch * 16, zs);
                     tmem_ld_wait();
-                    const int64_t v0 = (int64_t)nt * BN + c0;
+                    const int c0 = ch * 16;
                     if (MODE == 0) {
-                        // online statistics over the in-vocabulary columns
-                        float cmx = -INFINITY, cmt = -INFINITY;
+                        if (c0 < nv) {
+                            float cmx = -INFINITY;
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) {
-                            if (v0 + j < a.vocab) {
-                                cmx = fmaxf(cmx, zs[j]);
-                                cmt = fmaxf(cmt, zt[j]);
+                            for (int j = 0; j < 16; ++j)
+                                if (c0 + j < nv)
+                                    cmx = fmaxf(cmx, zs[j]);
+                            if (cmx > ms) {
+                                const float f = ex2((ms - cmx) * kLog2e);
+                                ss *= f;
+                                sa *= f;
+                                ms = cmx;
+                            }
+                            const float ns = -ms * kLog2e;
+#pragma unroll
+                            for (int j = 0; j < 16; ++j) {
+                                if (c0 + j < nv) {
+                                    const float e = ex2(fmaf(zs[j], kLog2e, ns));
+                                    ss += e;
+                                    sa = fmaf(e, zs[j] - zt[c0 + j], sa);
+                                }
                             }
                         }
-                        if (cmx > ms) {
-                            const float f = ex2((ms - cmx) * kLog2e);
-                            ss *= f;
-                            sa *= f;
-                            ms = cmx;
-                        }
-                        if (cmt > mt_) {
-                            st *= ex2((mt_ - cmt) * kLog2e);
-                            mt_ = cmt;
-                        }
-                        const float ns = -ms * kLog2e, ntt = -mt_ * kLog2e;
+                    } else if (valid_row && vbase + c0 < a.vpad) {
+                        // G = w p ((z_s - z_t) - E_p[z_s - z_t]); zero beyond the vocabulary.
+                        // vpad is a multiple of 64, so a 16-column chunk is wholly inside
+                        // [0, vpad) or wholly outside it.
+                        uint32_t pk[8];
 #pragma unroll
-                        for (int j = 0; j < 32; ++j) {
-                            if (v0 + j < a.vocab) {
-                                const float e = ex2(fmaf(zs[j], kLog2e, ns));
-                                ss += e;
-                                sa = fmaf(e, zs[j] - zt[j], sa);
-                                st += ex2(fmaf(zt[j], kLog2e, ntt));
-                            }
-                        }
-                    } else if (valid_row && v0 < a.vpad) {
-                        // G = w p ((z_s - z_t) - E_p[z_s - z_t]); zero beyond the vocabulary
-                        uint32_t pk[16];
-#pragma unroll
-                        for (int j = 0; j < 32; j += 2) {
+                        for (int j = 0; j < 16; j += 2) {
                             float g0 = 0.f, g1 = 0.f;
-                            if (v0 + j < a.vocab)
-                                g0 = sg * ex2(fmaf(zs[j], kLog2e, -nl)) * ((zs[j] - zt[j]) - cp);
-                            if (v0 + j + 1 < a.vocab)
-                                g1 = sg * ex2(fmaf(zs[j + 1], kLog2e, -nl)) * ((zs[j + 1] - zt[j + 1]) - cp);
+                            if (c0 + j < nv)
+                                g0 = sg * ex2(fmaf(zs[j], kLog2e, -nl)) * ((zs[j] - zt[c0 + j]) - cp);
+                            if (c0 + j + 1 < nv)
+                                g1 = sg * ex2(fmaf(zs[j + 1], kLog2e, -nl)) *
+                                     ((zs[j + 1] - zt[c0 + j + 1]) - cp);
                             pk[j / 2] = pack_bf16x2(g0, g1);
                         }
-                        uint4 *dst = reinterpret_cast<uint4 *>(a.G + (size_t)row * a.vpad + v0);
-                        // vpad is a multiple of BK = 64, so a 32-column chunk is either
-                        // wholly inside [0, vpad) or wholly outside it
-#pragma unroll
-                        for (int j = 0; j < 4; ++j)
-                            dst[j] = make_uint4(pk[4 * j], pk[4 * j + 1], pk[4 * j + 2], pk[4 * j + 3]);
+                        uint4 *dst = reinterpret_cast<uint4 *>(a.G + (size_t)row * a.vpad + vbase + c0);
+                        dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                        dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                     }
                 }
                 tc_fence_before();
                 __syncwarp();
                 if (lane == 0)
-                    mbar_arrive(sm.acce);
+                    mbar_arrive(sm.free_s);
             }
             if (MODE == 0 && valid_row) {
-                float *pp = a.part + (((size_t)g * 2 + half) * a.cap + row) * 8;
+                float *pp = a.part + (((size_t)g * kColQuarters + cq) * a.cap + row) * 8;
                 reinterpret_cast<float4 *>(pp)[0] = make_float4(ms, ss, sa, mt_);
                 reinterpret_cast<float4 *>(pp)[1] = make_float4(st, 0.f, 0.f, 0.f);
             }
         }
     }
 
-    // drain (after a timeout, let in-flight tensor-core work finish) and release
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 1) {
-        if (lane == 0 && *(volatile int *)&s_dead) {
-            // one more bounded wait on the accumulator barrier's next phase
-            for (uint32_t i = 0; i < kLimit; ++i)
-                if (mbar_try_wait(sm.accf, 0) || mbar_try_wait(sm.accf, 1))
-                    break;
-        }
-        __syncwarp();
+    if (warp == 1)
         tmem_dealloc(tmem, 512);
-    }
 }
 
 // ----------------------------------------------------------------------------
-// dH = G W_s: A = G [rows, vpad] (K-major), B = W_s^T [d_s, vpad] (K-major).
-// Output tile 128 x 256 fp32 in tensor memory; rows scattered to their tokens.
+// dH = G W_s: A = G [rows, vpad] (K-major, K = vocabulary), B = W_s [V, d_s]
+// read in place as an MN-major operand (four 64-column TMA boxes per stage).
+// Output tile 128 x 256 fp32 in tensor memory.  Work split: the first
+// floor(tiles / P) * P tiles are whole tiles, P = grid size, one per CTA per
+// wave, written straight to their token rows; the remaining tiles' k-blocks
+// are split evenly over all P CTAs (each range covers at most two tiles) and
+// written as partial tiles, which k_dh_fixup sums in CTA order.  The result
+// is bitwise reproducible for a given grid size.
+struct DhArgs {
+    const int4 *rows;
+    const int32_t *nvalid;
+    int d_s;
+    int kbs;         // vpad / BK
+    float *dh;       // [T, d_s]
+    float *partial;  // [P][2][BM][BN]
+    int32_t *status;
+};
+
+struct DhSeg {
+    int tile, k0, k1, slot;  // slot -1: whole tile; 0/1: partial slot of this CTA
+};
+
+template <class F>
+__device__ __forceinline__ void dh_segments(int tiles, int kbs, F &&f)
+{
+    const int P = gridDim.x, c = blockIdx.x;
+    const int full = tiles / P * P;
+    for (int t = c; t < full; t += P)
+        f(DhSeg{t, 0, kbs, -1});
+    const int rem = tiles - full;
+    if (rem > 0) {
+        const int64_t total = (int64_t)rem * kbs;
+        const int64_t b = total * c / P, e = total * (c + 1) / P;
+        int slot = 0;
+        for (int64_t it = b; it < e;) {
+            const int j = (int)(it / kbs), k0 = (int)(it % kbs);
+            const int64_t k1l = k0 + (e - it);
+            const int k1 = k1l < kbs ? (int)k1l : kbs;
+            f(DhSeg{full + j, k0, k1, slot++});
+            it += k1 - k0;
+        }
+    }
+}
+
 __global__ void __launch_bounds__(kThreads, 1)
-k_fused_dh(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUtensorMap tWT, const int4 *rows,
-           const int32_t *nvalid_p, int d_s, int64_t vpad, float *dh_out, int32_t *status)
+k_fused_dh(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUtensorMap tW, DhArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ int s_dead;
-    FusedSmem sm = carve(smem_raw);
+    FusedSmem sm = carve(smem_raw, kDhBRegion);
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
-    const int nvalid = *nvalid_p;
+    const int nvalid = *a.nvalid;
     const int m_tiles = (nvalid + BM - 1) / BM;
-    const int n_tiles = d_s / BN;
+    const int n_tiles = a.d_s / BN;
     const int tiles = m_tiles * n_tiles;
-    const int kbs = (int)(vpad / BK);
 
     if (threadIdx.x == 0) {
         s_dead = 0;
-        for (int s = 0; s < STAGES; ++s) {
-            mbar_init(&sm.full[s], 1);
-            mbar_init(&sm.empty[s], 1);
-        }
-        mbar_init(sm.accf, 1);
-        mbar_init(sm.acce, kEpiWarps);
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        init_barriers(sm);
     }
     if (warp == 1) {
         tmem_alloc(sm.tslot, 256);
@@ -330,84 +434,129 @@ k_fused_dh(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
     tc_fence_after();
     const uint32_t tmem = *sm.tslot;
 
-    // tile order: N-tile fastest, so CTAs running together share the G rows (A)
+    // whole tiles: N-tile fastest, so the CTAs of one wave share the G rows (A)
     if (warp == 0 && lane == 0) {
         tma_prefetch_desc(&tG);
-        tma_prefetch_desc(&tWT);
+        tma_prefetch_desc(&tW);
         uint32_t it = 0;
-        for (int t = blockIdx.x; t < tiles; t += gridDim.x) {
-            const int mt = t / n_tiles, nt = t % n_tiles;
-            for (int kb = 0; kb < kbs; ++kb, ++it) {
+        dh_segments(tiles, a.kbs, [&](const DhSeg &sg) {
+            const int mt = sg.tile / n_tiles, nt = sg.tile % n_tiles;
+            for (int kb = sg.k0; kb < sg.k1; ++kb, ++it) {
                 const int s = it % STAGES;
                 if (it >= STAGES)
-                    wait_lim(&sm.empty[s], ((it / STAGES) - 1) & 1, status, &s_dead);
+                    wait_lim(&sm.empty[s], ((it / STAGES) - 1) & 1, a.status, &s_dead);
                 mbar_arrive_expect_tx(&sm.full[s], STAGE_BYTES);
                 tma_load_2d(sm.a + s * A_BYTES, &tG, kb * BK, mt * BM, &sm.full[s]);
-                tma_load_2d(sm.b + s * B_BYTES, &tWT, kb * BK, nt * BN, &sm.full[s]);
+#pragma unroll
+                for (int j = 0; j < BN / 64; ++j)
+                    tma_load_2d(sm.b + s * B_BYTES + j * (B_BYTES / 4), &tW, nt * BN + j * 64, kb * BK,
+                                &sm.full[s]);
             }
-        }
+        });
+        drain_loads(sm, it);
     } else if (warp == 1 && lane == 0) {
-        constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+        constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, true);
         uint32_t it = 0, tile = 0;
-        for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++tile) {
+        dh_segments(tiles, a.kbs, [&](const DhSeg &sg) {
             if (tile > 0)
-                wait_lim(sm.acce, (tile - 1) & 1, status, &s_dead);
+                wait_lim(sm.free_s, (tile - 1) & 1, a.status, &s_dead);
             tc_fence_after();
-            for (int kb = 0; kb < kbs; ++kb, ++it) {
+            for (int kb = sg.k0; kb < sg.k1; ++kb, ++it) {
                 const int s = it % STAGES;
-                wait_lim(&sm.full[s], (it / STAGES) & 1, status, &s_dead);
+                wait_lim(&sm.full[s], (it / STAGES) & 1, a.status, &s_dead);
                 tc_fence_after();
 #pragma unroll
                 for (int k = 0; k < BK / 16; ++k) {
                     const uint64_t ad = smem_desc_sw128(smem_u32(sm.a + s * A_BYTES) + k * 32);
-                    const uint64_t bd = smem_desc_sw128(smem_u32(sm.b + s * B_BYTES) + k * 32);
-                    tc_mma(tmem, ad, bd, idesc, kb > 0 || k > 0);
+                    // 16 K-rows of 128 B per step; 64-wide N blocks 8 KB apart; 8-row atoms 1 KB apart
+                    const uint64_t bd = smem_desc_sw128_mn(smem_u32(sm.b + s * B_BYTES) + k * 2048,
+                                                           B_BYTES / 4, 1024);
+                    tc_mma(tmem, ad, bd, idesc, kb > sg.k0 || k > 0);
                 }
                 tc_commit(&sm.empty[s]);
             }
-            tc_commit(sm.accf);
-        }
+            tc_commit(sm.acc_s);
+            ++tile;
+        });
+        drain_mma(sm);
     } else if (warp >= 2) {
-        const int ew = warp - 2, q = warp % 4, half = ew / 4;
+        const int ew = warp - 2, q = warp % 4, cq = ew / 4;
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+        const int col0 = cq * kEpiCols;
+        const int rloc = q * 32 + lane;
         uint32_t tile = 0;
-        for (int t = blockIdx.x; t < tiles; t += gridDim.x, ++tile) {
-            const int mt = t / n_tiles, nt = t % n_tiles;
-            const int row = mt * BM + q * 32 + lane;
-            wait_lim(sm.accf, tile & 1, status, &s_dead);
+        dh_segments(tiles, a.kbs, [&](const DhSeg &sg) {
+            const int mt = sg.tile / n_tiles, nt = sg.tile % n_tiles;
+            const int row = mt * BM + rloc;
+            wait_lim(sm.acc_s, tile & 1, a.status, &s_dead);
             tc_fence_after();
             const bool valid = row < nvalid;
-            const int token = valid ? rows[row].x : 0;
+            float *dst = nullptr;
+            if (valid) {
+                if (sg.slot < 0)
+                    dst = a.dh + (size_t)a.rows[row].x * a.d_s + nt * BN + col0;
+                else
+                    dst = a.partial + (((size_t)blockIdx.x * 2 + sg.slot) * BM + rloc) * BN + col0;
+            }
 #pragma unroll 1
-            for (int ch = 0; ch < 4; ++ch) {
-                const int c0 = half * 128 + ch * 32;
+            for (int ch = 0; ch < kEpiCols / 32; ++ch) {
                 float v[32];
-                tmem_ld32(tmem + lane_off + (uint32_t)c0, v);
+                tmem_ld32(tmem + lane_off + (uint32_t)(col0 + ch * 32), v);
                 tmem_ld_wait();
                 if (valid) {
-                    float4 *dst = reinterpret_cast<float4 *>(dh_out + (size_t)token * d_s + nt * BN + c0);
+                    float4 *d4 = reinterpret_cast<float4 *>(dst + ch * 32);
 #pragma unroll
                     for (int j = 0; j < 8; ++j)
-                        dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                        d4[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
                 }
             }
             tc_fence_before();
             __syncwarp();
             if (lane == 0)
-                mbar_arrive(sm.acce);
-        }
+                mbar_arrive(sm.free_s);
+            ++tile;
+        });
     }
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 1) {
-        if (lane == 0 && *(volatile int *)&s_dead) {
-            for (uint32_t i = 0; i < kLimit; ++i)
-                if (mbar_try_wait(sm.accf, 0) || mbar_try_wait(sm.accf, 1))
-                    break;
-        }
-        __syncwarp();
+    if (warp == 1)
         tmem_dealloc(tmem, 256);
+}
+
+// Sum the partial tiles of the split part of dH in CTA order (P = the dH grid
+// size) and write them to their token rows.
+__global__ void k_dh_fixup(const float *__restrict__ partial, const int4 *__restrict__ rows,
+                           const int32_t *__restrict__ nvalid_p, int d_s, int kbs, int P, float *__restrict__ dh)
+{
+    const int nvalid = *nvalid_p;
+    const int n_tiles = d_s / BN;
+    const int tiles = (nvalid + BM - 1) / BM * n_tiles;
+    const int full = tiles / P * P;
+    const int rem = tiles - full;
+    const int64_t total = (int64_t)rem * kbs;
+    for (int j = blockIdx.x; j < rem; j += gridDim.x) {
+        const int t = full + j, mt = t / n_tiles, nt = t % n_tiles;
+        const int64_t lo = (int64_t)j * kbs, hi = lo + kbs;
+        // CTAs whose non-empty k-block range meets [lo, hi)
+        const int64_t c_lo_l = lo * P / total - 1, c_hi_l = hi * P / total + 1;
+        const int c_lo = c_lo_l < 0 ? 0 : (int)c_lo_l;
+        const int c_hi = c_hi_l > P - 1 ? P - 1 : (int)c_hi_l;
+        for (int e = threadIdx.x; e < BM * BN; e += blockDim.x) {
+            const int r = e / BN, col = e % BN;
+            const int row = mt * BM + r;
+            if (row >= nvalid)
+                continue;
+            float acc = 0.f;
+            for (int c = c_lo; c <= c_hi; ++c) {
+                const int64_t b = total * c / P, en = total * (c + 1) / P;
+                if (b >= en || en <= lo || b >= hi)
+                    continue;
+                const int slot = (b / kbs == j) ? 0 : 1;
+                acc += partial[(((size_t)c * 2 + slot) * BM + r) * BN + col];
+            }
+            dh[(size_t)rows[row].x * d_s + nt * BN + col] = acc;
+        }
     }
 }
 
@@ -426,27 +575,6 @@ __global__ void k_gather_rows(const int4 *__restrict__ rows, const int32_t *__re
     }
 }
 
-// W [V, d] -> W^T [d, vpad], zero for columns v >= V (32 x 32 tiles).
-__global__ void k_transpose_pad(const __nv_bfloat16 *__restrict__ W, int64_t V, int d, int64_t vpad,
-                                __nv_bfloat16 *__restrict__ WT)
-{
-    __shared__ __nv_bfloat16 tile[32][34];
-    const int64_t v0 = (int64_t)blockIdx.x * 32;
-    const int c0 = blockIdx.y * 32;
-    for (int r = threadIdx.y; r < 32; r += blockDim.y) {
-        const int64_t v = v0 + r;
-        const int c = c0 + threadIdx.x;
-        tile[r][threadIdx.x] = (v < V && c < d) ? W[v * d + c] : __float2bfloat16(0.f);
-    }
-    __syncthreads();
-    for (int r = threadIdx.y; r < 32; r += blockDim.y) {
-        const int c = c0 + r;
-        const int64_t v = v0 + threadIdx.x;
-        if (c < d && v < vpad)
-            WT[(int64_t)c * vpad + v] = tile[threadIdx.x][r];
-    }
-}
-
 // Per supervised row: merge the vocabulary-group partials into LSE_s, LSE_t,
 // KL; write l, w*l and the backward constants.
 __global__ void k_fused_merge(const int4 *__restrict__ rows, const int32_t *__restrict__ nvalid,
@@ -458,7 +586,7 @@ __global__ void k_fused_merge(const int4 *__restrict__ rows, const int32_t *__re
     for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < n; j += gridDim.x * blockDim.x) {
         Student S = student_empty();
         Teacher T = teacher_empty();
-        for (int gh = 0; gh < 2 * n_groups; ++gh) {
+        for (int gh = 0; gh < kColQuarters * n_groups; ++gh) {
             const float *pp = part + ((size_t)gh * cap + j) * 8;
             const float4 x = reinterpret_cast<const float4 *>(pp)[0];
             const float4 y = reinterpret_cast<const float4 *>(pp)[1];
@@ -498,14 +626,16 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn()
     return fn;
 }
 
-bool make_map(CUtensorMap *m, const void *base, int64_t rows, int64_t cols, int box_rows)
+// 2-D bf16 tensor map over a row-major [rows, cols] matrix, 128-byte swizzle,
+// box of box_cols (128 B) x box_rows; rows beyond the matrix read as zero.
+bool make_map(CUtensorMap *m, const void *base, int64_t rows, int64_t cols, int box_rows, int box_cols)
 {
     auto fn = encode_fn();
     if (!fn)
         return false;
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
     cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
-    cuuint32_t box[2] = {BK, (cuuint32_t)box_rows};
+    cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
     cuuint32_t es[2] = {1, 1};
     return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -516,12 +646,12 @@ struct FusedLayout {
     int4 *rows;
     int32_t *blk_count, *nvalid;
     double *row_wl;
-    __nv_bfloat16 *hs, *ht, *G, *wsT;
-    float *part, *rowc;
+    __nv_bfloat16 *hs, *ht, *G;
+    float *part, *rowc, *dh_partial;
     size_t bytes;
 };
 
-FusedLayout fused_layout(void *ws, int64_t T, int64_t V, int64_t d_s, int64_t d_t, int n_groups)
+FusedLayout fused_layout(void *ws, int64_t T, int64_t V, int64_t d_s, int64_t d_t, int n_groups, int sms)
 {
     const int64_t vpad = (V + BK - 1) / BK * BK;
     const int64_t cap = (T + BM - 1) / BM * BM;
@@ -540,10 +670,10 @@ FusedLayout fused_layout(void *ws, int64_t T, int64_t V, int64_t d_s, int64_t d_
     L.row_wl = reinterpret_cast<double *>(take(sizeof(double) * (size_t)T));
     L.hs = reinterpret_cast<__nv_bfloat16 *>(take(2 * (size_t)cap * d_s));
     L.ht = reinterpret_cast<__nv_bfloat16 *>(take(2 * (size_t)cap * d_t));
-    L.part = reinterpret_cast<float *>(take(sizeof(float) * 8 * 2 * (size_t)n_groups * cap));
+    L.part = reinterpret_cast<float *>(take(sizeof(float) * 8 * kColQuarters * (size_t)n_groups * cap));
     L.rowc = reinterpret_cast<float *>(take(sizeof(float) * 4 * (size_t)cap));
     L.G = reinterpret_cast<__nv_bfloat16 *>(take(2 * (size_t)cap * vpad));
-    L.wsT = reinterpret_cast<__nv_bfloat16 *>(take(2 * (size_t)d_s * vpad));
+    L.dh_partial = reinterpret_cast<float *>(take(sizeof(float) * (size_t)sms * 2 * BM * BN));
     L.bytes = off + 256;
     return L;
 }
@@ -554,16 +684,16 @@ int groups_for(int64_t V) { return (int)(((V + BN - 1) / BN + kTilesPerGroup - 1
 
 size_t fused_workspace_bytes(int64_t T, int64_t V, int64_t d_s, int64_t d_t)
 {
-    return fused_layout(nullptr, T, V, d_s, d_t, groups_for(V)).bytes;
+    return fused_layout(nullptr, T, V, d_s, d_t, groups_for(V), device_sm_count()).bytes;
 }
 
 cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream)
 {
     const int n_groups = groups_for(c.vocab);
-    FusedLayout L = fused_layout(c.workspace, c.T, c.vocab, c.d_s, c.d_t, n_groups);
+    const int sms = device_sm_count();
+    FusedLayout L = fused_layout(c.workspace, c.T, c.vocab, c.d_s, c.d_t, n_groups, sms);
     const int64_t vpad = (c.vocab + BK - 1) / BK * BK;
     const int64_t cap = (c.T + BM - 1) / BM * BM;
-    const int sms = device_sm_count();
 
     // supervised rows (the compaction of the loss path), then the gathered hidden rows
     LossArgs la{};
@@ -582,19 +712,16 @@ cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream)
                                                reinterpret_cast<uint4 *>(L.hs));
     k_gather_rows<<<sms * 4, 256, 0, stream>>>(L.rows, L.nvalid, static_cast<const uint4 *>(c.h_t), c.d_t / 8,
                                                reinterpret_cast<uint4 *>(L.ht));
-    {
-        dim3 grid((unsigned)((vpad + 31) / 32), (unsigned)((c.d_s + 31) / 32));
-        k_transpose_pad<<<grid, dim3(32, 8), 0, stream>>>(static_cast<const __nv_bfloat16 *>(c.W_s), c.vocab,
-                                                          (int)c.d_s, vpad, L.wsT);
-    }
     e = cudaGetLastError();
     if (e != cudaSuccess)
         return e;
 
-    alignas(64) CUtensorMap tHs, tWs, tHt, tWt, tG, tWT;
-    if (!make_map(&tHs, L.hs, cap, c.d_s, BM) || !make_map(&tWs, c.W_s, c.vocab, c.d_s, BN) ||
-        !make_map(&tHt, L.ht, cap, c.d_t, BM) || !make_map(&tWt, c.W_t, c.vocab, c.d_t, BN) ||
-        !make_map(&tG, L.G, cap, vpad, BM) || !make_map(&tWT, L.wsT, c.d_s, vpad, BN))
+    alignas(64) CUtensorMap tHs, tWs, tHt, tWt, tG, tWmn;
+    if (!make_map(&tHs, L.hs, cap, c.d_s, BM, BK) || !make_map(&tWs, c.W_s, c.vocab, c.d_s, BN, BK) ||
+        !make_map(&tHt, L.ht, cap, c.d_t, BM, BK) || !make_map(&tWt, c.W_t, c.vocab, c.d_t, BN, BK) ||
+        !make_map(&tG, L.G, cap, vpad, BM, BK) ||
+        // W_s as the MN-major B of dH: boxes of 64 d-columns x BK vocabulary rows
+        !make_map(&tWmn, c.W_s, c.vocab, c.d_s, BK, 64))
         return cudaErrorInvalidValue;
 
     static bool attr_done = false;
@@ -603,7 +730,7 @@ cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream)
         if (e == cudaSuccess)
             e = cudaFuncSetAttribute(k_fused_lm<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedSmem);
         if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(k_fused_dh, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedSmem);
+            e = cudaFuncSetAttribute(k_fused_dh, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDhSmem);
         if (e != cudaSuccess)
             return e;
         attr_done = true;
@@ -632,8 +759,16 @@ cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream)
     if (c.dh_s) {
         k_fused_lm<1><<<sms, kThreads, kFusedSmem, stream>>>(tHs, tWs, tHt, tWt, fa);
         launch_zero_masked_f32(c.mask, c.T, (int64_t)c.d_s, c.dh_s, stream);
-        k_fused_dh<<<sms, kThreads, kFusedSmem, stream>>>(tG, tWT, L.rows, L.nvalid, (int)c.d_s, vpad, c.dh_s,
-                                                         c.status);
+        DhArgs da;
+        da.rows = L.rows;
+        da.nvalid = L.nvalid;
+        da.d_s = (int)c.d_s;
+        da.kbs = (int)(vpad / BK);
+        da.dh = c.dh_s;
+        da.partial = L.dh_partial;
+        da.status = c.status;
+        k_fused_dh<<<sms, kThreads, kDhSmem, stream>>>(tG, tWmn, da);
+        k_dh_fixup<<<sms, 256, 0, stream>>>(L.dh_partial, L.rows, L.nvalid, (int)c.d_s, da.kbs, sms, c.dh_s);
     }
     launch_loss_sum(L.row_wl, L.nvalid, c.loss, c.status, stream);
     return cudaGetLastError();

@@ -175,13 +175,28 @@ __device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr)
            | ((uint64_t)2 << 61);               // 128-byte swizzle
 }
 
+// Shared-memory matrix descriptor of an MN-major operand tile (the N index
+// contiguous) laid out by 128-byte-swizzled TMA boxes of 64 N-values x BK
+// K-rows: each K index is one 128-byte row, 8-row atoms are `sbo` bytes apart
+// along K, and 64-wide N blocks are `lbo` bytes apart.  `saddr` advances by
+// 2048 B (16 K-rows) per K=16 step and stays 1024-byte aligned.
+__device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t saddr, uint32_t lbo, uint32_t sbo)
+{
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4)
+           | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16)
+           | ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32)
+           | ((uint64_t)1 << 46)
+           | ((uint64_t)2 << 61);
+}
+
 // Instruction descriptor of kind::f16 with bf16 A and B (both K-major) and an
-// fp32 accumulator, for an M x N tile.
-__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N)
+// fp32 accumulator, for an M x N tile.  `b_mn_major` selects an MN-major B.
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool b_mn_major = false)
 {
     return (1u << 4)                      // D: fp32
            | (1u << 7)                    // A: bf16
            | (1u << 10)                   // B: bf16
+           | ((b_mn_major ? 1u : 0u) << 16)  // B major-ness (0: K-major, 1: MN-major)
            | ((uint32_t)(N >> 3) << 17)   // N / 8
            | ((uint32_t)(M >> 4) << 24);  // M / 16
 }
@@ -220,6 +235,19 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32])
           "=f"(v[14]), "=f"(v[15]), "=f"(v[16]), "=f"(v[17]), "=f"(v[18]), "=f"(v[19]), "=f"(v[20]),
           "=f"(v[21]), "=f"(v[22]), "=f"(v[23]), "=f"(v[24]), "=f"(v[25]), "=f"(v[26]), "=f"(v[27]),
           "=f"(v[28]), "=f"(v[29]), "=f"(v[30]), "=f"(v[31])
+        : "r"(taddr)
+        : "memory");
+}
+
+// 16 consecutive fp32 columns of this thread's tensor-memory lane.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16])
+{
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, "
+        "%12, %13, %14, %15}, [%16];"
+        : "=f"(v[0]), "=f"(v[1]), "=f"(v[2]), "=f"(v[3]), "=f"(v[4]), "=f"(v[5]), "=f"(v[6]),
+          "=f"(v[7]), "=f"(v[8]), "=f"(v[9]), "=f"(v[10]), "=f"(v[11]), "=f"(v[12]), "=f"(v[13]),
+          "=f"(v[14]), "=f"(v[15])
         : "r"(taddr)
         : "memory");
 }

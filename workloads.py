@@ -159,10 +159,10 @@ def multihop(seed: int = 0, num_traj: int = 64, min_len: int = 512, max_len: int
     return _from_spans(f"multihop_{num_traj}", out, max_turns=12)
 
 
-def fused(seed: int = 0) -> Batch:
+def fused(seed: int = 0, num_traj: int = 8, traj_len: int = 2048) -> Batch:
     """Fused LM-head case: 8 x 2048 tokens with the packed-batch turn structure."""
-    b = packed(seed, num_traj=8, traj_len=2048)
-    b.name = "fused_8x2048"
+    b = packed(seed, num_traj=num_traj, traj_len=traj_len)
+    b.name = f"fused_{num_traj}x{traj_len}"
     return b
 
 
