@@ -3,9 +3,9 @@
 // in the epilogue, never stored.
 //
 //   forward   Z_t = H_t W_t^T (K = d_t), then Z_s = H_s W_s^T (K = d_s), per
-//             128-row x 256-vocab tile, accumulated in tensor memory (512 fp32
-//             columns: Z_t in [0,256), Z_s in [256,512)); the epilogue folds
-//             each tile into per-row online statistics (max, sum exp,
+//             256-row x 256-vocab tile, accumulated in tensor memory (512 fp32
+//             columns per CTA: Z_t in [0,256), Z_s in [256,512)); the epilogue
+//             folds each tile into per-row online statistics (max, sum exp,
 //             sum exp (z_s - z_t)) for both models over a group of tiles;
 //   merge     per row: LSE_s, LSE_t, KL = E_p[z_s - z_t] - (LSE_s - LSE_t);
 //   backward  the same tiles are recomputed; the epilogue forms
@@ -14,18 +14,23 @@
 //   dH_s      = G W_s by a second tensor-core GEMM over the vocabulary, W_s read
 //             in place as an MN-major operand.
 //
-// GEMM structure (persistent, one CTA per SM): warp 0 streams 128x64 A and
-// 256x64 B bf16 tiles with TMA (128-byte swizzle) into a 4-stage ring, warp 1
-// allocates tensor memory and issues tcgen05.mma (one thread), warps 2..17
-// read the accumulator back (tcgen05.ld) for the epilogue.  The two halves of
-// the accumulator are released separately: the epilogue copies Z_t of tile j
-// into registers while Z_s of tile j is computed, and reads Z_s of tile j
-// while Z_t of tile j+1 is computed, so the tensor pipe does not wait for the
-// epilogue.  Hand-offs are mbarriers completed by TMA transaction counts,
-// tcgen05.commit and epilogue-warp arrivals.  Every wait is bounded; on
-// timeout the kernel records TURNOPD_ERR_TIMEOUT, keeps its hand-off sequence
-// without waiting, drains its own in-flight copies and tensor-core work with
-// bounded waits, and releases its tensor memory before it exits.
+// GEMM structure: persistent 2-CTA clusters, one CTA per SM.  A tile is
+// computed by the pair with cta_group::2 instructions (M = 256, N = 256): each
+// CTA stages its own 128 rows of A and 128 rows of B per 64-deep k-block, so a
+// pair reads 2/3 of the operand bytes two independent 128 x 256 tiles would.
+// In each CTA warp 0 streams the operand tiles with TMA (128-byte swizzle)
+// into a 4-stage ring, every copy counted on the even CTA's barrier; warp 1
+// allocates tensor memory, and in the even CTA one thread issues tcgen05.mma
+// and multicasts its commits to both CTAs; warps 2..17 read this CTA's 128
+// accumulator rows back (tcgen05.ld) for the epilogue.  The two halves of the
+// accumulator are released separately: the epilogue copies Z_t of tile j into
+// registers while Z_s of tile j is computed, and reads Z_s of tile j while Z_t
+// of tile j+1 is computed.  The backward epilogue stages each warp's 32 x 64
+// block of G in shared memory (128-byte swizzle) and writes it with a TMA
+// store, so G leaves the SM in whole 128-byte rows.  Every wait is bounded; on timeout the kernel
+// records TURNOPD_ERR_TIMEOUT, keeps its hand-off sequence without waiting,
+// drains its in-flight copies and tensor-core work with bounded waits, and
+// releases its tensor memory before it exits.
 
 #include <cudaTypedefs.h>
 
@@ -38,8 +43,22 @@
 namespace turnopd {
 namespace {
 
-constexpr int BM = 128, BN = 256, BK = 64, STAGES = 4;
-constexpr int A_BYTES = BM * BK * 2, B_BYTES = BN * BK * 2, STAGE_BYTES = A_BYTES + B_BYTES;
+constexpr int BM = 128;             // accumulator rows per CTA
+constexpr int BMP = 2 * BM;         // rows per pair tile
+constexpr int BN = 256;             // columns per pair tile
+constexpr int BNH = BN / 2;         // B rows staged per CTA
+#ifndef TURNOPD_FUSED_STAGES
+#define TURNOPD_FUSED_STAGES 4
+#endif
+// L2 prefetch distance of the B operand in k-blocks (0: none).  Measured on
+// GB300 it slows the GEMMs (the extra tensor requests compete with the ring's
+// own copies), so it is off.
+#ifndef TURNOPD_FUSED_PF
+#define TURNOPD_FUSED_PF 0
+#endif
+constexpr int BK = 64, STAGES = TURNOPD_FUSED_STAGES;
+constexpr int kPrefetch = TURNOPD_FUSED_PF;   // k-blocks of B brought into L2 ahead of the ring
+constexpr int A_BYTES = BM * BK * 2, B_BYTES = BNH * BK * 2, STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int kEpiWarps = 16;                    // 4 per tensor-memory lane quarter
 constexpr int kColQuarters = kEpiWarps / 4;      // column slices of a tile
 constexpr int kEpiCols = BN / kColQuarters;      // 64 columns per epilogue thread
@@ -47,6 +66,7 @@ constexpr int kThreads = 32 * (2 + kEpiWarps);
 constexpr uint32_t kLimit = 1u << 24;
 constexpr int kTilesPerGroup = 10;  // vocabulary tiles one work unit folds into one partial
 constexpr uint32_t kColT = 0, kColS = 256;  // tensor-memory columns of Z_t and Z_s
+constexpr uint16_t kPairMask = 0x3;
 
 struct FusedArgs {
     int64_t vocab;
@@ -56,18 +76,19 @@ struct FusedArgs {
     const int32_t *nvalid;
     int n_groups;          // vocabulary groups (units per M tile)
     float *part;           // [n_groups][kColQuarters][cap rows][8] partial statistics
-    int64_t cap;           // row capacity of the gathered buffers
+    int64_t cap;           // row capacity of the gathered buffers (multiple of BMP)
     const float *rowc;     // [cap][4]: lse_s * log2e - log2 |w|, E_p[z_s - z_t], sign w, -
     __nv_bfloat16 *G;      // [cap][vpad] backward output
     int32_t *status;
 };
 
-__device__ __forceinline__ bool wait_lim(uint64_t *bar, uint32_t parity, int32_t *status, int *dead)
+__device__ __forceinline__ bool wait_lim(uint64_t *bar, uint32_t parity, int32_t *status, int *dead,
+                                         bool cluster_scope = false)
 {
     if (*(volatile int *)dead)
         return false;
     for (uint32_t i = 0; i < kLimit; ++i)
-        if (mbar_try_wait(bar, parity))
+        if (cluster_scope ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity))
             return true;
     *(volatile int *)dead = 1;
     set_status(status, TURNOPD_ERR_TIMEOUT);
@@ -78,27 +99,31 @@ __device__ __forceinline__ bool wait_lim(uint64_t *bar, uint32_t parity, int32_t
 __device__ __forceinline__ void wait_drain(uint64_t *bar, uint32_t parity)
 {
     for (uint32_t i = 0; i < kLimit; ++i)
-        if (mbar_try_wait(bar, parity))
+        if (mbar_try_wait_cluster(bar, parity))
             return;
 }
 
-// Shared memory: ring of STAGES x (A tile | B tile), then barriers.
+// Shared memory: ring of STAGES x (A tile | B half tile), then barriers.  The
+// layout is identical in both CTAs of a pair (the tensor-core instructions
+// address the peer's operands at the issuing CTA's offsets).
 struct FusedSmem {
     uint8_t *a, *b;
+    uint8_t *stg;               // backward: per-epilogue-warp 32 x 64 bf16 G staging (4 KB each)
     uint64_t *full, *empty;
     uint64_t *acc_t, *acc_s;    // tensor core -> epilogue: Z_t / Z_s of a tile complete
-    uint64_t *free_t, *free_s;  // epilogue -> tensor core: Z_t / Z_s columns read
+    uint64_t *free_t, *free_s;  // epilogue (both CTAs) -> tensor core: columns read
     uint64_t *drain;
     uint32_t *tslot;
 };
 
-__device__ __forceinline__ FusedSmem carve(uint8_t *raw, int b_bytes_padded)
+__device__ __forceinline__ FusedSmem carve(uint8_t *raw, int b_region, int stg_bytes)
 {
     FusedSmem s;
     uint8_t *base = raw + ((1024 - (smem_u32(raw) & 1023)) & 1023);
     s.a = base;
     s.b = base + STAGES * A_BYTES;
-    s.full = reinterpret_cast<uint64_t *>(s.b + b_bytes_padded);
+    s.stg = s.b + b_region;
+    s.full = reinterpret_cast<uint64_t *>(s.stg + stg_bytes);
     s.empty = s.full + STAGES;
     s.acc_t = s.empty + STAGES;
     s.acc_s = s.acc_t + 1;
@@ -110,10 +135,13 @@ __device__ __forceinline__ FusedSmem carve(uint8_t *raw, int b_bytes_padded)
 }
 
 constexpr int kLmBRegion = STAGES * B_BYTES;
-// The dH kernel reads B as an MN-major operand; 32 KB of slack after the ring
+constexpr int kStgWarpBytes = 32 * kEpiCols * 2;             // 32 rows x 128 B
+constexpr int kStgBytes = kEpiWarps * kStgWarpBytes;          // 64 KB
+// The dH kernel reads B as an MN-major operand; 16 KB of slack after the ring
 // keeps every address its descriptors can form inside the allocation.
-constexpr int kDhBRegion = STAGES * B_BYTES + 32768;
-constexpr size_t kFusedSmem = STAGES * A_BYTES + kLmBRegion + 1024 + 256;
+constexpr int kDhBRegion = STAGES * B_BYTES + 16384;
+constexpr size_t kFusedSmem = STAGES * A_BYTES + kLmBRegion + kStgBytes + 1024 + 256;
+static_assert(kFusedSmem <= 232448, "shared memory per CTA");
 constexpr size_t kDhSmem = STAGES * A_BYTES + kDhBRegion + 1024 + 256;
 static_assert(kDhSmem <= 232448, "shared memory per CTA");
 
@@ -125,60 +153,112 @@ __device__ __forceinline__ void init_barriers(const FusedSmem &sm)
     }
     mbar_init(sm.acc_t, 1);
     mbar_init(sm.acc_s, 1);
-    mbar_init(sm.free_t, kEpiWarps);
-    mbar_init(sm.free_s, kEpiWarps);
+    mbar_init(sm.free_t, 2 * kEpiWarps);
+    mbar_init(sm.free_s, 2 * kEpiWarps);
     mbar_init(sm.drain, 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// Producer exit: wait (bounded) for the last copy issued into every stage.
-__device__ __forceinline__ void drain_loads(const FusedSmem &sm, uint32_t issued)
+// Common prologue: barriers, tensor memory for the pair, cluster-wide visibility.
+__device__ __forceinline__ uint32_t pair_prologue(const FusedSmem &sm, int *s_dead, uint32_t ncols)
 {
-    const uint32_t first = issued > STAGES ? issued - STAGES : 0;
-    for (uint32_t j = first; j < issued; ++j)
-        wait_drain(&sm.full[j % STAGES], (j / STAGES) & 1);
+    const int warp = threadIdx.x / 32;
+    if (threadIdx.x == 0) {
+        *s_dead = 0;
+        init_barriers(sm);
+    }
+    if (warp == 1) {
+        tmem_alloc_pair(sm.tslot, ncols);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();
+    tc_fence_after();
+    return *sm.tslot;
 }
 
-// MMA issuer exit: wait (bounded) until every tcgen05 operation it issued is done.
-__device__ __forceinline__ void drain_mma(const FusedSmem &sm)
+// Producer exit (both CTAs): wait (bounded) until the tensor core has released
+// the last copy of every stage, so no multicast commit is still on its way to
+// this CTA's barriers; the even CTA also waits for its full barriers, which
+// count the copies of both CTAs.
+__device__ __forceinline__ void drain_producer(const FusedSmem &sm, uint32_t issued, uint32_t rank)
 {
-    tc_commit(sm.drain);
-    wait_drain(sm.drain, 0);
+    const uint32_t first = issued > STAGES ? issued - STAGES : 0;
+    for (uint32_t j = first; j < issued; ++j) {
+        if (rank == 0)
+            wait_drain(&sm.full[j % STAGES], (j / STAGES) & 1);
+        wait_drain(&sm.empty[j % STAGES], (j / STAGES) & 1);
+    }
+}
+
+// Epilogue -> tensor core: this warp has finished reading a half of the accumulator.
+__device__ __forceinline__ void release_cols(uint32_t bar_leader, int lane)
+{
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0)
+        mbar_arrive_cluster(bar_leader);
+}
+
+// Common epilogue of the kernels: every tcgen05 operation of the pair is
+// complete (drain barrier in both CTAs) before tensor memory is released.
+__device__ __forceinline__ void pair_epilogue(const FusedSmem &sm, uint32_t tmem, uint32_t ncols, uint32_t rank)
+{
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    if (warp == 1 && lane == 0) {
+        if (rank == 0)
+            tc_commit_pair(sm.drain, kPairMask);
+        wait_drain(sm.drain, 0);
+    }
+    tc_fence_before();
+    __syncthreads();
+    cluster_sync();
+    tc_fence_after();
+    if (warp == 1)
+        tmem_dealloc_pair(tmem, ncols);
+}
+
+// Work unit u -> (pair M tile, vocabulary group).  The M tiles are cut into
+// blocks of at most kMBlock; the units of a block are enumerated group-major,
+// so the pairs running side by side share the H rows of one block and the W
+// tiles of a few groups: a working set of about (kMBlock + pairs / kMBlock)
+// 4.7 MB operand panels, which stays in L2.
+constexpr int kMBlock = 16;
+__device__ __forceinline__ void unit_coords(int u, int m_tiles, int n_groups, int *mt, int *g)
+{
+    const int nb = (m_tiles + kMBlock - 1) / kMBlock;
+    const int mb = (m_tiles + nb - 1) / nb;          // block height (last block may be shorter)
+    const int b = u / (mb * n_groups);
+    const int rest = u - b * mb * n_groups;
+    const int h = min(mb, m_tiles - b * mb);
+    *g = rest / h;
+    *mt = b * mb + rest % h;
 }
 
 // ----------------------------------------------------------------------------
 // Forward statistics (MODE 0) / backward logit gradient (MODE 1).
-// Work unit u: M tile (u % m_tiles), vocabulary group (u / m_tiles) of
-// kTilesPerGroup 256-wide tiles.  Units of one group run side by side, so a
-// group's W tiles are read from HBM about once and then served from L2.
+// Work unit: one pair M tile x one vocabulary group of kTilesPerGroup
+// 256-wide tiles, folded into one partial per row.
 template <int MODE>
 __global__ void __launch_bounds__(kThreads, 1)
 k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUtensorMap tWs,
-           const __grid_constant__ CUtensorMap tHt, const __grid_constant__ CUtensorMap tWt, FusedArgs a)
+           const __grid_constant__ CUtensorMap tHt, const __grid_constant__ CUtensorMap tWt,
+           const __grid_constant__ CUtensorMap tGst, FusedArgs a)
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ int s_dead;
-    FusedSmem sm = carve(smem_raw, kLmBRegion);
+    FusedSmem sm = carve(smem_raw, kLmBRegion, kStgBytes);
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const uint32_t rank = cluster_ctarank();
+    const int pair = (int)cluster_id(), n_pairs = (int)cluster_count();
     const int nvalid = *a.nvalid;
-    const int m_tiles = (nvalid + BM - 1) / BM;
+    const int m_tiles = (nvalid + BMP - 1) / BMP;
     const int n_tiles = (int)((a.vocab + BN - 1) / BN);
     const int units = m_tiles * a.n_groups;
     const int kb_s = a.d_s / BK, kb_t = a.d_t / BK;
-
-    if (threadIdx.x == 0) {
-        s_dead = 0;
-        init_barriers(sm);
-    }
-    if (warp == 1) {
-        tmem_alloc(sm.tslot, 512);
-        tmem_relinquish();
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = *sm.tslot;
+    const uint32_t tmem = pair_prologue(sm, &s_dead, 512);
 
     if (warp == 0 && lane == 0) {
         // ---------------- producer: per tile the teacher k-blocks, then the student's
@@ -186,30 +266,52 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
         tma_prefetch_desc(&tWs);
         tma_prefetch_desc(&tHt);
         tma_prefetch_desc(&tWt);
+        const uint32_t full0 = mapa(smem_u32(sm.full), 0);
+        const int kb_tile = kb_t + kb_s;
         uint32_t it = 0;
-        for (int u = blockIdx.x; u < units; u += gridDim.x) {
-            const int mt = u % m_tiles, g = u / m_tiles;
+        for (int u = pair; u < units; u += n_pairs) {
+            int mt, g;
+            unit_coords(u, m_tiles, a.n_groups, &mt, &g);
             const int t0 = g * kTilesPerGroup, t1 = min(n_tiles, t0 + kTilesPerGroup);
+            const int ya = mt * BMP + (int)rank * BM;
+            const int n_pos = (t1 - t0) * kb_tile;   // (tile, k-block) positions of this unit
+            // L2 prefetch of this CTA's B rows at unit position p
+            auto prefetch_b = [&](int p) {
+                if (kPrefetch == 0 || p >= n_pos)
+                    return;
+                const int nt2 = t0 + p / kb_tile, kb2 = p % kb_tile;
+                const int yb2 = nt2 * BN + (int)rank * BNH;
+                if (kb2 < kb_t)
+                    tma_prefetch_l2_2d(&tWt, kb2 * BK, yb2);
+                else
+                    tma_prefetch_l2_2d(&tWs, (kb2 - kb_t) * BK, yb2);
+            };
+            for (int p = 0; p < kPrefetch; ++p)
+                prefetch_b(p);
             for (int nt = t0; nt < t1; ++nt) {
-                for (int kb = 0; kb < kb_t + kb_s; ++kb, ++it) {
+                const int yb = nt * BN + (int)rank * BNH;
+                for (int kb = 0; kb < kb_tile; ++kb, ++it) {
+                    prefetch_b((nt - t0) * kb_tile + kb + kPrefetch);
                     const int s = it % STAGES;
                     if (it >= STAGES)
                         wait_lim(&sm.empty[s], ((it / STAGES) - 1) & 1, a.status, &s_dead);
-                    mbar_arrive_expect_tx(&sm.full[s], STAGE_BYTES);
+                    if (rank == 0)
+                        mbar_arrive_expect_tx(&sm.full[s], 2 * STAGE_BYTES);
+                    const uint32_t fb = full0 + (uint32_t)s * 8u;
                     if (kb < kb_t) {
-                        tma_load_2d(sm.a + s * A_BYTES, &tHt, kb * BK, mt * BM, &sm.full[s]);
-                        tma_load_2d(sm.b + s * B_BYTES, &tWt, kb * BK, nt * BN, &sm.full[s]);
+                        tma_load_2d_pair(sm.a + s * A_BYTES, &tHt, kb * BK, ya, fb);
+                        tma_load_2d_pair(sm.b + s * B_BYTES, &tWt, kb * BK, yb, fb);
                     } else {
-                        tma_load_2d(sm.a + s * A_BYTES, &tHs, (kb - kb_t) * BK, mt * BM, &sm.full[s]);
-                        tma_load_2d(sm.b + s * B_BYTES, &tWs, (kb - kb_t) * BK, nt * BN, &sm.full[s]);
+                        tma_load_2d_pair(sm.a + s * A_BYTES, &tHs, (kb - kb_t) * BK, ya, fb);
+                        tma_load_2d_pair(sm.b + s * B_BYTES, &tWs, (kb - kb_t) * BK, yb, fb);
                     }
                 }
             }
         }
-        drain_loads(sm, it);
-    } else if (warp == 1 && lane == 0) {
-        // ---------------- MMA issuer
-        constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+        drain_producer(sm, it, rank);
+    } else if (warp == 1 && lane == 0 && rank == 0) {
+        // ---------------- MMA issuer (even CTA)
+        constexpr uint32_t idesc = idesc_bf16_f32(BMP, BN);
         uint32_t it = 0, tile = 0;
         auto run_k = [&](uint32_t dcol, int nkb) {
             for (int kb = 0; kb < nkb; ++kb, ++it) {
@@ -220,28 +322,28 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
                 for (int k = 0; k < BK / 16; ++k) {
                     const uint64_t ad = smem_desc_sw128(smem_u32(sm.a + s * A_BYTES) + k * 32);
                     const uint64_t bd = smem_desc_sw128(smem_u32(sm.b + s * B_BYTES) + k * 32);
-                    tc_mma(tmem + dcol, ad, bd, idesc, kb > 0 || k > 0);
+                    tc_mma_pair(tmem + dcol, ad, bd, idesc, kb > 0 || k > 0);
                 }
-                tc_commit(&sm.empty[s]);
+                tc_commit_pair(&sm.empty[s], kPairMask);
             }
         };
-        for (int u = blockIdx.x; u < units; u += gridDim.x) {
-            const int g = u / m_tiles;
+        for (int u = pair; u < units; u += n_pairs) {
+            int mt, g;
+            unit_coords(u, m_tiles, a.n_groups, &mt, &g);
             const int t0 = g * kTilesPerGroup, t1 = min(n_tiles, t0 + kTilesPerGroup);
             for (int nt = t0; nt < t1; ++nt, ++tile) {
-                if (tile > 0)  // the epilogue holds Z_t of the previous tile in registers
-                    wait_lim(sm.free_t, (tile - 1) & 1, a.status, &s_dead);
+                if (tile > 0)  // both epilogues hold Z_t of the previous tile in registers
+                    wait_lim(sm.free_t, (tile - 1) & 1, a.status, &s_dead, true);
                 tc_fence_after();
                 run_k(kColT, kb_t);
-                tc_commit(sm.acc_t);
-                if (tile > 0)  // the epilogue has read Z_s of the previous tile
-                    wait_lim(sm.free_s, (tile - 1) & 1, a.status, &s_dead);
+                tc_commit_pair(sm.acc_t, kPairMask);
+                if (tile > 0)  // both epilogues have read Z_s of the previous tile
+                    wait_lim(sm.free_s, (tile - 1) & 1, a.status, &s_dead, true);
                 tc_fence_after();
                 run_k(kColS, kb_s);
-                tc_commit(sm.acc_s);
+                tc_commit_pair(sm.acc_s, kPairMask);
             }
         }
-        drain_mma(sm);
     } else if (warp >= 2) {
         // ---------------- epilogue: warp (q, cq) owns rows q*32.. and columns cq*64..
         const int ew = warp - 2;
@@ -249,11 +351,14 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
         const int cq = ew / 4;               // column slice [cq*64, cq*64 + 64) of the tile
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
         const uint32_t col0 = (uint32_t)(cq * kEpiCols);
+        const uint32_t free_t0 = mapa(smem_u32(sm.free_t), 0), free_s0 = mapa(smem_u32(sm.free_s), 0);
+        uint8_t *stg = sm.stg + ew * kStgWarpBytes;
         uint32_t tile = 0;
-        for (int u = blockIdx.x; u < units; u += gridDim.x) {
-            const int mt = u % m_tiles, g = u / m_tiles;
+        for (int u = pair; u < units; u += n_pairs) {
+            int mt, g;
+            unit_coords(u, m_tiles, a.n_groups, &mt, &g);
             const int t0 = g * kTilesPerGroup, t1 = min(n_tiles, t0 + kTilesPerGroup);
-            const int row = mt * BM + q * 32 + lane;
+            const int row = mt * BMP + (int)rank * BM + q * 32 + lane;
             const bool valid_row = row < nvalid;
             float ms = -INFINITY, ss = 0.f, sa = 0.f, mt_ = -INFINITY, st = 0.f;
             float nl = 0.f, cp = 0.f, sg = 1.f;
@@ -272,10 +377,7 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
                 tmem_ld32(tmem + lane_off + kColT + col0, *reinterpret_cast<float(*)[32]>(&zt[0]));
                 tmem_ld32(tmem + lane_off + kColT + col0 + 32, *reinterpret_cast<float(*)[32]>(&zt[32]));
                 tmem_ld_wait();
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0)
-                    mbar_arrive(sm.free_t);
+                release_cols(free_t0, lane);
                 if (MODE == 0 && nv > 0) {
                     float cmt = -INFINITY;
 #pragma unroll
@@ -291,6 +393,15 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
                     for (int j = 0; j < kEpiCols; ++j)
                         if (j < nv)
                             st += ex2(fmaf(zt[j], kLog2e, ntt));
+                }
+                // G columns [vbase, vbase + 64) lie wholly inside or outside [0, vpad)
+                // (both multiples of 64); the staging buffer is free once the previous
+                // tile's store has read it
+                const bool in_g = MODE == 1 && vbase < a.vpad;
+                if (in_g) {
+                    if (lane == 0)
+                        bulk_wait_read0();
+                    __syncwarp();
                 }
                 // Z_s: 16 columns at a time
                 wait_lim(sm.acc_s, tile & 1, a.status, &s_dead);
@@ -324,30 +435,37 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
                                 }
                             }
                         }
-                    } else if (valid_row && vbase + c0 < a.vpad) {
-                        // G = w p ((z_s - z_t) - E_p[z_s - z_t]); zero beyond the vocabulary.
-                        // vpad is a multiple of 64, so a 16-column chunk is wholly inside
-                        // [0, vpad) or wholly outside it.
+                    } else if (in_g) {
+                        // G = w p ((z_s - z_t) - E_p[z_s - z_t]); zero beyond the vocabulary
+                        // and on rows past the supervised ones.
                         uint32_t pk[8];
 #pragma unroll
                         for (int j = 0; j < 16; j += 2) {
                             float g0 = 0.f, g1 = 0.f;
-                            if (c0 + j < nv)
+                            if (valid_row && c0 + j < nv)
                                 g0 = sg * ex2(fmaf(zs[j], kLog2e, -nl)) * ((zs[j] - zt[c0 + j]) - cp);
-                            if (c0 + j + 1 < nv)
+                            if (valid_row && c0 + j + 1 < nv)
                                 g1 = sg * ex2(fmaf(zs[j + 1], kLog2e, -nl)) *
                                      ((zs[j + 1] - zt[c0 + j + 1]) - cp);
                             pk[j / 2] = pack_bf16x2(g0, g1);
                         }
-                        uint4 *dst = reinterpret_cast<uint4 *>(a.G + (size_t)row * a.vpad + vbase + c0);
-                        dst[0] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-                        dst[1] = make_uint4(pk[4], pk[5], pk[6], pk[7]);
+                        // this row's two 16-byte pieces 2ch, 2ch+1 of the 128-byte staging row,
+                        // placed by the 128-byte swizzle (piece ^ row % 8)
+                        uint8_t *srow = stg + lane * 128;
+                        const int p0 = (2 * ch) ^ (lane & 7), p1 = (2 * ch + 1) ^ (lane & 7);
+                        *reinterpret_cast<uint4 *>(srow + p0 * 16) = make_uint4(pk[0], pk[1], pk[2], pk[3]);
+                        *reinterpret_cast<uint4 *>(srow + p1 * 16) = make_uint4(pk[4], pk[5], pk[6], pk[7]);
                     }
                 }
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0)
-                    mbar_arrive(sm.free_s);
+                release_cols(free_s0, lane);
+                if (MODE == 1 && in_g) {
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_2d(&tGst, (int)vbase, mt * BMP + (int)rank * BM + q * 32, stg);
+                        bulk_commit();
+                    }
+                }
             }
             if (MODE == 0 && valid_row) {
                 float *pp = a.part + (((size_t)g * kColQuarters + cq) * a.cap + row) * 8;
@@ -355,42 +473,38 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
                 reinterpret_cast<float4 *>(pp)[1] = make_float4(st, 0.f, 0.f, 0.f);
             }
         }
+        if (MODE == 1 && lane == 0)
+            bulk_wait0();
     }
-
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (warp == 1)
-        tmem_dealloc(tmem, 512);
+    pair_epilogue(sm, tmem, 512, rank);
 }
 
 // ----------------------------------------------------------------------------
 // dH = G W_s: A = G [rows, vpad] (K-major, K = vocabulary), B = W_s [V, d_s]
-// read in place as an MN-major operand (four 64-column TMA boxes per stage).
-// Output tile 128 x 256 fp32 in tensor memory.  Work split: the first
-// floor(tiles / P) * P tiles are whole tiles, P = grid size, one per CTA per
-// wave, written straight to their token rows; the remaining tiles' k-blocks
-// are split evenly over all P CTAs (each range covers at most two tiles) and
-// written as partial tiles, which k_dh_fixup sums in CTA order.  The result
-// is bitwise reproducible for a given grid size.
+// read in place as an MN-major operand (per CTA two 64-column TMA boxes per
+// stage).  Output pair tile 256 x 256 fp32 in tensor memory.  Work split, with
+// P pairs: the first floor(tiles / P) * P tiles are whole tiles, one per pair
+// per wave, written straight to their token rows; the remaining tiles'
+// k-blocks are split evenly over all P pairs (each range covers at most two
+// tiles) and written as partial tiles, which k_dh_fixup sums in pair order.
+// The result is bitwise reproducible for a given number of pairs.
 struct DhArgs {
     const int4 *rows;
     const int32_t *nvalid;
     int d_s;
     int kbs;         // vpad / BK
     float *dh;       // [T, d_s]
-    float *partial;  // [P][2][BM][BN]
+    float *partial;  // [P][2][BMP][BN]
     int32_t *status;
 };
 
 struct DhSeg {
-    int tile, k0, k1, slot;  // slot -1: whole tile; 0/1: partial slot of this CTA
+    int tile, k0, k1, slot;  // slot -1: whole tile; 0/1: partial slot of this pair
 };
 
 template <class F>
-__device__ __forceinline__ void dh_segments(int tiles, int kbs, F &&f)
+__device__ __forceinline__ void dh_segments(int tiles, int kbs, int P, int c, F &&f)
 {
-    const int P = gridDim.x, c = blockIdx.x;
     const int full = tiles / P * P;
     for (int t = c; t < full; t += P)
         f(DhSeg{t, 0, kbs, -1});
@@ -414,52 +528,57 @@ k_fused_dh(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
 {
     extern __shared__ uint8_t smem_raw[];
     __shared__ int s_dead;
-    FusedSmem sm = carve(smem_raw, kDhBRegion);
+    FusedSmem sm = carve(smem_raw, kDhBRegion, 0);
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const uint32_t rank = cluster_ctarank();
+    const int pair = (int)cluster_id(), n_pairs = (int)cluster_count();
     const int nvalid = *a.nvalid;
-    const int m_tiles = (nvalid + BM - 1) / BM;
+    const int m_tiles = (nvalid + BMP - 1) / BMP;
     const int n_tiles = a.d_s / BN;
     const int tiles = m_tiles * n_tiles;
+    const uint32_t tmem = pair_prologue(sm, &s_dead, 256);
 
-    if (threadIdx.x == 0) {
-        s_dead = 0;
-        init_barriers(sm);
-    }
-    if (warp == 1) {
-        tmem_alloc(sm.tslot, 256);
-        tmem_relinquish();
-    }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    const uint32_t tmem = *sm.tslot;
-
-    // whole tiles: N-tile fastest, so the CTAs of one wave share the G rows (A)
+    // whole tiles: N-tile fastest, so the pairs of one wave share the G rows (A)
     if (warp == 0 && lane == 0) {
         tma_prefetch_desc(&tG);
         tma_prefetch_desc(&tW);
+        const uint32_t full0 = mapa(smem_u32(sm.full), 0);
         uint32_t it = 0;
-        dh_segments(tiles, a.kbs, [&](const DhSeg &sg) {
+        dh_segments(tiles, a.kbs, n_pairs, pair, [&](const DhSeg &sg) {
             const int mt = sg.tile / n_tiles, nt = sg.tile % n_tiles;
+            const int ya = mt * BMP + (int)rank * BM;
+            const int xb = nt * BN + (int)rank * BNH;
+            auto prefetch = [&](int kb) {
+                if (kPrefetch == 0 || kb >= sg.k1)
+                    return;
+                tma_prefetch_l2_2d(&tG, kb * BK, ya);
+#pragma unroll
+                for (int j = 0; j < BNH / 64; ++j)
+                    tma_prefetch_l2_2d(&tW, xb + j * 64, kb * BK);
+            };
+            for (int p = 0; p < kPrefetch; ++p)
+                prefetch(sg.k0 + p);
             for (int kb = sg.k0; kb < sg.k1; ++kb, ++it) {
+                prefetch(kb + kPrefetch);
                 const int s = it % STAGES;
                 if (it >= STAGES)
                     wait_lim(&sm.empty[s], ((it / STAGES) - 1) & 1, a.status, &s_dead);
-                mbar_arrive_expect_tx(&sm.full[s], STAGE_BYTES);
-                tma_load_2d(sm.a + s * A_BYTES, &tG, kb * BK, mt * BM, &sm.full[s]);
+                if (rank == 0)
+                    mbar_arrive_expect_tx(&sm.full[s], 2 * STAGE_BYTES);
+                const uint32_t fb = full0 + (uint32_t)s * 8u;
+                tma_load_2d_pair(sm.a + s * A_BYTES, &tG, kb * BK, ya, fb);
 #pragma unroll
-                for (int j = 0; j < BN / 64; ++j)
-                    tma_load_2d(sm.b + s * B_BYTES + j * (B_BYTES / 4), &tW, nt * BN + j * 64, kb * BK,
-                                &sm.full[s]);
+                for (int j = 0; j < BNH / 64; ++j)
+                    tma_load_2d_pair(sm.b + s * B_BYTES + j * (64 * BK * 2), &tW, xb + j * 64, kb * BK, fb);
             }
         });
-        drain_loads(sm, it);
-    } else if (warp == 1 && lane == 0) {
-        constexpr uint32_t idesc = idesc_bf16_f32(BM, BN, true);
+        drain_producer(sm, it, rank);
+    } else if (warp == 1 && lane == 0 && rank == 0) {
+        constexpr uint32_t idesc = idesc_bf16_f32(BMP, BN, true);
         uint32_t it = 0, tile = 0;
-        dh_segments(tiles, a.kbs, [&](const DhSeg &sg) {
+        dh_segments(tiles, a.kbs, n_pairs, pair, [&](const DhSeg &sg) {
             if (tile > 0)
-                wait_lim(sm.free_s, (tile - 1) & 1, a.status, &s_dead);
+                wait_lim(sm.free_s, (tile - 1) & 1, a.status, &s_dead, true);
             tc_fence_after();
             for (int kb = sg.k0; kb < sg.k1; ++kb, ++it) {
                 const int s = it % STAGES;
@@ -469,25 +588,25 @@ k_fused_dh(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
                 for (int k = 0; k < BK / 16; ++k) {
                     const uint64_t ad = smem_desc_sw128(smem_u32(sm.a + s * A_BYTES) + k * 32);
                     // 16 K-rows of 128 B per step; 64-wide N blocks 8 KB apart; 8-row atoms 1 KB apart
-                    const uint64_t bd = smem_desc_sw128_mn(smem_u32(sm.b + s * B_BYTES) + k * 2048,
-                                                           B_BYTES / 4, 1024);
-                    tc_mma(tmem, ad, bd, idesc, kb > sg.k0 || k > 0);
+                    const uint64_t bd =
+                        smem_desc_sw128_mn(smem_u32(sm.b + s * B_BYTES) + k * 2048, 64 * BK * 2, 1024);
+                    tc_mma_pair(tmem, ad, bd, idesc, kb > sg.k0 || k > 0);
                 }
-                tc_commit(&sm.empty[s]);
+                tc_commit_pair(&sm.empty[s], kPairMask);
             }
-            tc_commit(sm.acc_s);
+            tc_commit_pair(sm.acc_s, kPairMask);
             ++tile;
         });
-        drain_mma(sm);
     } else if (warp >= 2) {
         const int ew = warp - 2, q = warp % 4, cq = ew / 4;
         const uint32_t lane_off = (uint32_t)(q * 32) << 16;
         const int col0 = cq * kEpiCols;
-        const int rloc = q * 32 + lane;
+        const int rloc = (int)rank * BM + q * 32 + lane;   // row within the pair tile
+        const uint32_t free_s0 = mapa(smem_u32(sm.free_s), 0);
         uint32_t tile = 0;
-        dh_segments(tiles, a.kbs, [&](const DhSeg &sg) {
+        dh_segments(tiles, a.kbs, n_pairs, pair, [&](const DhSeg &sg) {
             const int mt = sg.tile / n_tiles, nt = sg.tile % n_tiles;
-            const int row = mt * BM + rloc;
+            const int row = mt * BMP + rloc;
             wait_lim(sm.acc_s, tile & 1, a.status, &s_dead);
             tc_fence_after();
             const bool valid = row < nvalid;
@@ -496,7 +615,7 @@ k_fused_dh(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
                 if (sg.slot < 0)
                     dst = a.dh + (size_t)a.rows[row].x * a.d_s + nt * BN + col0;
                 else
-                    dst = a.partial + (((size_t)blockIdx.x * 2 + sg.slot) * BM + rloc) * BN + col0;
+                    dst = a.partial + (((size_t)pair * 2 + sg.slot) * BMP + rloc) * BN + col0;
             }
 #pragma unroll 1
             for (int ch = 0; ch < kEpiCols / 32; ++ch) {
@@ -510,52 +629,63 @@ k_fused_dh(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
                         d4[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
                 }
             }
-            tc_fence_before();
-            __syncwarp();
-            if (lane == 0)
-                mbar_arrive(sm.free_s);
+            release_cols(free_s0, lane);
             ++tile;
         });
     }
-    tc_fence_before();
-    __syncthreads();
-    tc_fence_after();
-    if (warp == 1)
-        tmem_dealloc(tmem, 256);
+    pair_epilogue(sm, tmem, 256, rank);
 }
 
-// Sum the partial tiles of the split part of dH in CTA order (P = the dH grid
-// size) and write them to their token rows.
-__global__ void k_dh_fixup(const float *__restrict__ partial, const int4 *__restrict__ rows,
-                           const int32_t *__restrict__ nvalid_p, int d_s, int kbs, int P, float *__restrict__ dh)
+// Sum the partial tiles of the split part of dH in pair order (P = pairs of
+// the dH launch, at most kMaxPairs) and write them to their token rows.  Job =
+// (split tile, 8-row block).
+constexpr int kMaxPairs = 256;
+inline int max_pairs(int sms) { return std::max(1, std::min(kMaxPairs, sms / 2)); }
+__global__ void __launch_bounds__(256)
+k_dh_fixup(const float *__restrict__ partial, const int4 *__restrict__ rows, const int32_t *__restrict__ nvalid_p,
+           int d_s, int kbs, int P, float *__restrict__ dh)
 {
+    __shared__ int s_src[kMaxPairs + 2];
+    __shared__ int s_n;
     const int nvalid = *nvalid_p;
     const int n_tiles = d_s / BN;
-    const int tiles = (nvalid + BM - 1) / BM * n_tiles;
+    const int tiles = (nvalid + BMP - 1) / BMP * n_tiles;
     const int full = tiles / P * P;
     const int rem = tiles - full;
     const int64_t total = (int64_t)rem * kbs;
-    for (int j = blockIdx.x; j < rem; j += gridDim.x) {
-        const int t = full + j, mt = t / n_tiles, nt = t % n_tiles;
-        const int64_t lo = (int64_t)j * kbs, hi = lo + kbs;
-        // CTAs whose non-empty k-block range meets [lo, hi)
-        const int64_t c_lo_l = lo * P / total - 1, c_hi_l = hi * P / total + 1;
-        const int c_lo = c_lo_l < 0 ? 0 : (int)c_lo_l;
-        const int c_hi = c_hi_l > P - 1 ? P - 1 : (int)c_hi_l;
-        for (int e = threadIdx.x; e < BM * BN; e += blockDim.x) {
-            const int r = e / BN, col = e % BN;
-            const int row = mt * BM + r;
-            if (row >= nvalid)
-                continue;
-            float acc = 0.f;
-            for (int c = c_lo; c <= c_hi; ++c) {
+    constexpr int kRowsPerJob = 8;
+    for (int job = blockIdx.x; job < rem * (BMP / kRowsPerJob); job += gridDim.x) {
+        const int j = job / (BMP / kRowsPerJob), rb = job % (BMP / kRowsPerJob);
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            // pairs whose non-empty k-block range meets tile j's [lo, hi), in pair order
+            const int64_t lo = (int64_t)j * kbs, hi = lo + kbs;
+            int n = 0;
+            for (int c = 0; c < P; ++c) {
                 const int64_t b = total * c / P, en = total * (c + 1) / P;
                 if (b >= en || en <= lo || b >= hi)
                     continue;
-                const int slot = (b / kbs == j) ? 0 : 1;
-                acc += partial[(((size_t)c * 2 + slot) * BM + r) * BN + col];
+                s_src[n++] = c * 2 + ((b / kbs == j) ? 0 : 1);
             }
-            dh[(size_t)rows[row].x * d_s + nt * BN + col] = acc;
+            s_n = n;
+        }
+        __syncthreads();
+        const int t = full + j, mt = t / n_tiles, nt = t % n_tiles;
+        const int n = s_n;
+        for (int e = threadIdx.x; e < kRowsPerJob * (BN / 4); e += blockDim.x) {
+            const int r = rb * kRowsPerJob + e / (BN / 4), c4 = e % (BN / 4);
+            const int row = mt * BMP + r;
+            if (row >= nvalid)
+                continue;
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int i = 0; i < n; ++i) {
+                const float4 v = reinterpret_cast<const float4 *>(partial)[((size_t)s_src[i] * BMP + r) * (BN / 4) + c4];
+                acc.x += v.x;
+                acc.y += v.y;
+                acc.z += v.z;
+                acc.w += v.w;
+            }
+            reinterpret_cast<float4 *>(dh + (size_t)rows[row].x * d_s + nt * BN)[c4] = acc;
         }
     }
 }
@@ -654,7 +784,7 @@ struct FusedLayout {
 FusedLayout fused_layout(void *ws, int64_t T, int64_t V, int64_t d_s, int64_t d_t, int n_groups, int sms)
 {
     const int64_t vpad = (V + BK - 1) / BK * BK;
-    const int64_t cap = (T + BM - 1) / BM * BM;
+    const int64_t cap = (T + BMP - 1) / BMP * BMP;
     const int64_t nblk = (T + kCompactBlock - 1) / kCompactBlock;
     char *p = static_cast<char *>(ws);
     size_t off = 0;
@@ -673,12 +803,71 @@ FusedLayout fused_layout(void *ws, int64_t T, int64_t V, int64_t d_s, int64_t d_
     L.part = reinterpret_cast<float *>(take(sizeof(float) * 8 * kColQuarters * (size_t)n_groups * cap));
     L.rowc = reinterpret_cast<float *>(take(sizeof(float) * 4 * (size_t)cap));
     L.G = reinterpret_cast<__nv_bfloat16 *>(take(2 * (size_t)cap * vpad));
-    L.dh_partial = reinterpret_cast<float *>(take(sizeof(float) * (size_t)sms * 2 * BM * BN));
+    L.dh_partial = reinterpret_cast<float *>(take(sizeof(float) * (size_t)max_pairs(sms) * 2 * BMP * BN));
     L.bytes = off + 256;
     return L;
 }
 
 int groups_for(int64_t V) { return (int)(((V + BN - 1) / BN + kTilesPerGroup - 1) / kTilesPerGroup); }
+
+// Launch `kern` on `pairs` 2-CTA clusters.
+template <class... KArgs, class... Args>
+cudaError_t launch_pairs(void (*kern)(KArgs...), int pairs, size_t smem, cudaStream_t stream, Args... args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cfg.gridDim = dim3(2 * pairs);
+    return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
+// Co-resident 2-CTA clusters of `kern` (cached per device), at most max_pairs.
+template <class... KArgs>
+cudaError_t pairs_for(void (*kern)(KArgs...), size_t smem, int slot, int *pairs)
+{
+    static int cache[64][3] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess)
+        return e;
+    if (dev < 64 && cache[dev][slot] > 0) {
+        *pairs = cache[dev][slot];
+        return cudaSuccess;
+    }
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess)
+        return e;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 2;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.gridDim = dim3(2);
+    int ncl = 0;
+    e = cudaOccupancyMaxActiveClusters(&ncl, kern, &cfg);
+    if (e != cudaSuccess)
+        return e;
+    if (ncl < 1)
+        return cudaErrorInvalidConfiguration;
+    ncl = std::min(ncl, max_pairs(device_sm_count()));
+    if (dev < 64)
+        cache[dev][slot] = ncl;
+    *pairs = ncl;
+    return cudaSuccess;
+}
 
 }  // namespace
 
@@ -693,7 +882,7 @@ cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream)
     const int sms = device_sm_count();
     FusedLayout L = fused_layout(c.workspace, c.T, c.vocab, c.d_s, c.d_t, n_groups, sms);
     const int64_t vpad = (c.vocab + BK - 1) / BK * BK;
-    const int64_t cap = (c.T + BM - 1) / BM * BM;
+    const int64_t cap = (c.T + BMP - 1) / BMP * BMP;
 
     // supervised rows (the compaction of the loss path), then the gathered hidden rows
     LossArgs la{};
@@ -716,25 +905,19 @@ cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream)
     if (e != cudaSuccess)
         return e;
 
-    alignas(64) CUtensorMap tHs, tWs, tHt, tWt, tG, tWmn;
-    if (!make_map(&tHs, L.hs, cap, c.d_s, BM, BK) || !make_map(&tWs, c.W_s, c.vocab, c.d_s, BN, BK) ||
-        !make_map(&tHt, L.ht, cap, c.d_t, BM, BK) || !make_map(&tWt, c.W_t, c.vocab, c.d_t, BN, BK) ||
-        !make_map(&tG, L.G, cap, vpad, BM, BK) ||
+    alignas(64) CUtensorMap tHs, tWs, tHt, tWt, tG, tGst, tWmn;
+    if (!make_map(&tHs, L.hs, cap, c.d_s, BM, BK) || !make_map(&tWs, c.W_s, c.vocab, c.d_s, BNH, BK) ||
+        !make_map(&tHt, L.ht, cap, c.d_t, BM, BK) || !make_map(&tWt, c.W_t, c.vocab, c.d_t, BNH, BK) ||
+        !make_map(&tG, L.G, cap, vpad, BM, BK) || !make_map(&tGst, L.G, cap, vpad, 32, kEpiCols) ||
         // W_s as the MN-major B of dH: boxes of 64 d-columns x BK vocabulary rows
         !make_map(&tWmn, c.W_s, c.vocab, c.d_s, BK, 64))
         return cudaErrorInvalidValue;
 
-    static bool attr_done = false;
-    if (!attr_done) {
-        e = cudaFuncSetAttribute(k_fused_lm<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedSmem);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(k_fused_lm<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kFusedSmem);
-        if (e == cudaSuccess)
-            e = cudaFuncSetAttribute(k_fused_dh, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDhSmem);
-        if (e != cudaSuccess)
-            return e;
-        attr_done = true;
-    }
+    int p_lm0 = 0, p_lm1 = 0, p_dh = 0;
+    if ((e = pairs_for(k_fused_lm<0>, kFusedSmem, 0, &p_lm0)) != cudaSuccess ||
+        (e = pairs_for(k_fused_lm<1>, kFusedSmem, 1, &p_lm1)) != cudaSuccess ||
+        (e = pairs_for(k_fused_dh, kDhSmem, 2, &p_dh)) != cudaSuccess)
+        return e;
 
     FusedArgs fa;
     fa.vocab = c.vocab;
@@ -750,14 +933,16 @@ cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream)
     fa.G = L.G;
     fa.status = c.status;
 
-    k_fused_lm<0><<<sms, kThreads, kFusedSmem, stream>>>(tHs, tWs, tHt, tWt, fa);
+    if ((e = launch_pairs(k_fused_lm<0>, p_lm0, kFusedSmem, stream, tHs, tWs, tHt, tWt, tGst, fa)) != cudaSuccess)
+        return e;
     k_fused_merge<<<(int)((cap + 255) / 256), 256, 0, stream>>>(L.rows, L.nvalid, L.part, n_groups, cap,
                                                                c.token_loss, L.row_wl, L.rowc, c.status);
     e = cudaGetLastError();
     if (e != cudaSuccess)
         return e;
     if (c.dh_s) {
-        k_fused_lm<1><<<sms, kThreads, kFusedSmem, stream>>>(tHs, tWs, tHt, tWt, fa);
+        if ((e = launch_pairs(k_fused_lm<1>, p_lm1, kFusedSmem, stream, tHs, tWs, tHt, tWt, tGst, fa)) != cudaSuccess)
+            return e;
         launch_zero_masked_f32(c.mask, c.T, (int64_t)c.d_s, c.dh_s, stream);
         DhArgs da;
         da.rows = L.rows;
@@ -767,8 +952,9 @@ cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream)
         da.dh = c.dh_s;
         da.partial = L.dh_partial;
         da.status = c.status;
-        k_fused_dh<<<sms, kThreads, kDhSmem, stream>>>(tG, tWmn, da);
-        k_dh_fixup<<<sms, 256, 0, stream>>>(L.dh_partial, L.rows, L.nvalid, (int)c.d_s, da.kbs, sms, c.dh_s);
+        if ((e = launch_pairs(k_fused_dh, p_dh, kDhSmem, stream, tG, tWmn, da)) != cudaSuccess)
+            return e;
+        k_dh_fixup<<<2 * sms, 256, 0, stream>>>(L.dh_partial, L.rows, L.nvalid, (int)c.d_s, da.kbs, p_dh, c.dh_s);
     }
     launch_loss_sum(L.row_wl, L.nvalid, c.loss, c.status, stream);
     return cudaGetLastError();

@@ -103,6 +103,26 @@ def test_fused_full_heads_sampled_tokens(P, oracle):
     assert abs(loss - wl) <= 1e-9 * abs(wl)
 
 
+def test_fused_all_masked_and_single_row(P, oracle):
+    """No supervised row (loss 0, dh zero), then a single supervised row (one
+    pair tile holding one valid row)."""
+    b = W.packed(seed=11, num_traj=1, traj_len=200)
+    b.loss_mask[:] = 0
+    heads, w, dh, tl, loss = run_fused(P, b, 256, 64, 700, seed=12)
+    assert loss == 0.0
+    assert (dh.cpu().numpy() == 0).all() and (tl == 0).all()
+    b.loss_mask[57] = 1
+    b.turn_id[57] = 0
+    heads, w, dh, tl, loss = run_fused(P, b, 256, 64, 700, seed=12)
+    bits = [W.bf16_bits(x) for x in heads]
+    dh_ref, tl_ref, loss_ref = oracle.fused_lmhead(*bits, b.loss_mask, w)
+    assert_token_loss(tl, tl_ref, b.loss_mask)
+    assert_loss(loss, loss_ref)
+    g = dh.cpu().numpy()
+    assert (np.delete(g, 57, axis=0) == 0).all()
+    assert_dh(g[57:58], dh_ref[57:58])
+
+
 def test_fused_errors(P):
     T, d_s, d_t, V = 8, 256, 64, 512
     z = lambda *s: torch.zeros(s, dtype=torch.bfloat16, device="cuda")
