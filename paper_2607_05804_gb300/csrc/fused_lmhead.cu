@@ -19,7 +19,7 @@
 // CTA stages its own 128 rows of A and 128 rows of B per 64-deep k-block, so a
 // pair reads 2/3 of the operand bytes two independent 128 x 256 tiles would.
 // In each CTA warp 0 streams the operand tiles with TMA (128-byte swizzle)
-// into a 4-stage ring, every copy counted on the even CTA's barrier; warp 1
+// into a 5-stage ring, every copy counted on the even CTA's barrier; warp 1
 // allocates tensor memory, and in the even CTA one thread issues tcgen05.mma
 // and multicasts its commits to both CTAs; warps 2..17 read this CTA's 128
 // accumulator rows back (tcgen05.ld) for the epilogue.  The two halves of the
@@ -47,8 +47,11 @@ constexpr int BM = 128;             // accumulator rows per CTA
 constexpr int BMP = 2 * BM;         // rows per pair tile
 constexpr int BN = 256;             // columns per pair tile
 constexpr int BNH = BN / 2;         // B rows staged per CTA
+// Operand ring depth: 5 x 32 KB plus the 64 KB G staging buffer fills the
+// 227 KB of shared memory a CTA may use (measured: 4 and 6 stages, the
+// latter with direct G stores, are both slower).
 #ifndef TURNOPD_FUSED_STAGES
-#define TURNOPD_FUSED_STAGES 4
+#define TURNOPD_FUSED_STAGES 5
 #endif
 // L2 prefetch distance of the B operand in k-blocks (0: none).  Measured on
 // GB300 it slows the GEMMs (the extra tensor requests compete with the ring's
@@ -82,9 +85,14 @@ struct FusedArgs {
     int32_t *status;
 };
 
+// The phase test comes first: the issuing thread's critical path holds no
+// other shared-memory access (a load of the timeout flag on every k-block
+// costs the tensor pipe about a third of its throughput).
 __device__ __forceinline__ bool wait_lim(uint64_t *bar, uint32_t parity, int32_t *status, int *dead,
                                          bool cluster_scope = false)
 {
+    if (cluster_scope ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity))
+        return true;
     if (*(volatile int *)dead)
         return false;
     for (uint32_t i = 0; i < kLimit; ++i)
@@ -316,8 +324,8 @@ k_fused_lm(const __grid_constant__ CUtensorMap tHs, const __grid_constant__ CUte
         auto run_k = [&](uint32_t dcol, int nkb) {
             for (int kb = 0; kb < nkb; ++kb, ++it) {
                 const int s = it % STAGES;
+                // TMA -> tensor core hand-off: the mbarrier completion suffices
                 wait_lim(&sm.full[s], (it / STAGES) & 1, a.status, &s_dead);
-                tc_fence_after();
 #pragma unroll
                 for (int k = 0; k < BK / 16; ++k) {
                     const uint64_t ad = smem_desc_sw128(smem_u32(sm.a + s * A_BYTES) + k * 32);
@@ -583,7 +591,6 @@ k_fused_dh(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
             for (int kb = sg.k0; kb < sg.k1; ++kb, ++it) {
                 const int s = it % STAGES;
                 wait_lim(&sm.full[s], (it / STAGES) & 1, a.status, &s_dead);
-                tc_fence_after();
 #pragma unroll
                 for (int k = 0; k < BK / 16; ++k) {
                     const uint64_t ad = smem_desc_sw128(smem_u32(sm.a + s * A_BYTES) + k * 32);
