@@ -62,12 +62,15 @@ def _L():
         lib.oracle_turn_stats.argtypes = [P, P, P, P, i32, i64, i32, P, P, P, P, P]
         lib.oracle_fused_lmhead.argtypes = [P, P, i64, P, P, i64, i64, P, P, i64, i32,
                                             P, P, P, P, P, i64]
+        lib.oracle_topk_row.argtypes = [P, P, i32, i64, i32, f64, P, P, P, P]
+        lib.oracle_topk_loss.argtypes = [P, P, i32, i64, i64, P, i64, P, P, i64, i32, P, P, P,
+                                         P, P, P, i64]
         lib.oracle_alpha_schedule.argtypes = [i64, i64, f64, f64]
         lib.oracle_alpha_schedule.restype = f64
         lib.oracle_num_threads.argtypes = []
         for name in ("oracle_turn_counts", "oracle_weights", "oracle_row",
                      "oracle_loss_fwd_bwd", "oracle_turn_stats", "oracle_fused_lmhead",
-                     "oracle_num_threads"):
+                     "oracle_topk_row", "oracle_topk_loss", "oracle_num_threads"):
             getattr(lib, name).restype = ctypes.c_int
         _lib = lib
     return _lib
@@ -194,6 +197,47 @@ def fused_lmhead(h_s, W_s, h_t, W_t, loss_mask, w, mode=FULL_VOCAB, sampled_ids=
                                     _p(wf), T, int(mode), _p(y), _p(dh), _p(tl), _p(loss),
                                     _p(sub), 0 if sub is None else sub.size), "fused_lmhead")
     return dh[:T], tl[:T], float(loss[0])
+
+
+def topk_row(zs, zt, k_top, w=1.0, grad=True):
+    """One row of the teacher top-K reverse KL -> (l, ids [K] int32, g_ids [K] float64,
+    dense g [V] float64 or None).  ids are in support order: larger teacher logit first,
+    lower id among equal logits."""
+    zs = np.ascontiguousarray(zs)
+    zt = np.ascontiguousarray(zt, dtype=zs.dtype)
+    V = zs.size
+    ids = np.zeros(max(int(k_top), 1), np.int32)
+    gk = np.zeros(max(int(k_top), 1), np.float64)
+    g = np.zeros(V, np.float64) if grad else None
+    ell = np.zeros(1, np.float64)
+    _check(_L().oracle_topk_row(_p(zs), _p(zt), _dtype_code(zs), V, int(k_top), float(w),
+                                _p(ids), _p(gk), _p(g), _p(ell)), "topk_row")
+    return float(ell[0]), ids[:k_top], gk[:k_top], g
+
+
+def topk_loss(zs, zt, vocab, loss_mask, w, k_top, row_of_token=None, grad=False, subset=None):
+    """Teacher top-K reverse KL over a batch.  zs, zt: [R, ld].
+    -> (topk_ids [T, K] int32, topk_g [T, K] float64, dense grad [R, V] or None,
+    token_loss [T], loss); topk rows of unsupervised tokens stay -1 / 0."""
+    zs = np.ascontiguousarray(zs)
+    zt = np.ascontiguousarray(zt, dtype=zs.dtype)
+    R, ld = zs.shape
+    msk = _c(loss_mask, np.uint8)
+    T = msk.size
+    K = int(k_top)
+    wf = _c(w, np.float32)
+    rot = _c(row_of_token, np.int32)
+    sub = _c(subset, np.int64)
+    ids = np.full((max(T, 1), max(K, 1)), -1, np.int32)
+    gk = np.zeros((max(T, 1), max(K, 1)), np.float64)
+    g = np.zeros((R, vocab), np.float64) if grad else None
+    tl = np.zeros(max(T, 1), np.float64)
+    loss = np.zeros(1, np.float64)
+    _check(_L().oracle_topk_loss(_p(zs), _p(zt), _dtype_code(zs), ld, vocab, _p(rot), R,
+                                 _p(msk), _p(wf), T, K, _p(ids), _p(gk), _p(g), _p(tl),
+                                 _p(loss), _p(sub), 0 if sub is None else sub.size),
+           "topk_loss")
+    return ids[:T], gk[:T], g, tl[:T], float(loss[0])
 
 
 def alpha_schedule(k, K, s=0.0, e=1.0) -> float:

@@ -32,6 +32,12 @@
  *                           counts n_t (Sec. 5.1; kl_per_turn/num_traj keys).
  *   oracle_fused_lmhead  -- logits z = h W^T from the two LM heads, then the
  *                           row oracle, then dL/dh_s = g W_s.
+ *   oracle_topk_row /    -- the paper's practical loss, the teacher top-K
+ *   oracle_topk_loss        reverse KL (loss_mode topk_reverse_kl with support
+ *                           size K_top = distill_topk = 50 in the full
+ *                           configuration table; Algorithm 1 "top-K reverse-KL
+ *                           token losses"): Eq. (opd-rkl) restricted to the K
+ *                           vocabulary ids of largest teacher logit.
  *   oracle_alpha_schedule-- alpha = clip((k/K - s)/(e - s), 0, 1) (Sec. 5.2,
  *                           Algorithm 1).
  *
@@ -42,7 +48,9 @@
  *   token; a turn index is reliable iff it is reached by >= n_min trajectories,
  *   tokens of unreliable turns keep the token-level weight and the reliable
  *   turns share the rest equally; the sampled-token gradient is the
- *   score-function form w * l * (e_y - p_s).
+ *   score-function form w * l * (e_y - p_s); the top-K support is the K ids of
+ *   largest teacher logit, the lower id first among equal logits, and both
+ *   distributions are renormalised over that support.
  *
  * Status codes returned (same meaning as the library's public codes):
  *   0 ok, 2 bad shape, 3 bad offsets, 4 turn id out of range,
@@ -546,6 +554,156 @@ int oracle_fused_lmhead(const uint16_t *h_s, const uint16_t *W_s, int64_t d_s,
         free(zs);
         free(zt);
         free(g);
+    }
+    if (err)
+        return err;
+    kahan_t L = {0, 0};
+    for (int64_t k = 0; k < n; ++k) {
+        int64_t i = subset ? subset[k] : k;
+        if (mask[i])
+            kadd(&L, (double)w[i] * token_loss[i]);
+    }
+    *loss = kval(&L);
+    return OR_OK;
+}
+
+/* ---- teacher top-K reverse KL -------------------------------------------- */
+
+/* order of the support: larger teacher logit first, lower id among equals */
+typedef struct { double zt; int64_t id; } topk_ent_t;
+static int topk_cmp(const void *a, const void *b)
+{
+    const topk_ent_t *x = (const topk_ent_t *)a, *y = (const topk_ent_t *)b;
+    if (x->zt > y->zt) return -1;
+    if (x->zt < y->zt) return 1;
+    return x->id < y->id ? -1 : (x->id > y->id ? 1 : 0);
+}
+
+/*
+ * One row.  S = the first K ids in the order above.  On S:
+ *   ps_v = exp(zs_v) / sum_{u in S} exp(zs_u),  pt_v likewise from zt,
+ *   l    = sum_{v in S} ps_v (log ps_v - log pt_v)
+ *   g_v  = w ps_v (log ps_v - log pt_v - l)        (= w dl/dzs_v; 0 off S)
+ * ids[K] receives S in order, gk[K] the g of those ids (both nullable);
+ * g (nullable) receives all V entries (0 off S).
+ */
+static int topk_core(const double *zs, const double *zt, int64_t V, int32_t K, double w,
+                     int32_t *ids, double *gk, double *g, double *ell)
+{
+    if (K < 1 || K > V)
+        return OR_SHAPE;
+    topk_ent_t *e = (topk_ent_t *)malloc(sizeof(topk_ent_t) * (size_t)V);
+    for (int64_t v = 0; v < V; ++v) {
+        if (!isfinite(zs[v]) || !isfinite(zt[v])) {
+            free(e);
+            return OR_NONFINITE;
+        }
+        e[v].zt = zt[v];
+        e[v].id = v;
+    }
+    qsort(e, (size_t)V, sizeof(topk_ent_t), topk_cmp);
+    double ms = -INFINITY, mt = -INFINITY;
+    for (int32_t r = 0; r < K; ++r) {
+        int64_t v = e[r].id;
+        if (zs[v] > ms) ms = zs[v];
+        if (zt[v] > mt) mt = zt[v];
+    }
+    kahan_t ss = {0, 0}, st = {0, 0};
+    for (int32_t r = 0; r < K; ++r) {
+        int64_t v = e[r].id;
+        kadd(&ss, exp(zs[v] - ms));
+        kadd(&st, exp(zt[v] - mt));
+    }
+    double lse_s = ms + log(kval(&ss)), lse_t = mt + log(kval(&st));
+    kahan_t kl = {0, 0};
+    for (int32_t r = 0; r < K; ++r) {
+        int64_t v = e[r].id;
+        double ls = zs[v] - lse_s, lt = zt[v] - lse_t;
+        kadd(&kl, exp(ls) * (ls - lt));
+    }
+    double l = kval(&kl);
+    if (g)
+        for (int64_t v = 0; v < V; ++v)
+            g[v] = 0.0;
+    for (int32_t r = 0; r < K; ++r) {
+        int64_t v = e[r].id;
+        double ls = zs[v] - lse_s, lt = zt[v] - lse_t;
+        double gv = w * exp(ls) * (ls - lt - l);
+        if (ids) ids[r] = (int32_t)v;
+        if (gk) gk[r] = gv;
+        if (g) g[v] = gv;
+    }
+    *ell = l;
+    free(e);
+    return OR_OK;
+}
+
+int oracle_topk_row(const void *zs, const void *zt, int32_t dtype, int64_t V, int32_t K,
+                    double w, int32_t *ids, double *gk, double *g, double *ell)
+{
+    if (V < 1)
+        return OR_SHAPE;
+    double *a = (double *)malloc(sizeof(double) * (size_t)V);
+    double *b = (double *)malloc(sizeof(double) * (size_t)V);
+    for (int64_t v = 0; v < V; ++v) {
+        a[v] = elem(zs, dtype, v);
+        b[v] = elem(zt, dtype, v);
+    }
+    int st = topk_core(a, b, V, K, w, ids, gk, g, ell);
+    free(a);
+    free(b);
+    return st;
+}
+
+/*
+ * The top-K loss over a packed batch (same conventions as
+ * oracle_loss_fwd_bwd): token_loss[i] = l_i, *loss = sum_i w_i l_i in token
+ * order, topk_ids / topk_g [T, K] (nullable) hold S and its g for supervised
+ * tokens (untouched otherwise), grad (nullable) a dense [num_rows, V] array.
+ */
+int oracle_topk_loss(const void *zs, const void *zt, int32_t dtype, int64_t ld, int64_t V,
+                     const int32_t *row_of_token, int64_t num_rows, const uint8_t *mask,
+                     const float *w, int64_t T, int32_t K, int32_t *topk_ids, double *topk_g,
+                     double *grad, double *token_loss, double *loss,
+                     const int64_t *subset, int64_t n_subset)
+{
+    if (V < 1 || ld < V || T < 0 || K < 1 || K > V)
+        return OR_SHAPE;
+    if (grad)
+        memset(grad, 0, sizeof(double) * (size_t)num_rows * (size_t)V);
+    int64_t n = subset ? n_subset : T;
+    for (int64_t k = 0; k < n; ++k) {
+        int64_t i = subset ? subset[k] : k;
+        if (i < 0 || i >= T)
+            return OR_SHAPE;
+        token_loss[i] = 0.0;
+        if (!mask[i])
+            continue;
+        int64_t r = row_of_token ? row_of_token[i] : i;
+        if (r < 0 || r >= num_rows)
+            return OR_TOKEN_RANGE;
+    }
+    int err = OR_OK;
+    size_t esz = dtype == OR_BF16 ? 2 : 4;
+#pragma omp parallel for schedule(dynamic, 1)
+    for (int64_t k = 0; k < n; ++k) {
+        int64_t i = subset ? subset[k] : k;
+        if (!mask[i])
+            continue;
+        int64_t r = row_of_token ? row_of_token[i] : i;
+        const char *ps = (const char *)zs + (size_t)r * (size_t)ld * esz;
+        const char *pt = (const char *)zt + (size_t)r * (size_t)ld * esz;
+        double l = 0.0;
+        int st = oracle_topk_row(ps, pt, dtype, V, K, (double)w[i],
+                                 topk_ids ? topk_ids + (size_t)i * (size_t)K : NULL,
+                                 topk_g ? topk_g + (size_t)i * (size_t)K : NULL,
+                                 grad ? grad + (size_t)r * (size_t)V : NULL, &l);
+        if (st) {
+#pragma omp critical
+            err = st;
+        } else {
+            token_loss[i] = l;
+        }
     }
     if (err)
         return err;
