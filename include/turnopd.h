@@ -258,6 +258,52 @@ turnopd_status turnopd_fused_lmhead_fwd_bwd(const void *h_s, const void *W_s, in
 size_t turnopd_fused_workspace_bytes(int64_t num_tokens, int64_t vocab, int64_t d_s, int64_t d_t);
 
 /*
+ * turnopd_topk_loss_fwd_bwd -- teacher top-K reverse KL and its gradient
+ * (the paper's practical loss, loss_mode topk_reverse_kl with support size
+ * K_top = distill_topk = 50 in the full configuration table; Algorithm 1,
+ * "top-K reverse-KL token losses").
+ *
+ * For every supervised token i (loss_mask[i] = 1), with row r = row_of_token[i]
+ * (or i when row_of_token is NULL): S_i = the k_top vocabulary ids of largest
+ * teacher logit z_teacher[r, .], the lower id first among equal logits (+0 and
+ * -0 are equal); both distributions are renormalised over S_i:
+ *   l_i    = sum_{v in S_i} ps_v (log ps_v - log pt_v),
+ *            ps_v = exp(z_s[r,v]) / sum_{u in S_i} exp(z_s[r,u]), pt likewise;
+ *   g_i,v  = w_i ps_v (log ps_v - log pt_v - l_i) for v in S_i, 0 elsewhere
+ *            (= w_i dl_i/dz_s[r, v]);
+ *   *loss_out = sum_i w_i l_i (fixed order, fp64).
+ * Inputs (device, row-major): z_student, z_teacher [num_rows, ld] of in_dtype
+ *   (TURNOPD_BF16 or TURNOPD_F32), ld >= vocab; loss_mask uint8[num_tokens];
+ *   w float32[num_tokens]; 1 <= k_top <= min(vocab, TURNOPD_TOPK_MAX).
+ * Outputs (each nullable except token_loss_out and loss_out):
+ *   topk_ids_out  int32 [num_tokens, k_top]: S_i in order (largest teacher
+ *                 logit first); topk_grad_out float32 [num_tokens, k_top]: g_i
+ *                 at those ids.  Rows of masked tokens are left as they are, or
+ *                 set to -1 / 0 with TURNOPD_ZERO_MASKED_GRAD.
+ *   grad_student  dense [num_rows, ld] of grad_dtype: row r gets zeros and g_i
+ *                 on S_i (columns >= vocab untouched); rows of masked tokens as
+ *                 in turnopd_loss_fwd_bwd.
+ *   token_loss_out float32[num_tokens] (0 for masked tokens), loss_out double.
+ * Workspace: turnopd_loss_workspace_bytes(num_tokens) bytes, 256-byte aligned.
+ * Flags: TURNOPD_ZERO_MASKED_GRAD only.
+ * Host errors: NULL / SHAPE (k_top out of range, misalignment) / UNSUPPORTED /
+ *   WORKSPACE, returned before any launch.  Device errors (in *dev_status):
+ *   TURNOPD_ERR_TOKEN_RANGE (row index), TURNOPD_ERR_NONFINITE, and
+ *   TURNOPD_ERR_UNSUPPORTED for a row whose selection did not settle within the
+ *   kernel's bounded rounds (only rows with thousands of equal top logits).
+ */
+#define TURNOPD_TOPK_MAX 1024
+turnopd_status turnopd_topk_loss_fwd_bwd(const void *z_student, const void *z_teacher,
+                                         int32_t in_dtype, int64_t ld, int64_t vocab,
+                                         int64_t num_rows, const int32_t *row_of_token,
+                                         const uint8_t *loss_mask, const float *w,
+                                         int64_t num_tokens, int32_t k_top, int32_t *topk_ids_out,
+                                         float *topk_grad_out, void *grad_student, int32_t grad_dtype,
+                                         uint32_t flags, float *token_loss_out, double *loss_out,
+                                         void *workspace, size_t workspace_bytes,
+                                         int32_t *dev_status, turnopd_stream_t stream);
+
+/*
  * turnopd_turn_stats -- turn statistics of the per-token losses
  * (Eq. observed-turn-kl: K_t is the mean per-token reverse KL over the
  * supervised tokens at turn t, over trajectories that reach t; the survivor

@@ -23,6 +23,7 @@ __all__ = [
     "turnopd_loss_fwd_bwd", "turnopd_loss_workspace_bytes", "turnopd_turn_stats",
     "turnopd_alpha_schedule", "turnopd_status_string", "turnopd_loss_fwd_bwd_static",
     "TURNOPD_STATIC_MAX_TOKENS", "turnopd_fused_lmhead_fwd_bwd", "turnopd_fused_workspace_bytes",
+    "turnopd_topk_loss_fwd_bwd", "TURNOPD_TOPK_MAX",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -35,6 +36,7 @@ TURNOPD_ZERO_MASKED_GRAD = 0x1
 TURNOPD_FORCE_PORTABLE = 0x100
 TURNOPD_MAX_TURNS = 4096
 TURNOPD_STATIC_MAX_TOKENS = 65536
+TURNOPD_TOPK_MAX = 1024
 
 STATUS_NAMES = {
     0: "TURNOPD_OK", 1: "TURNOPD_ERR_NULL", 2: "TURNOPD_ERR_SHAPE", 3: "TURNOPD_ERR_OFFSETS",
@@ -79,6 +81,8 @@ def load():
                                         u32, P, P, P, P],
         "turnopd_fused_lmhead_fwd_bwd": [P, P, i64, P, P, i64, i64, P, P, i64, i32, P, P, P, P, sz,
                                          P, P],
+        "turnopd_topk_loss_fwd_bwd": [P, P, i32, i64, i64, i64, P, P, P, i64, i32, P, P, P, i32, u32,
+                                      P, P, P, sz, P, P],
     }
     for name, args in sig.items():
         fn = getattr(lib, name)
@@ -261,6 +265,45 @@ def turnopd_loss_fwd_bwd(z_student, z_teacher, vocab, row_of_token, sampled_ids,
         int(mode), _ptr(grad_student), gdt, int(flags), _ptr(token_loss_out), _ptr(loss_out),
         _ptr(workspace), workspace.numel() * workspace.element_size(), _ptr(dev_status),
         _stream(stream)), "turnopd_loss_fwd_bwd")
+
+
+def turnopd_topk_loss_fwd_bwd(z_student, z_teacher, vocab, row_of_token, loss_mask, w, k_top,
+                              topk_ids_out, topk_grad_out, grad_student, flags, token_loss_out,
+                              loss_out, workspace, dev_status, stream=None):
+    """Teacher top-K reverse KL.  z_student, z_teacher: [num_rows, ld] tensors;
+    topk_ids_out int32 / topk_grad_out float32 [T, k_top] or None; grad_student None or
+    a tensor shaped like z_student."""
+    import torch
+
+    T = loss_mask.numel()
+    for name, z in (("z_student", z_student), ("z_teacher", z_teacher)):
+        if not z.is_cuda or z.dim() != 2 or z.stride(1) != 1:
+            raise ValueError(f"{name} must be a 2-D CUDA tensor with unit column stride")
+    if z_teacher.shape != z_student.shape or z_teacher.stride() != z_student.stride() \
+            or z_teacher.dtype != z_student.dtype:
+        raise ValueError("z_teacher must match z_student in shape, stride and dtype")
+    ld = z_student.stride(0)
+    if grad_student is not None and (grad_student.shape != z_student.shape
+                                     or grad_student.stride(0) != ld or grad_student.stride(1) != 1
+                                     or not grad_student.is_cuda):
+        raise ValueError("grad_student must match z_student in shape and row stride")
+    _need(row_of_token, "row_of_token", torch.int32, T)
+    _need(loss_mask, "loss_mask", torch.uint8)
+    _need(w, "w", torch.float32, T)
+    _need(topk_ids_out, "topk_ids_out", torch.int32, T * int(k_top))
+    _need(topk_grad_out, "topk_grad_out", torch.float32, T * int(k_top))
+    _need(token_loss_out, "token_loss_out", torch.float32, T)
+    _need(loss_out, "loss_out", torch.float64, 1)
+    _need(workspace, "workspace")
+    _need(dev_status, "dev_status", torch.int32, 1)
+    gdt = _dtype_code(grad_student, "grad_student") if grad_student is not None else TURNOPD_F32
+    _check(load().turnopd_topk_loss_fwd_bwd(
+        _ptr(z_student), _ptr(z_teacher), _dtype_code(z_student, "z_student"), ld, int(vocab),
+        z_student.shape[0], _ptr(row_of_token), _ptr(loss_mask), _ptr(w), T, int(k_top),
+        _ptr(topk_ids_out), _ptr(topk_grad_out), _ptr(grad_student), gdt, int(flags),
+        _ptr(token_loss_out), _ptr(loss_out), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream)),
+        "turnopd_topk_loss_fwd_bwd")
 
 
 def turnopd_turn_stats(token_loss, turn_id, loss_mask, traj_offsets, max_turns, traj_turn_sum,

@@ -166,6 +166,22 @@ __device__ __forceinline__ int64_t warp_sum_i64(int64_t x)
     return x;
 }
 
+__device__ __forceinline__ float warp_sum_f(float x)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+        x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+__device__ __forceinline__ float warp_max_f(float x)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+        x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, o));
+    return x;
+}
+
 __device__ __forceinline__ int warp_sum_i32(int x)
 {
 #pragma unroll

@@ -88,6 +88,32 @@ void launch_loss_sum(const double *row_wl, const int32_t *nvalid, double *loss, 
                      cudaStream_t stream);
 // Zero rows i (of d fp32 values) of out where mask[i] == 0.
 void launch_zero_masked_f32(const uint8_t *mask, int64_t T, int64_t d, float *out, cudaStream_t stream);
+// Zero the gradient rows (row_of_token[i] or i, ld apart, vocab entries) of masked tokens.
+void launch_zero_masked_grad(const uint8_t *mask, const int32_t *row_of_token, int64_t T, int64_t num_rows,
+                             int64_t ld, int64_t vocab, void *grad, int32_t grad_dtype, cudaStream_t stream);
+
+// Teacher top-K reverse KL.
+constexpr int kTopkMaxK = 1024;
+struct TopkCall {
+    const void *zs, *zt;
+    int32_t in_dtype;
+    int64_t ld, vocab, num_rows;
+    const int32_t *row_of_token;
+    const uint8_t *mask;
+    const float *w;
+    int64_t T;
+    int32_t K;
+    int32_t *topk_ids;
+    float *topk_grad;
+    void *grad;
+    int32_t grad_dtype;
+    uint32_t flags;
+    float *token_loss;
+    double *loss;
+    void *workspace;
+    int32_t *status;
+};
+cudaError_t launch_topk(const TopkCall &c, cudaStream_t stream);
 
 // Fused LM heads (bf16 hidden states and heads) + loss + dL/dh_s.
 struct FusedCall {

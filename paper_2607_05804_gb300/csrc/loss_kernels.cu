@@ -427,6 +427,18 @@ void launch_zero_masked_f32(const uint8_t *mask, int64_t T, int64_t d, float *ou
     k_zero_masked<float><<<grid, 256, 0, stream>>>(mask, nullptr, T, T, d, d, out);
 }
 
+void launch_zero_masked_grad(const uint8_t *mask, const int32_t *row_of_token, int64_t T, int64_t num_rows,
+                             int64_t ld, int64_t vocab, void *grad, int32_t grad_dtype, cudaStream_t stream)
+{
+    const int grid = (int)std::min<int64_t>(std::max<int64_t>(T, 1), (int64_t)device_sm_count() * 8);
+    if (grad_dtype == TURNOPD_BF16)
+        k_zero_masked<__nv_bfloat16><<<grid, 256, 0, stream>>>(mask, row_of_token, T, num_rows, ld, vocab,
+                                                                static_cast<__nv_bfloat16 *>(grad));
+    else
+        k_zero_masked<float><<<grid, 256, 0, stream>>>(mask, row_of_token, T, num_rows, ld, vocab,
+                                                        static_cast<float *>(grad));
+}
+
 cudaError_t launch_loss(const LossArgs &a, const LossWorkspace &ws, cudaStream_t stream)
 {
     cudaError_t e = launch_compaction(a, ws.rows, ws.blk_count, ws.nvalid, stream);
@@ -434,16 +446,9 @@ cudaError_t launch_loss(const LossArgs &a, const LossWorkspace &ws, cudaStream_t
         return e;
 
     const int sms = device_sm_count();
-    if (a.grad && (a.flags & TURNOPD_ZERO_MASKED_GRAD)) {
-        const int grid = (int)std::min<int64_t>(a.T, (int64_t)sms * 8);
-        if (a.grad_dtype == TURNOPD_BF16)
-            k_zero_masked<__nv_bfloat16><<<grid, 256, 0, stream>>>(
-                a.mask, a.row_of_token, a.T, a.num_rows, a.ld, a.vocab,
-                static_cast<__nv_bfloat16 *>(a.grad));
-        else
-            k_zero_masked<float><<<grid, 256, 0, stream>>>(a.mask, a.row_of_token, a.T, a.num_rows,
-                                                            a.ld, a.vocab, static_cast<float *>(a.grad));
-    }
+    if (a.grad && (a.flags & TURNOPD_ZERO_MASKED_GRAD))
+        launch_zero_masked_grad(a.mask, a.row_of_token, a.T, a.num_rows, a.ld, a.vocab, a.grad, a.grad_dtype,
+                                stream);
 
     RowIn p{a.zs, a.zt, a.ld, a.vocab, a.row_of_token, a.sampled_ids, a.w, a.mode, a.grad,
             a.token_loss, ws.row_wl, ws.rows, ws.nvalid, a.status};

@@ -194,6 +194,64 @@ turnopd_status turnopd_loss_fwd_bwd(const void *z_student, const void *z_teacher
     return cuda_status(launch_loss(a, loss_workspace_layout(workspace, num_tokens), s));
 }
 
+turnopd_status turnopd_topk_loss_fwd_bwd(const void *z_student, const void *z_teacher, int32_t in_dtype,
+                                         int64_t ld, int64_t vocab, int64_t num_rows,
+                                         const int32_t *row_of_token, const uint8_t *loss_mask,
+                                         const float *w, int64_t num_tokens, int32_t k_top,
+                                         int32_t *topk_ids_out, float *topk_grad_out, void *grad_student,
+                                         int32_t grad_dtype, uint32_t flags, float *token_loss_out,
+                                         double *loss_out, void *workspace, size_t workspace_bytes,
+                                         int32_t *dev_status, turnopd_stream_t stream)
+{
+    if (!loss_out || !dev_status)
+        return TURNOPD_ERR_NULL;
+    if (num_tokens > 0 && (!z_student || !z_teacher || !loss_mask || !w || !token_loss_out))
+        return TURNOPD_ERR_NULL;
+    if ((in_dtype != TURNOPD_F32 && in_dtype != TURNOPD_BF16) ||
+        (grad_student && grad_dtype != TURNOPD_F32 && grad_dtype != TURNOPD_BF16))
+        return TURNOPD_ERR_UNSUPPORTED;
+    if (flags & ~(uint32_t)TURNOPD_ZERO_MASKED_GRAD)
+        return TURNOPD_ERR_UNSUPPORTED;
+    if (num_tokens < 0 || num_tokens > INT32_MAX || vocab < 1 || vocab > INT32_MAX || ld < vocab ||
+        num_rows < 0 || (!row_of_token && num_rows < num_tokens) || k_top < 1 || k_top > TURNOPD_TOPK_MAX ||
+        k_top > vocab || num_tokens * (int64_t)k_top > INT64_MAX / 8)
+        return TURNOPD_ERR_SHAPE;
+    const size_t esz = in_dtype == TURNOPD_BF16 ? 2 : 4;
+    if (misaligned(z_student, esz) || misaligned(z_teacher, esz) ||
+        (grad_student && misaligned(grad_student, grad_dtype == TURNOPD_BF16 ? 2 : 4)) ||
+        (topk_ids_out && misaligned(topk_ids_out, 4)) || (topk_grad_out && misaligned(topk_grad_out, 4)) ||
+        misaligned(loss_out, 8))
+        return TURNOPD_ERR_SHAPE;
+    if (!workspace || misaligned(workspace, 256) ||
+        workspace_bytes < loss_workspace_bytes(num_tokens))
+        return TURNOPD_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (num_tokens == 0)
+        return cuda_status(cudaMemsetAsync(loss_out, 0, sizeof(double), s));
+    TopkCall c;
+    c.zs = z_student;
+    c.zt = z_teacher;
+    c.in_dtype = in_dtype;
+    c.ld = ld;
+    c.vocab = vocab;
+    c.num_rows = num_rows;
+    c.row_of_token = row_of_token;
+    c.mask = loss_mask;
+    c.w = w;
+    c.T = num_tokens;
+    c.K = k_top;
+    c.topk_ids = topk_ids_out;
+    c.topk_grad = topk_grad_out;
+    c.grad = grad_student;
+    c.grad_dtype = grad_dtype;
+    c.flags = flags;
+    c.token_loss = token_loss_out;
+    c.loss = loss_out;
+    c.workspace = workspace;
+    c.status = dev_status;
+    return cuda_status(launch_topk(c, s));
+}
+
 size_t turnopd_fused_workspace_bytes(int64_t num_tokens, int64_t vocab, int64_t d_s, int64_t d_t)
 {
     if (num_tokens < 0 || vocab < 1 || d_s < 1 || d_t < 1)

@@ -117,3 +117,28 @@ def test_alpha_schedule_and_status_strings(lib, oracle):
     for code in range(11):
         assert P.turnopd_status_string(code)
     assert P.turnopd_status_string(0) == "ok"
+
+
+def test_topk_host_validation(lib):
+    f = lib.turnopd_topk_loss_fwd_bwd
+    ws_need = lib.turnopd_loss_workspace_bytes(64)
+
+    def call(zs=FAKE, ld=1024, vocab=1024, rows=64, T=64, k=50, in_dtype=1, grad_dtype=0,
+             flags=0, ws=FAKE, wsb=None, loss=FAKE, status=FAKE, ids=FAKE, g=FAKE, grad=None):
+        return f(zs, FAKE, in_dtype, ld, vocab, rows, None, FAKE, FAKE, T, k, ids, g, grad,
+                 grad_dtype, flags, FAKE, loss, ws, ws_need if wsb is None else wsb, status, None)
+
+    assert call(zs=None) == 1
+    assert call(loss=None) == 1
+    assert call(status=None) == 1
+    assert call(k=0) == 2
+    assert call(k=1025) == 2
+    assert call(k=51, vocab=50, ld=64) == 2          # k_top > vocab
+    assert call(ld=100, vocab=101) == 2
+    assert call(rows=10) == 2
+    assert call(ids=ctypes.c_void_p(0x10002)) == 2   # misaligned int32 output
+    assert call(in_dtype=5) == 6
+    assert call(grad=FAKE, grad_dtype=4) == 6
+    assert call(flags=0x100) == 6                     # only TURNOPD_ZERO_MASKED_GRAD
+    assert call(ws=None) == 10
+    assert call(wsb=ws_need - 1) == 10

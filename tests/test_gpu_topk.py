@@ -1,0 +1,218 @@
+"""GPU parity of the teacher top-K reverse KL (turnopd_topk_loss_fwd_bwd)
+against the fp64 oracle.
+
+The selected ids are compared bit for bit (the selection is a decision on the
+bf16/fp32 teacher logits, taken exactly on both sides).  Per-token loss and
+total loss use the loss path's bounds; the gradient at the selected ids is
+within 1e-4 of the row's largest |g| (fp32 output) and the dense bf16 rows
+within 2 bf16 ulps or that bound.
+"""
+import numpy as np
+import pytest
+
+import workloads as W
+from parity import assert_loss, assert_token_loss, bf16_ulp
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def P():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import paper_2607_05804_gb300 as P
+
+    P.load()
+    return P
+
+
+def host(t):
+    if t.dtype == torch.bfloat16:
+        return t.view(torch.int16).cpu().numpy().view(np.uint16)
+    return t.cpu().numpy()
+
+
+def run_topk(P, zs, zt, V, mask, w, K, rot=None, dense=None, flags=0, ids_fill=-7, g_fill=9.0):
+    T = mask.numel()
+    dev = zs.device
+    ids = torch.full((T, K), ids_fill, dtype=torch.int32, device=dev)
+    gk = torch.full((T, K), g_fill, dtype=torch.float32, device=dev)
+    tl = torch.full((T,), 5.0, dtype=torch.float32, device=dev)
+    loss = torch.zeros(1, dtype=torch.float64, device=dev)
+    st = torch.zeros(1, dtype=torch.int32, device=dev)
+    ws = torch.empty(max(P.turnopd_loss_workspace_bytes(T), 256), dtype=torch.uint8, device=dev)
+    P.turnopd_topk_loss_fwd_bwd(zs, zt, V, rot, mask, w, K, ids, gk, dense, flags, tl, loss, ws, st)
+    torch.cuda.synchronize()
+    return ids.cpu().numpy(), gk.cpu().numpy(), tl.cpu().numpy(), loss.item(), st.item()
+
+
+def check_against_oracle(oracle, zs, zt, V, mask, w, K, ids, gk, tl, loss, rot=None, subset=None):
+    m = mask.cpu().numpy()
+    rids, rg, _, rtl, rloss = oracle.topk_loss(host(zs), host(zt), V, m, w.cpu().numpy(), K,
+                                               row_of_token=None if rot is None else rot.cpu().numpy(),
+                                               subset=subset)
+    toks = np.nonzero(m)[0] if subset is None else np.asarray([t for t in subset if m[t]])
+    np.testing.assert_array_equal(ids[toks], rids[toks])
+    assert_token_loss(tl[toks], rtl[toks])
+    rowmax = np.abs(rg[toks]).max(axis=1, keepdims=True)
+    err = np.abs(gk[toks] - rg[toks])
+    assert (err <= 1e-4 * rowmax + 1e-30).all(), float((err / np.maximum(rowmax, 1e-30)).max())
+    if subset is None:
+        assert_loss(loss, rloss)
+    return rids, rg
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("K", [1, 5, 50])
+def test_tiny_all_rows(P, oracle, dtype, K):
+    b = W.tiny(seed=1)
+    V = 1024
+    zs, zt = W.make_logits(b.num_tokens, V, "tiny", dtype, seed=11, device="cuda")
+    mask = torch.from_numpy(b.loss_mask).cuda()
+    w = torch.rand(b.num_tokens, generator=torch.Generator().manual_seed(2)).cuda()
+    ids, gk, tl, loss, st = run_topk(P, zs, zt, V, mask, w, K)
+    assert st == 0
+    check_against_oracle(oracle, zs, zt, V, mask, w, K, ids, gk, tl, loss)
+    m = b.loss_mask == 0
+    assert (tl[m] == 0).all()
+    assert (ids[m] == -7).all() and (gk[m] == 9.0).all()  # masked rows untouched without the flag
+
+
+def test_ties_and_signed_zero(P, oracle):
+    """Rows built from few distinct dyadic bf16 values: many equal teacher
+    logits around the K-th, and rows mixing +0 and -0."""
+    g = torch.Generator().manual_seed(3)
+    T, V, K = 64, 5000, 50
+    levels = torch.tensor([-2.0, -1.0, -0.0, 0.0, 0.5, 1.0, 1.5], dtype=torch.float32)
+    pick = torch.randint(0, len(levels), (T, V), generator=g)
+    zt = levels[pick].to(torch.bfloat16)
+    zs = (torch.randn(T, V, generator=g) * 2).to(torch.bfloat16)
+    # a few rows with a unique top and otherwise all equal logits
+    zt[5] = 0.0
+    zt[5, 4321] = 1.0
+    zt[6] = -0.0
+    zt[6, 7] = 0.0
+    zs, zt = zs.cuda(), zt.cuda()
+    mask = torch.ones(T, dtype=torch.uint8, device="cuda")
+    w = torch.full((T,), 0.5, dtype=torch.float32, device="cuda")
+    ids, gk, tl, loss, st = run_topk(P, zs, zt, V, mask, w, K)
+    assert st == 0
+    check_against_oracle(oracle, zs, zt, V, mask, w, K, ids, gk, tl, loss)
+    assert ids[5, 0] == 4321 and ids[5, 1:].tolist() == list(range(K - 1))
+    assert ids[6].tolist() == list(range(K))
+
+
+def test_all_equal_row_takes_the_lowest_ids(P, oracle):
+    """Every teacher logit equal: the candidate buffer overflows and the
+    selection settles by the id bytes."""
+    T, V, K = 4, 151936, 50
+    zt = torch.full((T, V), 0.75, dtype=torch.bfloat16, device="cuda")
+    zs = torch.randn(T, V, generator=torch.Generator(device="cuda").manual_seed(4), device="cuda").to(torch.bfloat16)
+    mask = torch.ones(T, dtype=torch.uint8, device="cuda")
+    w = torch.ones(T, dtype=torch.float32, device="cuda")
+    ids, gk, tl, loss, st = run_topk(P, zs, zt, V, mask, w, K)
+    assert st == 0
+    for i in range(T):
+        assert ids[i].tolist() == list(range(K))
+    check_against_oracle(oracle, zs, zt, V, mask, w, K, ids, gk, tl, loss, subset=[0, 3])
+
+
+def test_k_equals_v_is_the_full_kl(P, oracle):
+    T, V = 16, 700
+    zs, zt = W.make_logits(T, V, "tiny", torch.float32, seed=5, device="cuda")
+    mask = torch.ones(T, dtype=torch.uint8, device="cuda")
+    w = torch.ones(T, dtype=torch.float32, device="cuda")
+    ids, gk, tl, loss, st = run_topk(P, zs, zt, V, mask, w, V)
+    assert st == 0
+    _, tl_full, _ = oracle.loss_fwd_bwd(host(zs), host(zt), V, mask.cpu().numpy(), w.cpu().numpy(),
+                                        grad=False)
+    assert_token_loss(tl, tl_full)
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+def test_dense_gradient_misaligned_stride_and_zero_flag(P, oracle, dtype):
+    """Row stride not a multiple of 16 bytes (the scalar path), dense gradient
+    rows, compact rows through row_of_token, and TURNOPD_ZERO_MASKED_GRAD."""
+    b = W.packed(seed=7, num_traj=2, traj_len=300)
+    T, V, K = b.num_tokens, 3001, 50
+    ld = 3003
+    rows = b.num_valid
+    zs, zt = W.make_logits(rows, V, "agent", dtype, seed=13, device="cuda", ld=ld)
+    rot_np = np.full(T, -1, np.int32)
+    rot_np[b.loss_mask == 1] = np.arange(rows, dtype=np.int32)
+    rot = torch.from_numpy(rot_np).cuda()
+    mask = torch.from_numpy(b.loss_mask).cuda()
+    w = torch.rand(T, generator=torch.Generator().manual_seed(8)).cuda()
+    dense = torch.full_like(zs, 3.0)
+    ids, gk, tl, loss, st = run_topk(P, zs, zt, V, mask, w, K, rot=rot, dense=dense,
+                                     flags=P.TURNOPD_ZERO_MASKED_GRAD)
+    assert st == 0
+    rids, rg = check_against_oracle(oracle, zs[:, :V], zt[:, :V], V, mask, w, K, ids, gk, tl, loss,
+                                    rot=rot)
+    m = b.loss_mask == 0
+    assert (ids[m] == -1).all() and (gk[m] == 0).all()
+    dn = dense.float().cpu().numpy()
+    assert (dn[:, V:] == 3.0).all()  # padding columns untouched
+    for t in np.nonzero(b.loss_mask)[0][:64]:
+        r = rot_np[t]
+        want = np.zeros(V)
+        want[rids[t]] = rg[t]
+        got = dn[r, :V]
+        tol = 1e-4 * np.abs(rg[t]).max()
+        if dtype == torch.bfloat16:
+            tol = np.maximum(tol, 2 * bf16_ulp(want))
+        assert (np.abs(got - want) <= tol + 1e-30).all()
+
+
+def test_full_vocab_packed_sampled_rows_and_properties(P, oracle):
+    """Bench-size rows (V = 151,936 bf16, compact): the oracle recomputes a few
+    rows; every row is checked by the selection's defining properties."""
+    b = W.packed(seed=0, num_traj=1, traj_len=4096)
+    V, K = W.V_QWEN, 50
+    R = b.num_valid
+    zs, zt = W.make_logits(R, V, "agent", torch.bfloat16, seed=1000, device="cuda")
+    T = b.num_tokens
+    rot_np = np.full(T, -1, np.int32)
+    rot_np[b.loss_mask == 1] = np.arange(R, dtype=np.int32)
+    rot = torch.from_numpy(rot_np).cuda()
+    mask = torch.from_numpy(b.loss_mask).cuda()
+    w = torch.rand(T, generator=torch.Generator().manual_seed(9)).cuda()
+    ids, gk, tl, loss, st = run_topk(P, zs, zt, V, mask, w, K, rot=rot)
+    assert st == 0
+    toks = np.nonzero(b.loss_mask)[0]
+    pick = list(toks[:2]) + list(toks[-2:]) + list(np.random.default_rng(0).choice(toks, 4, replace=False))
+    check_against_oracle(oracle, zs, zt, V, mask, w, K, ids, gk, tl, loss, rot=rot, subset=pick)
+    # properties on every row: the selected teacher logits are the K largest, in order
+    sel = torch.from_numpy(ids[toks].astype(np.int64)).cuda()
+    rows_t = torch.from_numpy(rot_np[toks].astype(np.int64)).cuda()
+    ztf = zt.float()
+    vals = torch.gather(ztf[rows_t], 1, sel)
+    assert bool((vals[:, :-1] >= vals[:, 1:]).all())
+    eq = vals[:, :-1] == vals[:, 1:]
+    assert bool((~eq | (sel[:, :-1] < sel[:, 1:])).all())
+    rest = ztf[rows_t].clone()
+    rest.scatter_(1, sel, -float("inf"))
+    kth = vals[:, -1:]
+    assert bool((rest.max(dim=1, keepdim=True).values <= kth).all())
+    # an unselected id equal to the K-th logit must come after every selected id of that logit
+    last_eq_id = torch.where(vals == kth, sel, torch.full_like(sel, -1)).max(dim=1, keepdim=True).values
+    ar = torch.arange(V, device="cuda").unsqueeze(0)
+    bad = (rest == kth) & (ar < last_eq_id)
+    assert not bool(bad.any())
+    assert (tl[toks] >= -1e-6).all()
+    assert abs(loss - float(np.dot(w.cpu().numpy().astype(np.float64)[toks], tl[toks].astype(np.float64)))) \
+        <= 1e-6 * abs(loss)
+
+
+def test_empty_and_all_masked(P):
+    V, K = 512, 8
+    zs = torch.zeros((4, V), dtype=torch.bfloat16, device="cuda")
+    mask = torch.zeros(4, dtype=torch.uint8, device="cuda")
+    w = torch.ones(4, dtype=torch.float32, device="cuda")
+    ids, gk, tl, loss, st = run_topk(P, zs, zs, V, mask, w, K)
+    assert st == 0 and loss == 0.0 and (tl == 0).all()
+    e = torch.zeros((0, V), dtype=torch.bfloat16, device="cuda")
+    ids, gk, tl, loss, st = run_topk(P, e, e, V, torch.zeros(0, dtype=torch.uint8, device="cuda"),
+                                     torch.zeros(0, dtype=torch.float32, device="cuda"), K)
+    assert st == 0 and loss == 0.0
