@@ -48,7 +48,8 @@ def parse():
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["native", "reference"], default="native")
     p.add_argument("--workload", default="packed", choices=["packed", "household", "multihop", "fused"])
-    p.add_argument("--mode", default="full", choices=["full", "sampled"])
+    p.add_argument("--mode", default="full", choices=["full", "sampled", "topk"])
+    p.add_argument("--k-top", type=int, default=50, help="support size of --mode topk")
     p.add_argument("--alpha", type=float, default=0.5)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -166,9 +167,11 @@ def build_inputs(args, rank, device):
         idx = torch.from_numpy(b.loss_mask.nonzero()[0]).to(device)
         y[idx] = y_c
     tid, msk, off, rot = to_device(b, device, compact=True)
+    k_top = args.k_top if args.mode == "topk" else 0
     step = LossStep(tid, msk, off, b.max_turns, V, row_of_token=rot, sampled_ids=y, mode=mode,
-                    alpha=args.alpha)
-    grad = torch.empty_like(zs)
+                    alpha=args.alpha, k_top=k_top)
+    # the top-K mode returns its gradient sparse: (ids, values) per token
+    grad = None if k_top else torch.empty_like(zs)
     return b, V, zs, zt, grad, step
 
 
@@ -189,7 +192,7 @@ def run_step(step, zs, zt, grad, world, dist, ev_pair=None):
         dp.reduce_step(step.loss, step.turn_sum, step.turn_cnt, step.turn_surv)
 
 
-def cpu_baseline(b, zs, zt, V, alpha, mode, rows_override=0, budget_s=15.0):
+def cpu_baseline(b, zs, zt, V, alpha, mode, rows_override=0, budget_s=15.0, k_top=0):
     """Time the fp64 CPU oracle on a bounded sample of the same workload: supervised
     rows in order, in chunks of 512 (so the oracle's fp64 gradient stays a few GB),
     until about `budget_s` seconds of oracle time or `rows_override` rows."""
@@ -208,12 +211,17 @@ def cpu_baseline(b, zs, zt, V, alpha, mode, rows_override=0, budget_s=15.0):
         n = min(chunk, limit - done)
         zsn, ztn = W.bf16_bits(zs[done:done + n]), W.bf16_bits(zt[done:done + n])
         t0 = time.perf_counter()
-        oracle.loss_fwd_bwd(zsn, ztn, V, np.ones(n, np.uint8), w[valid[done:done + n]], mode=0)
+        if k_top:
+            oracle.topk_loss(zsn, ztn, V, np.ones(n, np.uint8), w[valid[done:done + n]], k_top)
+        else:
+            oracle.loss_fwd_bwd(zsn, ztn, V, np.ones(n, np.uint8), w[valid[done:done + n]], mode=0)
         spent += time.perf_counter() - t0
         done += n
+    what = (f"teacher top-{k_top} reverse KL and its sparse gradient" if k_top
+            else "full-vocabulary loss and gradient")
     return {"value": done / spent, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
-            "sample": f"first {done} supervised rows of the same batch, full-vocabulary loss and "
-                      f"gradient in fp64 ({spent:.1f} s of oracle time, chunks of {chunk} rows)"}
+            "sample": f"first {done} supervised rows of the same batch, {what} in fp64 "
+                      f"({spent:.1f} s of oracle time, chunks of {chunk} rows)"}
 
 
 def reference_arm(args, world, rank):
@@ -258,8 +266,8 @@ def reference_arm(args, world, rank):
     print(json.dumps(out), flush=True)
 
 
-# weights (3) + fused call (compaction 2, gathers 2, W_s transpose, statistics pass,
-# merge, gradient pass, masked-row zeroing, dL/dh_s, loss sum) + turn statistics (2)
+# weights (3) + fused call (compaction 2, gathers 2, statistics pass, merge, gradient
+# pass, masked-row zeroing, dL/dh_s, dL/dh_s fix-up, loss sum) + turn statistics (2)
 FUSED_KERNELS_PER_STEP = 16
 
 
@@ -431,7 +439,11 @@ def main():
 
     value = tot_rows * args.steps / (ms / 1e3)
     peak, peak_kind = load_peaks()
-    bytes_per_row = 3 * V * 2  # two bf16 logit rows read + one bf16 gradient row written
+    if args.mode == "topk":
+        # teacher row read; the student logits at the K ids; K (id, value) outputs
+        bytes_per_row = V * 2 + args.k_top * (2 + 4 + 4)
+    else:
+        bytes_per_row = 3 * V * 2  # two bf16 logit rows read + one bf16 gradient row written
     alg_bytes = R * bytes_per_row
     loss_avg_ms = statistics.mean(loss_ms)
     achieved = alg_bytes / (loss_avg_ms / 1e3) / 1e9
@@ -442,7 +454,8 @@ def main():
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(b, zs, zt, V, args.alpha, 0, args.cpu_sample_rows)
+        cpu = cpu_baseline(b, zs, zt, V, args.alpha, 0, args.cpu_sample_rows,
+                           k_top=args.k_top if args.mode == "topk" else 0)
 
     if rank == 0:
         out = {
@@ -452,18 +465,22 @@ def main():
             "config": {
                 "workload": f"{b.name}_V{V}", "tokens": b.num_tokens, "supervised_tokens": R,
                 "tokens_counted": "supervised (assistant) tokens", "vocab": V,
-                "layout": "compact rows (one per supervised token)", "grad_dtype": "bf16",
+                "layout": "compact rows (one per supervised token)",
+                "grad_dtype": "fp32 sparse (ids, values)" if args.mode == "topk" else "bf16",
                 "mode": args.mode, "alpha": args.alpha, "scope": "traj",
+                **({"k_top": args.k_top} if args.mode == "topk" else {}),
                 "l2": "inputs larger than L2 (%.1f GB streamed per step), no flush" % (alg_bytes / 1e9),
                 "packed_tokens_per_s": b.num_tokens * world * args.steps / (ms / 1e3),
             },
             "roofline": {
                 "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "peak_kind": peak_kind,
-                "kernel": "turnopd_loss_fwd_bwd launch sequence (row kernel + compaction + loss sum)",
+                "kernel": ("turnopd_topk_loss_fwd_bwd launch sequence (k_topk_rows + compaction + loss sum)"
+                           if args.mode == "topk" else
+                           "turnopd_loss_fwd_bwd launch sequence (row kernel + compaction + loss sum)"),
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "launch_ms": loss_avg_ms,
-                "traffic": committed_traffic(args.workload),
+                "traffic": None if args.mode == "topk" else committed_traffic(args.workload),
             },
             "gpu_launches": KERNELS_PER_STEP * args.steps,
             "clocks": clocks,

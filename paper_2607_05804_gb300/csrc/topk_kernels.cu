@@ -9,17 +9,18 @@
 // One CTA per row at a time (persistent).  Selection with 64-bit keys
 // (order-preserving logit bits << 32 | ~id, so larger key = larger logit,
 // then lower id):
-//   pass A   one read of the teacher row: every thread keeps the 4 largest
-//            keys of its elements; a vector of 8 is looked at element by
-//            element only when its packed max beats the thread's 4th key;
-//   bound    tau = the K-th largest logit among the 4 x 512 held keys: a
-//            lower bound of the row's K-th largest (a subset's K-th largest
-//            never exceeds the set's);
-//   collect  held keys >= tau go to a shared-memory buffer; a thread whose
-//            4th held key is >= tau may hold fewer than all of its keys >= tau
-//            and rescans its own elements (rare);  a buffer overflow (rows of
-//            many equal logits) raises tau to the K-th largest buffered key
-//            and collects again (bounded rounds);
+//   pass A   one read of the teacher row, warp-uniform: for every group of 16
+//            consecutive ids the largest logit is recorded in shared memory as
+//            a 16-bit ordered bucket (the top 16 bits of the order-preserving
+//            bits), and every thread keeps the largest logit it saw;
+//   bound    tau = the K-th largest of the 8 (or ceil(K/8)) largest lane
+//            maxima of every warp: K-th largest of distinct elements of the
+//            row, so a lower bound of the row's K-th largest logit;
+//   collect  only the groups whose bucket reaches tau's are read again (a few
+//            dozen per row), and their elements >= tau go to a shared-memory
+//            candidate buffer; a buffer overflow (rows of many equal logits)
+//            raises tau to the K-th largest buffered key and collects again
+//            (bounded rounds);
 //   select   the exact K-th largest buffered key by radix select, then each
 //            selected key's rank among the selected gives its position.
 // The KL over S is evaluated by one warp in fp32 with
@@ -35,10 +36,13 @@
 namespace turnopd {
 namespace {
 
-constexpr int kTkThreads = 512;
-constexpr int kTkHold = 4;        // keys each thread keeps during pass A
-constexpr int kTkCap = 4096;      // candidate buffer (keys)
+constexpr int kTkThreads = 256;   // 4 CTAs (rows) per SM
+constexpr int kTkCap = 1024;      // candidate buffer (keys and student logits)
+// candidate groups whose loads a thread issues together (bf16 / fp32)
+template <bool BF16>
+__host__ __device__ constexpr int tk_hits() { return BF16 ? 2 : 1; }
 constexpr int kTkRounds = 16;     // bound on overflow rounds
+constexpr int kTkGroup = 16;      // ids per recorded bucket
 
 __device__ __forceinline__ uint32_t ord16(uint32_t u)
 {
@@ -85,60 +89,52 @@ __device__ __forceinline__ uint32_t bf16_max8_ord(const uint4 &v)
     return ord16(__bfloat16_as_ushort(mm));
 }
 
-// Visit this thread's elements of one row in increasing id order, calling
-// f(key) for every element whose logit may reach `*thr` (an ordered value;
-// elements of smaller ordered value may be skipped).  f may raise *thr.
-template <bool BF16, class F>
-__device__ __forceinline__ void scan_row(const void *row, int64_t V, bool vec_ok, const uint32_t *thr, F &&f)
+// Ordered value of an element (16 significant bits for bf16, 32 for fp32).
+template <bool BF16>
+__device__ __forceinline__ uint32_t elem_ord(const void *row, int64_t e)
 {
-    constexpr int EPV = BF16 ? 8 : 4;  // elements per 16-byte vector
-    const int64_t nvec = vec_ok ? V / EPV : 0;
-    const uint4 *rv = static_cast<const uint4 *>(row);
-    for (int64_t j0 = threadIdx.x; j0 < nvec; j0 += 4 * kTkThreads) {
-        uint4 v[4];
+    return BF16 ? ord16(static_cast<const uint16_t *>(row)[e]) : ord32(static_cast<const uint32_t *>(row)[e]);
+}
+
+// 16-bit bucket of an ordered value: monotone in the value.
+template <bool BF16>
+__device__ __forceinline__ uint32_t bucket(uint32_t ord)
+{
+    return BF16 ? ord : ord >> 16;
+}
+
+// Largest ordered value of the elements e0 .. e0+15 of a row, clipped to V
+// (element by element: the partial last group and misaligned rows).
+template <bool BF16>
+__device__ __forceinline__ uint32_t group_max_ord_scalar(const void *row, int64_t V, int64_t g)
+{
+    const int64_t e0 = g * kTkGroup;
+    uint32_t m = 0;
+    for (int64_t e = e0; e < e0 + kTkGroup && e < V; ++e)
+        m = max(m, elem_ord<BF16>(row, e));
+    return m;
+}
+
+// Ordered values of the 16 elements held in the 16-byte vectors v[0 .. VPG).
+template <bool BF16>
+__device__ __forceinline__ void unpack_ords(const uint4 *v, uint32_t (&o)[kTkGroup])
+{
+    if (BF16) {
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int64_t j = j0 + (int64_t)u * kTkThreads;
-            if (j < nvec)
-                v[u] = __ldg(rv + j);
+        for (int q = 0; q < 2; ++q) {
+            const uint32_t w4[4] = {v[q].x, v[q].y, v[q].z, v[q].w};
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                o[q * 8 + e] = ord16(e & 1 ? w4[e >> 1] >> 16 : w4[e >> 1]);
         }
+    } else {
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int64_t j = j0 + (int64_t)u * kTkThreads;
-            if (j >= nvec)
-                break;
-            const uint32_t id0 = (uint32_t)(j * EPV);
-            if (BF16) {
-                if (bf16_max8_ord(v[u]) < *thr)
-                    continue;
-                const uint32_t w4[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const uint32_t o = ord16(e & 1 ? w4[e >> 1] >> 16 : w4[e >> 1]);
-                    if (o >= *thr)
-                        f(mkkey(o, id0 + e));
-                }
-            } else {
-                const float x0 = __uint_as_float(v[u].x), x1 = __uint_as_float(v[u].y);
-                const float x2 = __uint_as_float(v[u].z), x3 = __uint_as_float(v[u].w);
-                if (ord32(__float_as_uint(fmaxf(fmaxf(x0, x1), fmaxf(x2, x3)))) < *thr)
-                    continue;
-                const uint32_t w4[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-#pragma unroll
-                for (int e = 0; e < 4; ++e) {
-                    const uint32_t o = ord32(w4[e]);
-                    if (o >= *thr)
-                        f(mkkey(o, id0 + e));
-                }
-            }
+        for (int q = 0; q < 4; ++q) {
+            o[q * 4 + 0] = ord32(v[q].x);
+            o[q * 4 + 1] = ord32(v[q].y);
+            o[q * 4 + 2] = ord32(v[q].z);
+            o[q * 4 + 3] = ord32(v[q].w);
         }
-    }
-    // elements not covered by whole aligned vectors
-    for (int64_t e = nvec * EPV + threadIdx.x; e < V; e += kTkThreads) {
-        const uint32_t o = BF16 ? ord16(static_cast<const uint16_t *>(row)[e])
-                                : ord32(static_cast<const uint32_t *>(row)[e]);
-        if (o >= *thr)
-            f(mkkey(o, (uint32_t)e));
     }
 }
 
@@ -233,28 +229,38 @@ struct TopkArgs {
     int32_t *status;
 };
 
-// Dynamic shared memory: held keys, candidate buffer, the selected keys and
-// their gradients.
-constexpr size_t kTkSmem = sizeof(uint64_t) * (kTkThreads * kTkHold + kTkCap + kTopkMaxK) +
-                           sizeof(float) * kTopkMaxK;
+// Dynamic shared memory: candidate keys, selected keys, candidate student
+// logits, the selected student logits / gradients, then one 16-bit bucket per
+// group of 16 ids.
+constexpr size_t kTkFixedSmem =
+    sizeof(uint64_t) * (kTkCap + kTopkMaxK) + sizeof(float) * (kTkCap + kTopkMaxK);
+
+__host__ __device__ __forceinline__ int64_t topk_groups(int64_t V) { return (V + kTkGroup - 1) / kTkGroup; }
+
+size_t topk_smem_bytes(int64_t V) { return kTkFixedSmem + align256(sizeof(uint16_t) * (size_t)topk_groups(V)); }
 
 template <bool BF16>
-__global__ void __launch_bounds__(kTkThreads, 2) k_topk_rows(TopkArgs a)
+__global__ void __launch_bounds__(kTkThreads, 4) k_topk_rows(TopkArgs a)
 {
     extern __shared__ uint64_t tk_smem[];
-    uint64_t *s_held = tk_smem;
-    uint64_t *s_cand = s_held + kTkThreads * kTkHold;
+    uint64_t *s_cand = tk_smem;
     uint64_t *s_top = s_cand + kTkCap;
-    float *s_g = reinterpret_cast<float *>(s_top + kTopkMaxK);
+    float *s_cz = reinterpret_cast<float *>(s_top + kTopkMaxK);   // student logit of each candidate
+    float *s_g = s_cz + kTkCap;                                    // selected: student logit, then g
+    uint16_t *s_bucket = reinterpret_cast<uint16_t *>(s_g + kTopkMaxK);
     __shared__ SelScratch s_sel;
     __shared__ int s_n, s_over;
+    __shared__ uint32_t s_wtop[kTkThreads];  // per-warp largest maxima (at most 32 per warp)
+    __shared__ uint32_t s_tau;
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int K = a.K;
     const int n_rows = *a.nvalid;
     const size_t esz = BF16 ? 2 : 4;
     const int hi_val = BF16 ? 5 : 7;  // top byte of the ordered logit inside a key
-    const bool base_ok = ((reinterpret_cast<uintptr_t>(a.zt) | (uintptr_t)(a.ld * esz)) & 15u) == 0;
+    const bool vec_ok =
+        ((reinterpret_cast<uintptr_t>(a.zt) | reinterpret_cast<uintptr_t>(a.zs) | (uintptr_t)(a.ld * esz)) & 15u) == 0;
+    const int64_t ng = topk_groups(a.vocab);
 
     for (int j = blockIdx.x; j < n_rows; j += gridDim.x) {
         const int4 m = a.rows[j];
@@ -263,72 +269,171 @@ __global__ void __launch_bounds__(kTkThreads, 2) k_topk_rows(TopkArgs a)
         const char *zt_row = static_cast<const char *>(a.zt) + (size_t)m.y * (size_t)a.ld * esz;
         const char *zs_row = static_cast<const char *>(a.zs) + (size_t)m.y * (size_t)a.ld * esz;
 
-        // ---- pass A: this thread's 4 largest keys
-        uint64_t h0 = 0, h1 = 0, h2 = 0, h3 = 0;
-        uint32_t thr = 1;  // admit every finite logit until 4 are held
-        scan_row<BF16>(zt_row, a.vocab, base_ok, &thr, [&](uint64_t k) {
-            if (k <= h3)
-                return;
-            h3 = k;
-            if (h3 > h2) { const uint64_t t = h2; h2 = h3; h3 = t; }
-            if (h2 > h1) { const uint64_t t = h1; h1 = h2; h2 = t; }
-            if (h1 > h0) { const uint64_t t = h0; h0 = h1; h1 = t; }
-            // a later element (larger id) needs a strictly larger logit than the 4th key
-            if (h3 != 0)
-                thr = (uint32_t)(h3 >> 32) + 1u;
-        });
-        s_held[tid * kTkHold + 0] = h0;
-        s_held[tid * kTkHold + 1] = h1;
-        s_held[tid * kTkHold + 2] = h2;
-        s_held[tid * kTkHold + 3] = h3;
+        // ---- pass A: group buckets and the thread's largest logit.  Whole groups of a
+        // 16-byte aligned row are read as vectors, 8 loads (128 B) in flight per thread.
+        uint32_t tmax = 0;
+        const int ngv = vec_ok ? (int)(a.vocab / kTkGroup) : 0;
+        constexpr int VPG = BF16 ? 2 : 4;  // 16-byte vectors per group
+        constexpr int U = 8 / VPG;         // groups per batch
+        const uint4 *rv = reinterpret_cast<const uint4 *>(zt_row);
+        for (int g0 = tid; g0 < ngv; g0 += U * kTkThreads) {
+            uint4 v[U * VPG];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int g = g0 + u * kTkThreads;
+#pragma unroll
+                for (int q = 0; q < VPG; ++q)
+                    if (g < ngv)
+                        v[u * VPG + q] = __ldg(rv + (size_t)g * VPG + q);
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int g = g0 + u * kTkThreads;
+                if (g >= ngv)
+                    break;
+                uint32_t o;
+                if (BF16) {
+                    const uint32_t o0 = bf16_max8_ord(v[u * 2]), o1 = bf16_max8_ord(v[u * 2 + 1]);
+                    o = max(o0, o1);
+                } else {
+                    float mx = -INFINITY;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        mx = fmaxf(mx, fmaxf(fmaxf(__uint_as_float(v[u * 4 + q].x), __uint_as_float(v[u * 4 + q].y)),
+                                             fmaxf(__uint_as_float(v[u * 4 + q].z), __uint_as_float(v[u * 4 + q].w))));
+                    o = ord32(__float_as_uint(mx));
+                }
+                s_bucket[g] = (uint16_t)bucket<BF16>(o);
+                tmax = max(tmax, o);
+            }
+        }
+        // groups left: the partial last group, or every group of a misaligned row
+        for (int g = ngv + tid; g < (int)ng; g += kTkThreads) {
+            const uint32_t o = group_max_ord_scalar<BF16>(zt_row, a.vocab, g);
+            s_bucket[g] = (uint16_t)bucket<BF16>(o);
+            tmax = max(tmax, o);
+        }
+        // ---- lower bound of the K-th largest logit: every warp contributes the c largest
+        // of its lanes' maxima (c = max(ceil(K / warps), 8) <= 32); the K-th largest of
+        // these 16c distinct elements cannot exceed the row's K-th largest.  0 (admit
+        // everything) when c would exceed 32 or fewer than K maxima exist.
+        constexpr int kWarps = kTkThreads / 32;
+        const int cw = max((K + kWarps - 1) / kWarps, 8);
+        if (cw <= 32) {
+            bool taken = false;
+            for (int i = 0; i < cw; ++i) {
+                const uint32_t mx = __reduce_max_sync(0xffffffffu, taken ? 0u : tmax);
+                const unsigned who = __ballot_sync(0xffffffffu, !taken && tmax == mx);
+                if (who != 0u && lane == __ffs(who) - 1)
+                    taken = true;
+                if (lane == 0)
+                    s_wtop[warp * cw + i] = mx;
+            }
+        }
         if (tid == 0) {
             s_n = 0;
             s_over = 0;
+            s_tau = 0;
         }
         __syncthreads();
-
-        // ---- lower bound on the K-th largest logit (value bytes only)
-        uint64_t tau = block_kth_largest(s_held, kTkThreads * kTkHold, K, hi_val, 4, s_sel);
-        uint32_t tau_ord = (uint32_t)(tau >> 32);
-        if (tau_ord == 0)
-            tau_ord = 1;
-
-        auto append = [&](uint64_t k) {
-            const int p = atomicAdd(&s_n, 1);
-            if (p < kTkCap)
-                s_cand[p] = k;
-            else
-                s_over = 1;
-        };
-        // ---- collect: held keys >= tau, and a rescan where the 4 held may not be all
-        const uint64_t hk[4] = {h0, h1, h2, h3};
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-            if (hk[q] != 0 && hk[q] >= tau)
-                append(hk[q]);
-        if (h3 != 0 && h3 >= tau) {
-            const uint64_t lim = h3;
-            scan_row<BF16>(zt_row, a.vocab, base_ok, &tau_ord, [&](uint64_t k) {
-                if (k >= tau && k < lim)
-                    append(k);
-            });
+        if (cw <= 32 && tid < kWarps * cw) {
+            const uint32_t v = s_wtop[tid];
+            int gt = 0, ge = 0;
+            for (int u = 0; u < kWarps * cw; ++u) {
+                const uint32_t x = s_wtop[u];
+                gt += x > v;
+                ge += x >= v;
+            }
+            if (v != 0 && gt < K && ge >= K)
+                s_tau = v;  // every such thread writes the same value
         }
+        __syncthreads();
+        const uint32_t tau_ord = s_tau;
+        uint64_t tau = (uint64_t)tau_ord << 32;  // admits every id of logit >= tau_ord
+        auto append = [&](uint64_t k, float zsv) {
+            const int p = atomicAdd(&s_n, 1);
+            if (p < kTkCap) {
+                s_cand[p] = k;
+                s_cz[p] = zsv;
+            } else {
+                s_over = 1;
+            }
+        };
+        const uint4 *sv = reinterpret_cast<const uint4 *>(zs_row);
+        // the candidate elements of up to kTkHits whole groups, teacher and student
+        // vectors of all of them loaded before any is used
+        constexpr int kTkHits = tk_hits<BF16>();
+        auto take_groups = [&](const int (&hg)[kTkHits], int nh) {
+            uint4 vt[kTkHits * VPG], vs[kTkHits * VPG];
+#pragma unroll
+            for (int h = 0; h < kTkHits; ++h)
+#pragma unroll
+                for (int q = 0; q < VPG; ++q)
+                    if (h < nh) {
+                        vt[h * VPG + q] = __ldg(rv + (size_t)hg[h] * VPG + q);
+                        vs[h * VPG + q] = __ldg(sv + (size_t)hg[h] * VPG + q);
+                    }
+#pragma unroll
+            for (int h = 0; h < kTkHits; ++h) {
+                if (h >= nh)
+                    break;
+                uint32_t o[kTkGroup];
+                unpack_ords<BF16>(&vt[h * VPG], o);
+                const uint32_t e0 = (uint32_t)hg[h] * kTkGroup;
+#pragma unroll
+                for (int e = 0; e < kTkGroup; ++e) {
+                    const uint64_t k = mkkey(o[e], e0 + e);
+                    if (k >= tau) {
+                        const uint4 &x = vs[h * VPG + e / (16 / (int)esz)];
+                        const int wi = (e % (16 / (int)esz)) * (int)esz / 4;
+                        const uint32_t word = wi == 0 ? x.x : wi == 1 ? x.y : wi == 2 ? x.z : x.w;
+                        const float zsv = BF16 ? __uint_as_float(((e & 1) ? word >> 16 : word & 0xFFFFu) << 16)
+                                               : __uint_as_float(word);
+                        append(k, zsv);
+                    }
+                }
+            }
+        };
+        // elements >= tau live in groups whose bucket reaches tau's
+        auto collect = [&]() {
+            const uint32_t tb = bucket<BF16>((uint32_t)(tau >> 32));
+            int hg[kTkHits];
+            int nh = 0;
+            for (int g = tid; g < ngv; g += kTkThreads) {
+                if (s_bucket[g] < tb)
+                    continue;
+                hg[nh++] = g;
+                if (nh == kTkHits) {
+                    take_groups(hg, nh);
+                    nh = 0;
+                }
+            }
+            if (nh > 0)
+                take_groups(hg, nh);
+            // the partial last group and misaligned rows, element by element
+            for (int g = ngv + tid; g < (int)ng; g += kTkThreads) {
+                if (s_bucket[g] < tb)
+                    continue;
+                const int64_t e0 = (int64_t)g * kTkGroup;
+                for (int64_t e = e0; e < e0 + kTkGroup && e < a.vocab; ++e) {
+                    const uint64_t k = mkkey(elem_ord<BF16>(zt_row, e), (uint32_t)e);
+                    if (k >= tau)
+                        append(k, BF16 ? __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(zs_row)[e])
+                                       : reinterpret_cast<const float *>(zs_row)[e]);
+                }
+            }
+        };
+        collect();
         __syncthreads();
         // ---- overflow: raise tau to the K-th largest buffered key and collect again
         for (int round = 0; s_over && round < kTkRounds; ++round) {
             tau = block_kth_largest(s_cand, kTkCap, K, 7, 0, s_sel);
-            tau_ord = (uint32_t)(tau >> 32);
-            if (tau_ord == 0)
-                tau_ord = 1;
             if (tid == 0) {
                 s_n = 0;
                 s_over = 0;
             }
             __syncthreads();
-            scan_row<BF16>(zt_row, a.vocab, base_ok, &tau_ord, [&](uint64_t k) {
-                if (k >= tau)
-                    append(k);
-            });
+            collect();
             __syncthreads();
         }
         const bool failed = s_over != 0;
@@ -342,17 +447,23 @@ __global__ void __launch_bounds__(kTkThreads, 2) k_topk_rows(TopkArgs a)
             }
             continue;
         }
-        // ---- the K largest: exact K-th key, then positions by rank
-        const uint64_t kth = block_kth_largest(s_cand, nc, K, 7, 0, s_sel);
+        // ---- the K largest: each candidate's rank among the candidates is its position
+        // (keys are unique); a large buffer is first cut to the K largest by radix select
+        const uint64_t kth = nc <= kTkThreads ? 0 : block_kth_largest(s_cand, nc, K, hi_val, 0, s_sel);
         for (int i = tid; i < nc; i += kTkThreads) {
             const uint64_t k = s_cand[i];
             if (k < kth)
                 continue;
             int rank = 0;
-            for (int i2 = 0; i2 < nc; ++i2)
+            int i2 = 0;
+            for (; i2 + 4 <= nc; i2 += 4)
+                rank += (s_cand[i2] > k) + (s_cand[i2 + 1] > k) + (s_cand[i2 + 2] > k) + (s_cand[i2 + 3] > k);
+            for (; i2 < nc; ++i2)
                 rank += s_cand[i2] > k;
-            if (rank < K)
+            if (rank < K) {
                 s_top[rank] = k;
+                s_g[rank] = s_cz[i];
+            }
         }
         __syncthreads();
 
@@ -360,11 +471,8 @@ __global__ void __launch_bounds__(kTkThreads, 2) k_topk_rows(TopkArgs a)
         if (warp == 0) {
             float m_s = -INFINITY, m_t = -INFINITY;
             for (int r = lane; r < K; r += 32) {
-                const uint32_t id = key_id(s_top[r]);
                 const float zt_v = key_value<BF16>(s_top[r]);
-                const float zs_v = BF16 ? __bfloat162float(reinterpret_cast<const __nv_bfloat16 *>(zs_row)[id])
-                                        : reinterpret_cast<const float *>(zs_row)[id];
-                s_g[r] = zs_v;  // student logit, kept for the second sweep
+                const float zs_v = s_g[r];  // student logit, carried with the candidate
                 m_s = fmaxf(m_s, zs_v);
                 m_t = fmaxf(m_t, zt_v);
             }
@@ -466,28 +574,26 @@ cudaError_t launch_topk(const TopkCall &c, cudaStream_t stream)
                                 stream);
     TopkArgs a{c.zs, c.zt, c.ld, c.vocab, c.K, ws.rows, ws.nvalid, c.topk_ids, c.topk_grad, c.grad,
                c.grad_dtype, c.token_loss, ws.row_wl, c.status};
-    static int per_sm[64][2] = {};
     int dev = 0;
     if ((e = cudaGetDevice(&dev)) != cudaSuccess)
         return e;
     const int ti = c.in_dtype == TURNOPD_BF16 ? 0 : 1;
     auto kern = c.in_dtype == TURNOPD_BF16 ? k_topk_rows<true> : k_topk_rows<false>;
-    if (dev >= 64 || per_sm[dev][ti] == 0) {
-        if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kTkSmem)) !=
+    const size_t smem = topk_smem_bytes(c.vocab);
+    static size_t attr_smem[64][2] = {};
+    const int di = dev < 64 ? dev : 0;
+    if (attr_smem[di][ti] < smem) {
+        if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
             cudaSuccess)
             return e;
-        int nb = 0;
-        if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, kern, kTkThreads, kTkSmem)) != cudaSuccess)
-            return e;
-        if (nb < 1)
-            return cudaErrorInvalidConfiguration;
-        if (dev < 64)
-            per_sm[dev][ti] = nb;
-        else
-            per_sm[0][ti] = nb;
+        attr_smem[di][ti] = smem;
     }
-    const int grid = sms * per_sm[dev < 64 ? dev : 0][ti];
-    kern<<<grid, kTkThreads, kTkSmem, stream>>>(a);
+    int nb = 0;
+    if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, kern, kTkThreads, smem)) != cudaSuccess)
+        return e;
+    if (nb < 1)
+        return cudaErrorInvalidConfiguration;
+    kern<<<sms * nb, kTkThreads, smem, stream>>>(a);
     e = cudaGetLastError();
     if (e != cudaSuccess)
         return e;

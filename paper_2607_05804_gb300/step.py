@@ -7,20 +7,21 @@ from __future__ import annotations
 import torch
 
 from . import (TURNOPD_FULL_VOCAB, TURNOPD_SCOPE_TRAJ, turnopd_loss_fwd_bwd,
-               turnopd_loss_workspace_bytes, turnopd_turn_counts, turnopd_turn_stats,
-               turnopd_weights, turnopd_weights_workspace_bytes)
+               turnopd_loss_workspace_bytes, turnopd_topk_loss_fwd_bwd, turnopd_turn_counts,
+               turnopd_turn_stats, turnopd_weights, turnopd_weights_workspace_bytes)
 
 
 class LossStep:
     """Holds the per-batch metadata and output buffers of one packed batch.
 
     turn_id int32[T], loss_mask uint8[T], traj_offsets int64[B+1] (device),
-    row_of_token int32[T] or None, sampled_ids int32[T] or None.
+    row_of_token int32[T] or None, sampled_ids int32[T] or None.  k_top > 0 selects the
+    teacher top-K reverse KL (sparse outputs topk_ids / topk_grad [T, k_top]).
     """
 
     def __init__(self, turn_id, loss_mask, traj_offsets, max_turns, vocab, *, row_of_token=None,
                  sampled_ids=None, mode=TURNOPD_FULL_VOCAB, alpha=0.5, scope=TURNOPD_SCOPE_TRAJ,
-                 n_min=0, flags=0, device=None):
+                 n_min=0, flags=0, k_top=0, device=None):
         dev = turn_id.device if device is None else torch.device(device)
         self.turn_id, self.loss_mask, self.traj_offsets = turn_id, loss_mask, traj_offsets
         self.row_of_token, self.sampled_ids = row_of_token, sampled_ids
@@ -41,6 +42,10 @@ class LossStep:
         self.turn_surv = torch.zeros(max_turns, dtype=torch.int32, device=dev)
         self.counts = torch.zeros(2 * max_turns + 1, dtype=torch.int64, device=dev)
         self.dev_status = torch.zeros(1, dtype=torch.int32, device=dev)
+        self.k_top = int(k_top)
+        if self.k_top > 0:
+            self.topk_ids = torch.full((max(T, 1), self.k_top), -1, dtype=torch.int32, device=dev)
+            self.topk_grad = torch.zeros((max(T, 1), self.k_top), dtype=torch.float32, device=dev)
 
     def local_counts(self, stream=None):
         """Per-rank count vector (sum it over data-parallel ranks for global_counts)."""
@@ -55,6 +60,13 @@ class LossStep:
         return self.w[:self.T]
 
     def loss_fwd_bwd(self, z_student, z_teacher, grad=None, stream=None):
+        if self.k_top > 0:
+            turnopd_topk_loss_fwd_bwd(z_student, z_teacher, self.vocab, self.row_of_token,
+                                      self.loss_mask, self.w[:self.T], self.k_top,
+                                      self.topk_ids[:self.T], self.topk_grad[:self.T], grad,
+                                      self.flags, self.token_loss[:self.T], self.loss, self.ws_l,
+                                      self.dev_status, stream)
+            return self.loss
         turnopd_loss_fwd_bwd(z_student, z_teacher, self.vocab, self.row_of_token, self.sampled_ids,
                              self.loss_mask, self.w[:self.T], self.mode, grad, self.flags,
                              self.token_loss[:self.T], self.loss, self.ws_l, self.dev_status,
