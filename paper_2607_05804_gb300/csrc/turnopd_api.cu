@@ -214,7 +214,7 @@ turnopd_status turnopd_topk_loss_fwd_bwd(const void *z_student, const void *z_te
         return TURNOPD_ERR_UNSUPPORTED;
     if (num_tokens < 0 || num_tokens > INT32_MAX || vocab < 1 || vocab > INT32_MAX || ld < vocab ||
         num_rows < 0 || (!row_of_token && num_rows < num_tokens) || k_top < 1 || k_top > TURNOPD_TOPK_MAX ||
-        k_top > vocab || num_tokens * (int64_t)k_top > INT64_MAX / 8)
+        k_top > vocab || vocab > TURNOPD_TOPK_MAX_VOCAB || num_tokens * (int64_t)k_top > INT64_MAX / 8)
         return TURNOPD_ERR_SHAPE;
     const size_t esz = in_dtype == TURNOPD_BF16 ? 2 : 4;
     if (misaligned(z_student, esz) || misaligned(z_teacher, esz) ||

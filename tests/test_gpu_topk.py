@@ -119,7 +119,7 @@ def test_all_equal_row_takes_the_lowest_ids(P, oracle):
 
 
 def test_k_equals_v_is_the_full_kl(P, oracle):
-    T, V = 16, 700
+    T, V = 16, 256
     zs, zt = W.make_logits(T, V, "tiny", torch.float32, seed=5, device="cuda")
     mask = torch.ones(T, dtype=torch.uint8, device="cuda")
     w = torch.ones(T, dtype=torch.float32, device="cuda")
