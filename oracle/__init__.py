@@ -61,7 +61,7 @@ def _L():
                                             i32, P, P, P, P, i64]
         lib.oracle_turn_stats.argtypes = [P, P, P, P, i32, i64, i32, P, P, P, P, P]
         lib.oracle_fused_lmhead.argtypes = [P, P, i64, P, P, i64, i64, P, P, i64, i32,
-                                            P, P, P, P, P, i64]
+                                            P, P, P, P, P, P, i64]
         lib.oracle_topk_row.argtypes = [P, P, i32, i64, i32, f64, P, P, P, P]
         lib.oracle_topk_loss.argtypes = [P, P, i32, i64, i64, P, i64, P, P, i64, i32, P, P, P,
                                          P, P, P, i64]
@@ -178,9 +178,10 @@ def turn_stats(token_loss, turn_id, loss_mask, traj_offsets, max_turns):
 
 
 def fused_lmhead(h_s, W_s, h_t, W_t, loss_mask, w, mode=FULL_VOCAB, sampled_ids=None,
-                 subset=None):
+                 subset=None, dW=False):
     """bf16 bit arrays h_s [T, d_s], W_s [V, d_s], h_t [T, d_t], W_t [V, d_t]
-    -> (dh_s [T, d_s] float64, token_loss, loss)."""
+    -> (dh_s [T, d_s] float64, token_loss, loss), plus dW_s [V, d_s] float64 last
+    when dW is true (over the evaluated tokens)."""
     hs, Ws = _c(h_s, np.uint16), _c(W_s, np.uint16)
     ht, Wt = _c(h_t, np.uint16), _c(W_t, np.uint16)
     T, d_s = hs.shape
@@ -191,11 +192,14 @@ def fused_lmhead(h_s, W_s, h_t, W_t, loss_mask, w, mode=FULL_VOCAB, sampled_ids=
     y = _c(sampled_ids, np.int32)
     sub = _c(subset, np.int64)
     dh = np.zeros((max(T, 1), d_s), np.float64)
+    dw = np.zeros((V, d_s), np.float64) if dW else None
     tl = np.zeros(max(T, 1), np.float64)
     loss = np.zeros(1, np.float64)
     _check(_L().oracle_fused_lmhead(_p(hs), _p(Ws), d_s, _p(ht), _p(Wt), d_t, V, _p(msk),
-                                    _p(wf), T, int(mode), _p(y), _p(dh), _p(tl), _p(loss),
+                                    _p(wf), T, int(mode), _p(y), _p(dh), _p(dw), _p(tl), _p(loss),
                                     _p(sub), 0 if sub is None else sub.size), "fused_lmhead")
+    if dW:
+        return dh[:T], tl[:T], float(loss[0]), dw
     return dh[:T], tl[:T], float(loss[0])
 
 

@@ -31,7 +31,8 @@
  *                           (trajectory, turn) and per turn index, plus survivor
  *                           counts n_t (Sec. 5.1; kl_per_turn/num_traj keys).
  *   oracle_fused_lmhead  -- logits z = h W^T from the two LM heads, then the
- *                           row oracle, then dL/dh_s = g W_s.
+ *                           row oracle, then dL/dh_s = g W_s and
+ *                           dL/dW_s = sum_i g_i^T h_s,i.
  *   oracle_topk_row /    -- the paper's practical loss, the teacher top-K
  *   oracle_topk_loss        reverse KL (loss_mode topk_reverse_kl with support
  *                           size K_top = distill_topk = 50 in the full
@@ -493,11 +494,17 @@ int oracle_turn_stats(const double *token_loss, const int32_t *turn_id,
  * dh_s rows of masked tokens are 0.  subset (nullable) restricts the tokens
  * that are computed, as in oracle_loss_fwd_bwd.
  */
+/*
+ * dh_s [T, d_s] receives dL/dh_s (rows of unsupervised tokens 0); dW_s
+ * (nullable) [V, d_s] receives dL/dW_s = sum_i g_i^T h_s,i over the evaluated
+ * supervised tokens (the chain rule through z_s = h_s W_s^T), each sum taken
+ * in increasing token order.
+ */
 int oracle_fused_lmhead(const uint16_t *h_s, const uint16_t *W_s, int64_t d_s,
                         const uint16_t *h_t, const uint16_t *W_t, int64_t d_t,
                         int64_t V, const uint8_t *mask, const float *w, int64_t T,
                         int32_t mode, const int32_t *sampled_ids, double *dh_s,
-                        double *token_loss, double *loss,
+                        double *dW_s, double *token_loss, double *loss,
                         const int64_t *subset, int64_t n_subset)
 {
     if (V < 1 || d_s < 1 || d_t < 1 || T < 0)
@@ -516,6 +523,8 @@ int oracle_fused_lmhead(const uint16_t *h_s, const uint16_t *W_s, int64_t d_s,
             return OR_TOKEN_RANGE;
     }
     int err = OR_OK;
+    /* per evaluated token, its logit gradient row (kept for dW_s) */
+    double *gall = dW_s ? (double *)calloc((size_t)(n > 0 ? n : 1) * (size_t)V, sizeof(double)) : NULL;
 #pragma omp parallel for schedule(dynamic, 1)
     for (int64_t k = 0; k < n; ++k) {
         int64_t i = subset ? subset[k] : k;
@@ -523,7 +532,7 @@ int oracle_fused_lmhead(const uint16_t *h_s, const uint16_t *W_s, int64_t d_s,
             continue;
         double *zs = (double *)malloc(sizeof(double) * (size_t)V);
         double *zt = (double *)malloc(sizeof(double) * (size_t)V);
-        double *g = (double *)malloc(sizeof(double) * (size_t)V);
+        double *g = gall ? gall + (size_t)k * (size_t)V : (double *)malloc(sizeof(double) * (size_t)V);
         for (int64_t v = 0; v < V; ++v) {
             double a = 0.0, b = 0.0;
             for (int64_t c = 0; c < d_s; ++c)
@@ -541,7 +550,8 @@ int oracle_fused_lmhead(const uint16_t *h_s, const uint16_t *W_s, int64_t d_s,
             err = st;
             free(zs);
             free(zt);
-            free(g);
+            if (!gall)
+                free(g);
             continue;
         }
         double ell = out[2];
@@ -553,10 +563,33 @@ int oracle_fused_lmhead(const uint16_t *h_s, const uint16_t *W_s, int64_t d_s,
         token_loss[i] = ell;
         free(zs);
         free(zt);
-        free(g);
+        if (!gall)
+            free(g);
     }
-    if (err)
+    if (err) {
+        free(gall);
         return err;
+    }
+    if (dW_s) {
+        /* dW_s[v,c] = sum over evaluated supervised tokens (in order) of g_i[v] h_s[i,c] */
+#pragma omp parallel for schedule(dynamic, 16)
+        for (int64_t v = 0; v < V; ++v) {
+            double *row = dW_s + v * d_s;
+            for (int64_t c = 0; c < d_s; ++c)
+                row[c] = 0.0;
+            for (int64_t k = 0; k < n; ++k) {
+                int64_t i = subset ? subset[k] : k;
+                if (!mask[i])
+                    continue;
+                double gv = gall[(size_t)k * (size_t)V + (size_t)v];
+                if (gv == 0.0)
+                    continue;
+                for (int64_t c = 0; c < d_s; ++c)
+                    row[c] += gv * widen_bf16(h_s[i * d_s + c]);
+            }
+        }
+        free(gall);
+    }
     kahan_t L = {0, 0};
     for (int64_t k = 0; k < n; ++k) {
         int64_t i = subset ? subset[k] : k;

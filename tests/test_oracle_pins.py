@@ -552,7 +552,8 @@ def test_fused_matches_matmul_then_rows(oracle):
     zt = f[2] @ f[3].T
     assert np.array_equal(f32(zs).astype(np.float64), zs) and np.array_equal(f32(zt).astype(np.float64), zt)
     for mode in (0, 1):
-        dh, tl, loss = oracle.fused_lmhead(*bits, mask, w, mode=mode, sampled_ids=y)
+        dh, tl, loss, dw = oracle.fused_lmhead(*bits, mask, w, mode=mode, sampled_ids=y, dW=True)
+        G = np.zeros((T, V))
         for i in range(T):
             if not mask[i]:
                 assert tl[i] == 0 and not dh[i].any()
@@ -560,4 +561,37 @@ def test_fused_matches_matmul_then_rows(oracle):
             _, _, ell, _, g = oracle.row(f32(zs[i]), f32(zt[i]), mode=mode, y=int(y[i]), w=float(w[i]))
             assert tl[i] == ell
             np.testing.assert_allclose(dh[i], g @ f[1], rtol=1e-12, atol=1e-15)
+            G[i] = g
+        np.testing.assert_allclose(dw, G.T @ f[0], rtol=1e-12, atol=1e-15)
         assert math.isclose(loss, float(np.dot(w.astype(np.float64), tl)), rel_tol=1e-12)
+
+
+def test_fused_gradients_match_finite_differences(oracle):
+    """dL/dh_s and dL/dW_s of the fused oracle against central differences of its
+    own loss.  Inputs on a grid of 1/32 and steps of 1/256 are exact in bf16."""
+    import torch
+
+    rng = np.random.default_rng(15)
+    T, d_s, d_t, V = 5, 6, 4, 9
+    def q(shape):
+        return rng.integers(-16, 17, shape).astype(np.float32) / 32.0
+    h_s, W_s, h_t, W_t = q((T, d_s)), q((V, d_s)), q((T, d_t)), q((V, d_t))
+    mask = np.array([1, 0, 1, 1, 1], np.uint8)
+    w = np.array([0.5, 0.0, 0.25, 1.0, 0.75], np.float32)
+    bits = lambda x: W.bf16_bits(torch.from_numpy(x).to(torch.bfloat16))
+    def loss(hs, Ws):
+        return oracle.fused_lmhead(bits(hs), bits(Ws), bits(h_t), bits(W_t), mask, w)[2]
+    dh, _, _, dw = oracle.fused_lmhead(bits(h_s), bits(W_s), bits(h_t), bits(W_t), mask, w, dW=True)
+    step = 1.0 / 256
+    for (i, c) in [(0, 0), (2, 3), (4, 5), (3, 1)]:
+        a, b = h_s.copy(), h_s.copy()
+        a[i, c] += step
+        b[i, c] -= step
+        fd = (loss(a, W_s) - loss(b, W_s)) / (2 * step)
+        assert abs(fd - dh[i, c]) <= 1e-4 * max(1.0, np.abs(dh).max()), (i, c, fd, dh[i, c])
+    for (v, c) in [(0, 0), (3, 2), (8, 5), (5, 4)]:
+        a, b = W_s.copy(), W_s.copy()
+        a[v, c] += step
+        b[v, c] -= step
+        fd = (loss(h_s, a) - loss(h_s, b)) / (2 * step)
+        assert abs(fd - dw[v, c]) <= 1e-4 * max(1.0, np.abs(dw).max()), (v, c, fd, dw[v, c])
