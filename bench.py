@@ -50,6 +50,7 @@ def parse():
     p.add_argument("--workload", default="packed", choices=["packed", "household", "multihop", "fused"])
     p.add_argument("--mode", default="full", choices=["full", "sampled", "topk"])
     p.add_argument("--k-top", type=int, default=50, help="support size of --mode topk")
+    p.add_argument("--dw", action="store_true", help="fused workload: also the weight gradient dL/dW_s")
     p.add_argument("--alpha", type=float, default=0.5)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -317,13 +318,14 @@ def fused_bench(args, world, rank, local):
     step = LossStep(tid, msk, off, b.max_turns, V, alpha=1.0)
     ws = torch.empty(P.turnopd_fused_workspace_bytes(T, V, d_s, d_t), dtype=torch.uint8, device=device)
     dh = torch.empty((T, d_s), dtype=torch.float32, device=device)
+    dW = torch.empty((V, d_s), dtype=torch.float32, device=device) if args.dw else None
 
     def one(ev=None):
         step.weights()
         if ev is not None:
             ev[0].record()
         P.turnopd_fused_lmhead_fwd_bwd(h_s, W_s, h_t, W_t, msk, step.w[:T], 0, dh,
-                                       step.token_loss[:T], step.loss, ws, step.dev_status)
+                                       step.token_loss[:T], step.loss, ws, step.dev_status, dW_s_out=dW)
         if ev is not None:
             ev[1].record()
         step.turn_stats()
@@ -349,6 +351,8 @@ def fused_bench(args, world, rank, local):
     call_ms = statistics.mean(x.elapsed_time(y) for x, y in evs)
     Tv = b.num_valid
     flops = 2.0 * Tv * V * (d_s + d_t) * 2 + 2.0 * Tv * V * d_s  # forward, recompute, dH
+    if args.dw:
+        flops += 2.0 * Tv * V * d_s  # dW_s
     peak = 1715.8
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as fh:
@@ -365,12 +369,14 @@ def fused_bench(args, world, rank, local):
            "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
            "config": {"workload": f"{b.name}_V{V}_ds{d_s}_dt{d_t}", "tokens": T, "supervised_tokens": Tv,
-                      "alpha": 1.0, "mode": "full", "flops_per_step": flops},
+                      "alpha": 1.0, "mode": "full", "flops_per_step": flops,
+                      "outputs": "loss, dL/dh_s" + (", dL/dW_s" if args.dw else "")},
            "roofline": {"bound": "tensor", "achieved": tflops, "peak": peak, "unit": "TFLOP/s",
                         "frac": tflops / peak, "peak_kind": peak_kind,
                         "kernel": "turnopd_fused_lmhead_fwd_bwd launch sequence", "launch_ms": call_ms,
                         "traffic": None},
-           "gpu_launches": FUSED_KERNELS_PER_STEP * args.steps, "clocks": clocks, "e2e": None,
+           "gpu_launches": (FUSED_KERNELS_PER_STEP + (1 if args.dw else 0)) * args.steps, "clocks": clocks,
+           "e2e": None,
            "cpu_baseline": cpu}
     print(json.dumps(out), flush=True)
 

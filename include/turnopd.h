@@ -237,8 +237,10 @@ turnopd_status turnopd_loss_fwd_bwd_static(const void *z_student, const void *z_
  *   d_s must be a multiple of 256, d_t of 64; every pointer 16-byte aligned.
  *   mode: TURNOPD_FULL_VOCAB only (others return TURNOPD_ERR_UNSUPPORTED).
  * Outputs:
- *   dh_s_out  float32[num_tokens, d_s] or NULL (forward only); rows of masked
- *             tokens are zero.
+ *   dh_s_out  float32[num_tokens, d_s] or NULL; rows of masked tokens are zero.
+ *   dW_s_out  float32[vocab, d_s] or NULL: dL/dW_s = sum_i G_i^T h_s,i over the
+ *             supervised tokens (overwritten, not accumulated).
+ *   (both NULL: forward only)
  *   token_loss_out float32[num_tokens] (0 for masked tokens), loss_out double.
  * Workspace: turnopd_fused_workspace_bytes(num_tokens, vocab, d_s, d_t) bytes,
  *   queried with the device that will run the call current (gathered hidden
@@ -250,7 +252,7 @@ turnopd_status turnopd_fused_lmhead_fwd_bwd(const void *h_s, const void *W_s, in
                                             const void *h_t, const void *W_t, int64_t d_t,
                                             int64_t vocab, const uint8_t *loss_mask,
                                             const float *w, int64_t num_tokens, int32_t mode,
-                                            float *dh_s_out, float *token_loss_out,
+                                            float *dh_s_out, float *dW_s_out, float *token_loss_out,
                                             double *loss_out, void *workspace,
                                             size_t workspace_bytes, int32_t *dev_status,
                                             turnopd_stream_t stream);

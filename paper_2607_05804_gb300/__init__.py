@@ -79,8 +79,8 @@ def load():
         "turnopd_turn_stats": [P, P, P, P, i32, i64, i32, P, P, P, P, P, P, P],
         "turnopd_loss_fwd_bwd_static": [P, P, i32, i64, i64, i64, P, P, P, P, i64, i32, P, i32,
                                         u32, P, P, P, P],
-        "turnopd_fused_lmhead_fwd_bwd": [P, P, i64, P, P, i64, i64, P, P, i64, i32, P, P, P, P, sz,
-                                         P, P],
+        "turnopd_fused_lmhead_fwd_bwd": [P, P, i64, P, P, i64, i64, P, P, i64, i32, P, P, P, P, P,
+                                         sz, P, P],
         "turnopd_topk_loss_fwd_bwd": [P, P, i32, i64, i64, i64, P, P, P, i64, i32, P, P, P, i32, u32,
                                       P, P, P, sz, P, P],
     }
@@ -169,8 +169,9 @@ def turnopd_fused_workspace_bytes(num_tokens: int, vocab: int, d_s: int, d_t: in
 
 
 def turnopd_fused_lmhead_fwd_bwd(h_s, W_s, h_t, W_t, loss_mask, w, mode, dh_s_out, token_loss_out,
-                                 loss_out, workspace, dev_status, stream=None):
-    """h_s [T, d_s], W_s [V, d_s], h_t [T, d_t], W_t [V, d_t] bf16; dh_s_out [T, d_s] fp32 or None."""
+                                 loss_out, workspace, dev_status, stream=None, dW_s_out=None):
+    """h_s [T, d_s], W_s [V, d_s], h_t [T, d_t], W_t [V, d_t] bf16; dh_s_out [T, d_s] fp32 or
+    None; dW_s_out [V, d_s] fp32 or None."""
     import torch
 
     T, d_s = h_s.shape
@@ -185,13 +186,14 @@ def turnopd_fused_lmhead_fwd_bwd(h_s, W_s, h_t, W_t, loss_mask, w, mode, dh_s_ou
     _need(loss_mask, "loss_mask", torch.uint8, T)
     _need(w, "w", torch.float32, T)
     _need(dh_s_out, "dh_s_out", torch.float32, T * d_s)
+    _need(dW_s_out, "dW_s_out", torch.float32, V * d_s)
     _need(token_loss_out, "token_loss_out", torch.float32, T)
     _need(loss_out, "loss_out", torch.float64, 1)
     _need(workspace, "workspace")
     _need(dev_status, "dev_status", torch.int32, 1)
     _check(load().turnopd_fused_lmhead_fwd_bwd(
         _ptr(h_s), _ptr(W_s), d_s, _ptr(h_t), _ptr(W_t), d_t, V, _ptr(loss_mask), _ptr(w), T,
-        int(mode), _ptr(dh_s_out), _ptr(token_loss_out), _ptr(loss_out), _ptr(workspace),
+        int(mode), _ptr(dh_s_out), _ptr(dW_s_out), _ptr(token_loss_out), _ptr(loss_out), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream)),
         "turnopd_fused_lmhead_fwd_bwd")
 

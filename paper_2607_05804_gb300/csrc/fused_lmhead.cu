@@ -643,6 +643,127 @@ k_fused_dh(const __grid_constant__ CUtensorMap tG, const __grid_constant__ CUten
     pair_epilogue(sm, tmem, 256, rank);
 }
 
+// ----------------------------------------------------------------------------
+// dW_s = G^T H_s: [V, d_s] fp32, K = the supervised tokens (padded to the pair
+// tile with zero rows of G and H_s).  A = G read as an MN-major operand (its
+// columns are vocabulary ids), B = the gathered H_s read MN-major (columns are
+// d_s); two 256-column accumulators in tensor memory, so the epilogue's stores
+// of tile j overlap the MMAs of tile j+1.  Tiles: 256 vocabulary rows x 256
+// columns of d_s, column tile fastest (pairs in flight share the G panel).
+struct DwArgs {
+    const int32_t *nvalid;
+    int64_t vocab;
+    int d_s;
+    float *dw;       // [vocab, d_s]
+    int32_t *status;
+};
+
+__global__ void __launch_bounds__(kThreads, 1)
+k_fused_dw(const __grid_constant__ CUtensorMap tGmn, const __grid_constant__ CUtensorMap tHmn, DwArgs a)
+{
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ int s_dead;
+    FusedSmem sm = carve(smem_raw, kDhBRegion, 0);
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const uint32_t rank = cluster_ctarank();
+    const int pair = (int)cluster_id(), n_pairs = (int)cluster_count();
+    const int nvalid = *a.nvalid;
+    const int kbs = (nvalid + BMP - 1) / BMP * (BMP / BK);
+    const int v_tiles = (int)((a.vocab + BMP - 1) / BMP);
+    const int d_tiles = a.d_s / BN;
+    const int tiles = kbs > 0 ? v_tiles * d_tiles : 0;
+    const uint32_t tmem = pair_prologue(sm, &s_dead, 512);
+    uint64_t *accf[2] = {sm.acc_t, sm.acc_s};
+    uint64_t *acce[2] = {sm.free_t, sm.free_s};
+
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&tGmn);
+        tma_prefetch_desc(&tHmn);
+        const uint32_t full0 = mapa(smem_u32(sm.full), 0);
+        uint32_t it = 0;
+        for (int t = pair; t < tiles; t += n_pairs) {
+            const int mv = t / d_tiles, nd = t % d_tiles;
+            const int xa = mv * BMP + (int)rank * BM;   // this CTA's 128 vocabulary ids
+            const int xb = nd * BN + (int)rank * BNH;   // this CTA's 128 columns of d_s
+            for (int kb = 0; kb < kbs; ++kb, ++it) {
+                const int s = it % STAGES;
+                if (it >= STAGES)
+                    wait_lim(&sm.empty[s], ((it / STAGES) - 1) & 1, a.status, &s_dead);
+                if (rank == 0)
+                    mbar_arrive_expect_tx(&sm.full[s], 2 * STAGE_BYTES);
+                const uint32_t fb = full0 + (uint32_t)s * 8u;
+#pragma unroll
+                for (int j = 0; j < BM / 64; ++j)
+                    tma_load_2d_pair(sm.a + s * A_BYTES + j * (64 * BK * 2), &tGmn, xa + j * 64, kb * BK, fb);
+#pragma unroll
+                for (int j = 0; j < BNH / 64; ++j)
+                    tma_load_2d_pair(sm.b + s * B_BYTES + j * (64 * BK * 2), &tHmn, xb + j * 64, kb * BK, fb);
+            }
+        }
+        drain_producer(sm, it, rank);
+    } else if (warp == 1 && lane == 0 && rank == 0 && kbs > 0) {
+        constexpr uint32_t idesc = idesc_bf16_f32(BMP, BN, true, true);
+        uint32_t it = 0, tile = 0;
+        for (int t = pair; t < tiles; t += n_pairs, ++tile) {
+            const int buf = tile & 1;
+            if (tile >= 2)  // both epilogues have read this buffer's previous tile
+                wait_lim(acce[buf], ((tile >> 1) - 1) & 1, a.status, &s_dead, true);
+            tc_fence_after();
+            for (int kb = 0; kb < kbs; ++kb, ++it) {
+                const int s = it % STAGES;
+                wait_lim(&sm.full[s], (it / STAGES) & 1, a.status, &s_dead);
+#pragma unroll
+                for (int k = 0; k < BK / 16; ++k) {
+                    // 16 K-rows (tokens) of 128 B per step; 64-wide M/N blocks 8 KB apart
+                    const uint64_t ad = smem_desc_sw128_mn(smem_u32(sm.a + s * A_BYTES) + k * 2048, 64 * BK * 2, 1024);
+                    const uint64_t bd = smem_desc_sw128_mn(smem_u32(sm.b + s * B_BYTES) + k * 2048, 64 * BK * 2, 1024);
+                    tc_mma_pair(tmem + (uint32_t)buf * 256u, ad, bd, idesc, kb > 0 || k > 0);
+                }
+                tc_commit_pair(&sm.empty[s], kPairMask);
+            }
+            tc_commit_pair(accf[buf], kPairMask);
+        }
+    } else if (warp >= 2) {
+        const int ew = warp - 2, q = warp % 4, cq = ew / 4;
+        const uint32_t lane_off = (uint32_t)(q * 32) << 16;
+        const int col0 = cq * kEpiCols;
+        const uint32_t acce0[2] = {mapa(smem_u32(acce[0]), 0), mapa(smem_u32(acce[1]), 0)};
+        uint32_t tile = 0;
+        if (kbs == 0) {  // no supervised token: dW_s = 0
+            for (int t = pair; t < v_tiles * d_tiles; t += n_pairs) {
+                const int mv = t / d_tiles, nd = t % d_tiles;
+                const int64_t v = (int64_t)mv * BMP + (int)rank * BM + q * 32 + lane;
+                if (v < a.vocab) {
+                    float4 *d4 = reinterpret_cast<float4 *>(a.dw + v * a.d_s + nd * BN + col0);
+                    for (int jj = 0; jj < kEpiCols / 4; ++jj)
+                        d4[jj] = make_float4(0.f, 0.f, 0.f, 0.f);
+                }
+            }
+        }
+        for (int t = pair; t < tiles; t += n_pairs, ++tile) {
+            const int mv = t / d_tiles, nd = t % d_tiles, buf = tile & 1;
+            const int64_t v = (int64_t)mv * BMP + (int)rank * BM + q * 32 + lane;
+            wait_lim(accf[buf], (tile >> 1) & 1, a.status, &s_dead);
+            tc_fence_after();
+            float *dst = a.dw + v * a.d_s + nd * BN + col0;
+#pragma unroll 1
+            for (int ch = 0; ch < kEpiCols / 32; ++ch) {
+                float x[32];
+                tmem_ld32(tmem + lane_off + (uint32_t)buf * 256u + (uint32_t)(col0 + ch * 32), x);
+                tmem_ld_wait();
+                if (v < a.vocab) {
+                    float4 *d4 = reinterpret_cast<float4 *>(dst + ch * 32);
+#pragma unroll
+                    for (int jj = 0; jj < 8; ++jj)
+                        d4[jj] = make_float4(x[4 * jj], x[4 * jj + 1], x[4 * jj + 2], x[4 * jj + 3]);
+                }
+            }
+            release_cols(acce0[buf], lane);
+        }
+    }
+    pair_epilogue(sm, tmem, 512, rank);
+}
+
 // Sum the partial tiles of the split part of dH in pair order (P = pairs of
 // the dH launch, at most kMaxPairs) and write them to their token rows.  Job =
 // (split tile, 8-row block).
@@ -699,16 +820,23 @@ k_dh_fixup(const float *__restrict__ partial, const int4 *__restrict__ rows, con
 
 // ----------------------------------------------------------------------------
 // Gather the supervised hidden rows: out[j] = h[token of row j] (16-byte copies).
+// Rows from the supervised count up to the next pair-tile boundary are zeroed
+// (the weight-gradient GEMM reads them as zero-weight tokens).
 __global__ void k_gather_rows(const int4 *__restrict__ rows, const int32_t *__restrict__ nvalid,
                               const uint4 *__restrict__ h, int vec_per_row, uint4 *__restrict__ out)
 {
     const int n = *nvalid;
-    for (int j = blockIdx.x; j < n; j += gridDim.x) {
-        const int64_t tok = rows[j].x;
-        const uint4 *src = h + tok * vec_per_row;
+    const int n_pad = (n + BMP - 1) / BMP * BMP;
+    for (int j = blockIdx.x; j < n_pad; j += gridDim.x) {
         uint4 *dst = out + (int64_t)j * vec_per_row;
-        for (int c = threadIdx.x; c < vec_per_row; c += blockDim.x)
-            dst[c] = src[c];
+        if (j < n) {
+            const uint4 *src = h + (int64_t)rows[j].x * vec_per_row;
+            for (int c = threadIdx.x; c < vec_per_row; c += blockDim.x)
+                dst[c] = src[c];
+        } else {
+            for (int c = threadIdx.x; c < vec_per_row; c += blockDim.x)
+                dst[c] = make_uint4(0, 0, 0, 0);
+        }
     }
 }
 
@@ -840,7 +968,7 @@ cudaError_t launch_pairs(void (*kern)(KArgs...), int pairs, size_t smem, cudaStr
 template <class... KArgs>
 cudaError_t pairs_for(void (*kern)(KArgs...), size_t smem, int slot, int *pairs)
 {
-    static int cache[64][3] = {};
+    static int cache[64][4] = {};
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess)
@@ -912,15 +1040,19 @@ cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream)
     if (e != cudaSuccess)
         return e;
 
-    alignas(64) CUtensorMap tHs, tWs, tHt, tWt, tG, tGst, tWmn;
+    alignas(64) CUtensorMap tHs, tWs, tHt, tWt, tG, tGst, tWmn, tGmn, tHmn;
     if (!make_map(&tHs, L.hs, cap, c.d_s, BM, BK) || !make_map(&tWs, c.W_s, c.vocab, c.d_s, BNH, BK) ||
         !make_map(&tHt, L.ht, cap, c.d_t, BM, BK) || !make_map(&tWt, c.W_t, c.vocab, c.d_t, BNH, BK) ||
         !make_map(&tG, L.G, cap, vpad, BM, BK) || !make_map(&tGst, L.G, cap, vpad, 32, kEpiCols) ||
         // W_s as the MN-major B of dH: boxes of 64 d-columns x BK vocabulary rows
-        !make_map(&tWmn, c.W_s, c.vocab, c.d_s, BK, 64))
+        !make_map(&tWmn, c.W_s, c.vocab, c.d_s, BK, 64) ||
+        // G and the gathered H_s as the MN-major operands of dW_s: 64 columns x BK token rows
+        !make_map(&tGmn, L.G, cap, vpad, BK, 64) || !make_map(&tHmn, L.hs, cap, c.d_s, BK, 64))
         return cudaErrorInvalidValue;
 
-    int p_lm0 = 0, p_lm1 = 0, p_dh = 0;
+    int p_lm0 = 0, p_lm1 = 0, p_dh = 0, p_dw = 0;
+    if ((e = pairs_for(k_fused_dw, kDhSmem, 3, &p_dw)) != cudaSuccess)
+        return e;
     if ((e = pairs_for(k_fused_lm<0>, kFusedSmem, 0, &p_lm0)) != cudaSuccess ||
         (e = pairs_for(k_fused_lm<1>, kFusedSmem, 1, &p_lm1)) != cudaSuccess ||
         (e = pairs_for(k_fused_dh, kDhSmem, 2, &p_dh)) != cudaSuccess)
@@ -947,9 +1079,21 @@ cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream)
     e = cudaGetLastError();
     if (e != cudaSuccess)
         return e;
-    if (c.dh_s) {
+    if (c.dh_s || c.dW_s) {
         if ((e = launch_pairs(k_fused_lm<1>, p_lm1, kFusedSmem, stream, tHs, tWs, tHt, tWt, tGst, fa)) != cudaSuccess)
             return e;
+    }
+    if (c.dW_s) {
+        DwArgs wa;
+        wa.nvalid = L.nvalid;
+        wa.vocab = c.vocab;
+        wa.d_s = (int)c.d_s;
+        wa.dw = c.dW_s;
+        wa.status = c.status;
+        if ((e = launch_pairs(k_fused_dw, p_dw, kDhSmem, stream, tGmn, tHmn, wa)) != cudaSuccess)
+            return e;
+    }
+    if (c.dh_s) {
         launch_zero_masked_f32(c.mask, c.T, (int64_t)c.d_s, c.dh_s, stream);
         DhArgs da;
         da.rows = L.rows;

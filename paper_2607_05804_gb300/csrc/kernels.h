@@ -122,6 +122,7 @@ struct FusedCall {
     const uint8_t *mask;
     const float *w;
     float *dh_s;
+    float *dW_s;
     float *token_loss;
     double *loss;
     void *workspace;

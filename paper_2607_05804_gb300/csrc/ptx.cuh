@@ -287,13 +287,15 @@ __device__ __forceinline__ uint64_t smem_desc_sw128_mn(uint32_t saddr, uint32_t 
            | ((uint64_t)2 << 61);
 }
 
-// Instruction descriptor of kind::f16 with bf16 A and B (both K-major) and an
-// fp32 accumulator, for an M x N tile.  `b_mn_major` selects an MN-major B.
-__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool b_mn_major = false)
+// Instruction descriptor of kind::f16 with bf16 A and B and an fp32
+// accumulator, for an M x N tile.  `b_mn_major` / `a_mn_major` select an
+// MN-major B / A (K-major otherwise).
+__host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N, bool b_mn_major = false, bool a_mn_major = false)
 {
     return (1u << 4)                      // D: fp32
            | (1u << 7)                    // A: bf16
            | (1u << 10)                   // B: bf16
+           | ((a_mn_major ? 1u : 0u) << 15)  // A major-ness (0: K-major, 1: MN-major)
            | ((b_mn_major ? 1u : 0u) << 16)  // B major-ness (0: K-major, 1: MN-major)
            | ((uint32_t)(N >> 3) << 17)   // N / 8
            | ((uint32_t)(M >> 4) << 24);  // M / 16

@@ -263,7 +263,7 @@ turnopd_status turnopd_fused_lmhead_fwd_bwd(const void *h_s, const void *W_s, in
                                             const void *h_t, const void *W_t, int64_t d_t,
                                             int64_t vocab, const uint8_t *loss_mask,
                                             const float *w, int64_t num_tokens, int32_t mode,
-                                            float *dh_s_out, float *token_loss_out,
+                                            float *dh_s_out, float *dW_s_out, float *token_loss_out,
                                             double *loss_out, void *workspace,
                                             size_t workspace_bytes, int32_t *dev_status,
                                             turnopd_stream_t stream)
@@ -278,15 +278,22 @@ turnopd_status turnopd_fused_lmhead_fwd_bwd(const void *h_s, const void *W_s, in
         d_s % 256 != 0 || d_t < 64 || d_t % 64 != 0 || d_s > 65536 || d_t > 65536)
         return TURNOPD_ERR_SHAPE;
     if (misaligned(h_s, 16) || misaligned(W_s, 16) || misaligned(h_t, 16) || misaligned(W_t, 16) ||
-        (dh_s_out && misaligned(dh_s_out, 16)) || misaligned(loss_out, 8))
+        (dh_s_out && misaligned(dh_s_out, 16)) || (dW_s_out && misaligned(dW_s_out, 16)) ||
+        misaligned(loss_out, 8))
         return TURNOPD_ERR_SHAPE;
     if (!workspace || misaligned(workspace, 256) ||
         workspace_bytes < fused_workspace_bytes(num_tokens, vocab, d_s, d_t))
         return TURNOPD_ERR_WORKSPACE;
     cudaStream_t s = (cudaStream_t)stream;
-    if (num_tokens == 0)
+    if (num_tokens == 0) {
+        if (dW_s_out) {
+            const cudaError_t e = cudaMemsetAsync(dW_s_out, 0, sizeof(float) * (size_t)vocab * (size_t)d_s, s);
+            if (e != cudaSuccess)
+                return cuda_status(e);
+        }
         return cuda_status(cudaMemsetAsync(loss_out, 0, sizeof(double), s));
-    FusedCall c{h_s, W_s, h_t, W_t, d_s, d_t, vocab, num_tokens, loss_mask, w, dh_s_out,
+    }
+    FusedCall c{h_s, W_s, h_t, W_t, d_s, d_t, vocab, num_tokens, loss_mask, w, dh_s_out, dW_s_out,
                 token_loss_out, loss_out, workspace, dev_status};
     return cuda_status(launch_fused(c, s));
 }

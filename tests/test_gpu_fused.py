@@ -38,7 +38,7 @@ def assert_dh(dh_gpu, dh_ref):
     assert (fro <= 4e-3).all(), fro.max()
 
 
-def run_fused(P, b, d_s, d_t, V, seed, alpha=1.0, grad=True):
+def run_fused(P, b, d_s, d_t, V, seed, alpha=1.0, grad=True, dw=False):
     from paper_2607_05804_gb300.step import LossStep, to_device
 
     T = b.num_tokens
@@ -48,11 +48,15 @@ def run_fused(P, b, d_s, d_t, V, seed, alpha=1.0, grad=True):
     w = step.weights()
     ws = torch.empty(P.turnopd_fused_workspace_bytes(T, V, d_s, d_t), dtype=torch.uint8, device="cuda")
     dh = torch.full((T, d_s), 3.0, dtype=torch.float32, device="cuda") if grad else None
+    dW = torch.full((V, d_s), 5.0, dtype=torch.float32, device="cuda") if dw else None
     tl = torch.full((T,), 7.0, dtype=torch.float32, device="cuda")
     loss = torch.zeros(1, dtype=torch.float64, device="cuda")
-    P.turnopd_fused_lmhead_fwd_bwd(h_s, W_s, h_t, W_t, msk, w, 0, dh, tl, loss, ws, step.dev_status)
+    P.turnopd_fused_lmhead_fwd_bwd(h_s, W_s, h_t, W_t, msk, w, 0, dh, tl, loss, ws, step.dev_status,
+                                   dW_s_out=dW)
     torch.cuda.synchronize()
     assert step.status() == 0
+    if dw:
+        return (h_s, W_s, h_t, W_t), w.cpu().numpy(), dh, tl.cpu().numpy(), loss.item(), dW
     return (h_s, W_s, h_t, W_t), w.cpu().numpy(), dh, tl.cpu().numpy(), loss.item()
 
 
@@ -121,6 +125,42 @@ def test_fused_all_masked_and_single_row(P, oracle):
     g = dh.cpu().numpy()
     assert (np.delete(g, 57, axis=0) == 0).all()
     assert_dh(g[57:58], dh_ref[57:58])
+
+
+def test_fused_weight_gradient_small(P, oracle):
+    """dL/dW_s on a ragged case (V = 1000: partial last vocabulary tile; 305
+    supervised rows: partial last token tile) against the oracle, row by row."""
+    b = W.packed(seed=3, num_traj=2, traj_len=160)
+    d_s, d_t, V = 256, 192, 1000
+    heads, w, dh, tl, loss, dW = run_fused(P, b, d_s, d_t, V, seed=4, dw=True)
+    bits = [W.bf16_bits(x) for x in heads]
+    dh_ref, tl_ref, loss_ref, dw_ref = oracle.fused_lmhead(*bits, b.loss_mask, w, dW=True)
+    assert_token_loss(tl, tl_ref, b.loss_mask)
+    assert_loss(loss, loss_ref)
+    assert_dh(dh.cpu().numpy()[b.loss_mask == 1], dh_ref[b.loss_mask == 1])
+    assert_dh(dW.cpu().numpy(), dw_ref)
+
+
+def test_fused_weight_gradient_only_and_full_size_identity(P):
+    """dW_s without dh_s, then full-size heads: dW_s . W_s and dh_s . h_s both equal
+    sum_t,v G[t,v] z_s[t,v] for the same G."""
+    b = W.packed(seed=9, num_traj=1, traj_len=600)
+    d_s, d_t, V = 4096, 5120, W.V_QWEN
+    heads, w, dh, tl, loss, dW = run_fused(P, b, d_s, d_t, V, seed=10, dw=True)
+    h_s, W_s = heads[0], heads[1]
+    a = float((dW.double() * W_s.double()).sum())
+    bsum = float((dh.double() * h_s.double()).sum())
+    scale = float((dh.double().abs() * h_s.double().abs()).sum())
+    assert abs(a - bsum) <= 2e-3 * scale, (a, bsum, scale)
+    heads2, _, dh2, tl2, loss2, dW2 = run_fused(P, b, d_s, d_t, V, seed=10, grad=False, dw=True)
+    assert torch.equal(dW2, dW) and loss2 == loss
+
+
+def test_fused_weight_gradient_all_masked_is_zero(P):
+    b = W.packed(seed=11, num_traj=1, traj_len=200)
+    b.loss_mask[:] = 0
+    heads, w, dh, tl, loss, dW = run_fused(P, b, 256, 64, 700, seed=12, dw=True)
+    assert loss == 0.0 and (dW == 0).all()
 
 
 def test_fused_errors(P):
