@@ -309,6 +309,80 @@ turnopd_status turnopd_topk_loss_fwd_bwd(const void *z_student, const void *z_te
                                          int32_t *dev_status, turnopd_stream_t stream);
 
 /*
+ * ---- Adaptive rollout-depth controller and loss-allocation diagnostics ----
+ * (Sec. 4.1 "Adaptive Rollout-Depth Budgeting", Algorithm 1, and the
+ * loss-allocation diagnostics of Sec. 3).  Host functions: every pointer is
+ * HOST memory (the per-turn tables of turnopd_turn_stats, copied back by the
+ * caller); nothing runs on the GPU and nothing is allocated.  round() is
+ * round-half-to-even; turn indices t are 0-based.
+ *
+ *   K_t    = turn_sum[t] / turn_cnt[t] (0 where turn_cnt[t] = 0)
+ *   m_t    = [K_t]_+ n_t / n_0,  n_t = turn_surv[t];  q_t = m_t / (sum_j m_j + eps)
+ *   H_eff  = round(sum_t t q_t)
+ *   H_cov  = min{H : 1 - n_{H+1} / n_1 >= p} over the probe trajectories that
+ *            succeeded (all of them when use_success = 0), where n_h counts
+ *            those with at least h turns; refreshed only when at least
+ *            min_cov_traj probe trajectories succeeded, else kept
+ *   probe step k: H_ctrl = max(H_eff, H_cov), h_bar <- (1 - ema_alpha) h_bar + ema_alpha H_ctrl
+ *   plan for step k (1-based): h_hat = clip(round(h_bar) + 1, h_min, h_max);
+ *            probe = (k <= warmup_steps) or (probe_interval > 0 and k % probe_interval == 0);
+ *            h_roll = probe ? h_max : h_hat
+ * Errors: TURNOPD_ERR_NULL for a missing pointer, TURNOPD_ERR_SHAPE for
+ * out-of-range parameters (h_min < 1, h_max < h_min, ema_alpha outside [0, 1],
+ * coverage_p outside (0, 1], negative counts or intervals, k < 1).
+ */
+typedef struct {
+    int32_t h_min, h_max;     /* clamp of the applied depth (defaults 2, 50) */
+    double ema_alpha;         /* EMA weight on H_ctrl (0.30) */
+    double coverage_p;        /* success-length quantile p (0.80) */
+    int32_t min_cov_traj;     /* successes needed to refresh H_cov (8) */
+    int32_t use_success;      /* 1: success-conditioned lengths, 0: all probe trajectories (1) */
+    int32_t warmup_steps;     /* every step k <= warmup_steps is a probe (3) */
+    int32_t probe_interval;   /* then every probe_interval-th step (8; 0 = never) */
+    double eps;               /* in q_t (1e-8) */
+} turnopd_depth_params;
+
+typedef struct {
+    double h_bar;             /* EMA of H_ctrl; h_max at start */
+    double h_eff_bar;         /* last unrounded centroid sum_t t q_t */
+    int32_t h_eff, h_cov, h_ctrl;  /* last efficiency centroid, coverage bound (0 at start), their max */
+} turnopd_depth_state;
+
+void turnopd_depth_default_params(turnopd_depth_params *p);
+turnopd_status turnopd_depth_init(const turnopd_depth_params *p, turnopd_depth_state *s);
+turnopd_status turnopd_depth_plan(const turnopd_depth_params *p, const turnopd_depth_state *s, int64_t k,
+                                  int32_t *h_hat, int32_t *is_probe, int32_t *h_roll);
+/* After step k; a no-op unless k is a probe step.  The turn tables are those
+ * of the (uncensored) probe batch, max_turns entries each; traj_len[b] = turns
+ * of probe trajectory b, traj_success[b] in {0, 1}; m_out / q_out (nullable)
+ * receive m_t and q_t. */
+turnopd_status turnopd_depth_update(const turnopd_depth_params *p, turnopd_depth_state *s, int64_t k,
+                                    const double *turn_sum, const int64_t *turn_cnt,
+                                    const int32_t *turn_surv, int32_t max_turns,
+                                    const int32_t *traj_len, const uint8_t *traj_success,
+                                    int32_t num_traj, double *m_out, double *q_out);
+/* The two arms on their own. */
+turnopd_status turnopd_depth_efficiency(const double *turn_sum, const int64_t *turn_cnt,
+                                        const int32_t *turn_surv, int32_t max_turns, double eps,
+                                        double *m_out, double *q_out, double *h_eff_bar,
+                                        int32_t *h_eff);
+turnopd_status turnopd_depth_coverage(const int32_t *traj_len, const uint8_t *traj_success,
+                                      int32_t num_traj, double p, int32_t min_cov_traj,
+                                      int32_t use_success, int32_t previous, int32_t *h_cov);
+/*
+ * Loss-allocation diagnostics of one batch: b_out[t] = turn_cnt[t] / N (token
+ * share), s_out[t] = turn_sum[t] / sum turn_sum (KL loss share); over the
+ * reliable prefix P (turns 0.. while turn_surv >= n_min and > 0) with
+ * third = floor(P / 3): deep_out[0] = P, deep_out[1] = mean K_t over the deepest
+ * third / mean K_t over the shallowest third, deep_out[2] = mean turn_surv over
+ * the deepest third / turn_surv[0], deep_out[3] = sum of s_t over the deepest
+ * third (NaN when P < 3).
+ */
+turnopd_status turnopd_turn_diagnostics(const double *turn_sum, const int64_t *turn_cnt,
+                                        const int32_t *turn_surv, int32_t max_turns, int32_t n_min,
+                                        double *b_out, double *s_out, double *deep_out);
+
+/*
  * turnopd_turn_stats -- turn statistics of the per-token losses
  * (Eq. observed-turn-kl: K_t is the mean per-token reverse KL over the
  * supervised tokens at turn t, over trajectories that reach t; the survivor

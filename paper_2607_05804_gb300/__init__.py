@@ -23,7 +23,10 @@ __all__ = [
     "turnopd_loss_fwd_bwd", "turnopd_loss_workspace_bytes", "turnopd_turn_stats",
     "turnopd_alpha_schedule", "turnopd_status_string", "turnopd_loss_fwd_bwd_static",
     "TURNOPD_STATIC_MAX_TOKENS", "turnopd_fused_lmhead_fwd_bwd", "turnopd_fused_workspace_bytes",
-    "turnopd_topk_loss_fwd_bwd", "TURNOPD_TOPK_MAX",
+    "turnopd_topk_loss_fwd_bwd", "TURNOPD_TOPK_MAX", "TURNOPD_TOPK_MAX_VOCAB",
+    "turnopd_depth_params", "turnopd_depth_state", "turnopd_depth_default_params",
+    "turnopd_depth_init", "turnopd_depth_plan", "turnopd_depth_update", "turnopd_depth_efficiency",
+    "turnopd_depth_coverage", "turnopd_turn_diagnostics",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -37,6 +40,7 @@ TURNOPD_FORCE_PORTABLE = 0x100
 TURNOPD_MAX_TURNS = 4096
 TURNOPD_STATIC_MAX_TOKENS = 65536
 TURNOPD_TOPK_MAX = 1024
+TURNOPD_TOPK_MAX_VOCAB = 1 << 20
 
 STATUS_NAMES = {
     0: "TURNOPD_OK", 1: "TURNOPD_ERR_NULL", 2: "TURNOPD_ERR_SHAPE", 3: "TURNOPD_ERR_OFFSETS",
@@ -84,6 +88,16 @@ def load():
         "turnopd_topk_loss_fwd_bwd": [P, P, i32, i64, i64, i64, P, P, P, i64, i32, P, P, P, i32, u32,
                                       P, P, P, sz, P, P],
     }
+    D, Pp = ctypes.c_double, ctypes.POINTER
+    sig.update({
+        "turnopd_depth_default_params": [P],
+        "turnopd_depth_init": [P, P],
+        "turnopd_depth_plan": [P, P, i64, P, P, P],
+        "turnopd_depth_update": [P, P, i64, P, P, P, i32, P, P, i32, P, P],
+        "turnopd_depth_efficiency": [P, P, P, i32, D, P, P, P, P],
+        "turnopd_depth_coverage": [P, P, i32, D, i32, i32, i32, P],
+        "turnopd_turn_diagnostics": [P, P, P, i32, i32, P, P, P],
+    })
     for name, args in sig.items():
         fn = getattr(lib, name)
         fn.argtypes = args
@@ -96,6 +110,7 @@ def load():
     lib.turnopd_fused_workspace_bytes.restype = sz
     lib.turnopd_alpha_schedule.argtypes = [i64, i64, f64, f64]
     lib.turnopd_alpha_schedule.restype = f64
+    lib.turnopd_depth_default_params.restype = None
     lib.turnopd_status_string.argtypes = [ctypes.c_int]
     lib.turnopd_status_string.restype = ctypes.c_char_p
     _lib = lib
@@ -306,6 +321,105 @@ def turnopd_topk_loss_fwd_bwd(z_student, z_teacher, vocab, row_of_token, loss_ma
         _ptr(token_loss_out), _ptr(loss_out), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream)),
         "turnopd_topk_loss_fwd_bwd")
+
+
+# ---------------------------------------------------------------- rollout-depth controller (host)
+
+class turnopd_depth_params(ctypes.Structure):
+    _fields_ = [("h_min", ctypes.c_int32), ("h_max", ctypes.c_int32), ("ema_alpha", ctypes.c_double),
+                ("coverage_p", ctypes.c_double), ("min_cov_traj", ctypes.c_int32),
+                ("use_success", ctypes.c_int32), ("warmup_steps", ctypes.c_int32),
+                ("probe_interval", ctypes.c_int32), ("eps", ctypes.c_double)]
+
+
+class turnopd_depth_state(ctypes.Structure):
+    _fields_ = [("h_bar", ctypes.c_double), ("h_eff_bar", ctypes.c_double), ("h_eff", ctypes.c_int32),
+                ("h_cov", ctypes.c_int32), ("h_ctrl", ctypes.c_int32)]
+
+
+def _host(a, dtype):
+    import numpy as np
+
+    if hasattr(a, "detach"):  # torch tensor (any device): copied to host memory
+        a = a.detach().cpu().numpy()
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+def _hp(a):
+    return None if a is None else ctypes.c_void_p(a.ctypes.data)
+
+
+def turnopd_depth_default_params() -> turnopd_depth_params:
+    p = turnopd_depth_params()
+    load().turnopd_depth_default_params(ctypes.byref(p))
+    return p
+
+
+def turnopd_depth_init(params: turnopd_depth_params) -> turnopd_depth_state:
+    st = turnopd_depth_state()
+    _check(load().turnopd_depth_init(ctypes.byref(params), ctypes.byref(st)), "turnopd_depth_init")
+    return st
+
+
+def turnopd_depth_plan(params, state, k: int):
+    """-> (h_hat, is_probe, h_roll) for step k (1-based)."""
+    h, pr, roll = ctypes.c_int32(), ctypes.c_int32(), ctypes.c_int32()
+    _check(load().turnopd_depth_plan(ctypes.byref(params), ctypes.byref(state), int(k), ctypes.byref(h),
+                                     ctypes.byref(pr), ctypes.byref(roll)), "turnopd_depth_plan")
+    return h.value, bool(pr.value), roll.value
+
+
+def turnopd_depth_update(params, state, k: int, turn_sum, turn_cnt, turn_surv, traj_len, traj_success,
+                         want_mq=False):
+    """Host arrays (numpy or torch, copied to host).  Updates `state` in place; returns
+    (m, q) when want_mq."""
+    import numpy as np
+
+    ts, tc, sv = _host(turn_sum, np.float64), _host(turn_cnt, np.int64), _host(turn_surv, np.int32)
+    tl, su = _host(traj_len, np.int32), _host(traj_success, np.uint8)
+    T = ts.size
+    m = np.zeros(max(T, 1)) if want_mq else None
+    q = np.zeros(max(T, 1)) if want_mq else None
+    _check(load().turnopd_depth_update(ctypes.byref(params), ctypes.byref(state), int(k), _hp(ts), _hp(tc),
+                                       _hp(sv), T, _hp(tl), _hp(su), tl.size, _hp(m), _hp(q)),
+           "turnopd_depth_update")
+    return (m[:T], q[:T]) if want_mq else None
+
+
+def turnopd_depth_efficiency(turn_sum, turn_cnt, turn_surv, eps=1e-8):
+    """-> (m, q, h_eff_bar, h_eff)."""
+    import numpy as np
+
+    ts, tc, sv = _host(turn_sum, np.float64), _host(turn_cnt, np.int64), _host(turn_surv, np.int32)
+    T = ts.size
+    m, q = np.zeros(max(T, 1)), np.zeros(max(T, 1))
+    hb, he = ctypes.c_double(), ctypes.c_int32()
+    _check(load().turnopd_depth_efficiency(_hp(ts), _hp(tc), _hp(sv), T, float(eps), _hp(m), _hp(q),
+                                           ctypes.byref(hb), ctypes.byref(he)), "turnopd_depth_efficiency")
+    return m[:T], q[:T], hb.value, he.value
+
+
+def turnopd_depth_coverage(traj_len, traj_success, p=0.8, min_cov_traj=8, use_success=True, previous=0):
+    import numpy as np
+
+    tl, su = _host(traj_len, np.int32), _host(traj_success, np.uint8)
+    h = ctypes.c_int32()
+    _check(load().turnopd_depth_coverage(_hp(tl), _hp(su), tl.size, float(p), int(min_cov_traj),
+                                         int(bool(use_success)), int(previous), ctypes.byref(h)),
+           "turnopd_depth_coverage")
+    return h.value
+
+
+def turnopd_turn_diagnostics(turn_sum, turn_cnt, turn_surv, n_min=1):
+    """-> (b [T], s [T], deep [4] = prefix, deep/shallow KL ratio, deep support, deep loss budget)."""
+    import numpy as np
+
+    ts, tc, sv = _host(turn_sum, np.float64), _host(turn_cnt, np.int64), _host(turn_surv, np.int32)
+    T = ts.size
+    b, sh, deep = np.zeros(max(T, 1)), np.zeros(max(T, 1)), np.zeros(4)
+    _check(load().turnopd_turn_diagnostics(_hp(ts), _hp(tc), _hp(sv), T, int(n_min), _hp(b), _hp(sh),
+                                           _hp(deep)), "turnopd_turn_diagnostics")
+    return b[:T], sh[:T], deep
 
 
 def turnopd_turn_stats(token_loss, turn_id, loss_mask, traj_offsets, max_turns, traj_turn_sum,

@@ -19,7 +19,9 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(HERE, "libturnopd.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "--expt-relaxed-constexpr",
+# host code: no floating-point contraction (the controller's doubles follow a fixed order)
+FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-ffp-contract=off",
+         "--expt-relaxed-constexpr",
          "-Xptxas", "-warn-spills"]
 # Extra nvcc flags (e.g. tuning macros such as -DTURNOPD_ROW_THREADS=384) for experiments.
 EXTRA = os.environ.get("TURNOPD_NVCC_FLAGS", "").split()
