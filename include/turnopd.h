@@ -309,6 +309,46 @@ turnopd_status turnopd_topk_loss_fwd_bwd(const void *z_student, const void *z_te
                                          int32_t *dev_status, turnopd_stream_t stream);
 
 /*
+ * ---- Vocabulary-parallel split of the reverse KL (Eq. opd-rkl) ----
+ * For logits sharded by vocabulary columns across ranks.  Each rank passes
+ * the base pointers of ITS shard (shard_vocab columns, rows ld elements
+ * apart; the same token -> row map on every rank):
+ *   1. turnopd_vocab_shard_stats: per supervised token i, the shard's partial
+ *      row statistics stats_out[i, 0..5] = (m_s, S_s, A, d, m_t, S_t):
+ *      m = max logit, S = sum exp(z - m), d = (z_s - z_t) at the student's
+ *      largest logit, A = sum exp(z_s - m_s) ((z_s - z_t) - d)  (float32,
+ *      turnopd_vocab_stats_bytes(num_tokens) bytes; masked rows untouched);
+ *   2. the caller gathers every shard's stats into parts[n_shards, num_tokens, 6]
+ *      in shard order (e.g. an all-gather);
+ *   3. turnopd_vocab_stats_merge: the whole vocabulary's row statistics, merged
+ *      in shard order (identical bits on every rank);
+ *   4. turnopd_vocab_shard_loss_grad: token_loss_out[i] = KL_i (0 for masked
+ *      tokens), *loss_out = sum_i w_i KL_i (fixed order, fp64; the same on every
+ *      rank), and this shard's gradient columns
+ *      g = w_i exp(z_s - LSE_s) ((z_s - z_t) - E_p[z_s - z_t])  (grad_shard
+ *      nullable, [num_rows, ld] of grad_dtype; TURNOPD_ZERO_MASKED_GRAD zeroes
+ *      the rows of masked tokens).  Full-vocabulary mode only.
+ * All arrays are device memory; host errors as for turnopd_loss_fwd_bwd;
+ * device errors TURNOPD_ERR_TOKEN_RANGE and TURNOPD_ERR_NONFINITE.
+ */
+size_t turnopd_vocab_stats_bytes(int64_t num_tokens);
+turnopd_status turnopd_vocab_shard_stats(const void *z_student, const void *z_teacher, int32_t in_dtype,
+                                         int64_t ld, int64_t shard_vocab, int64_t num_rows,
+                                         const int32_t *row_of_token, const uint8_t *loss_mask,
+                                         int64_t num_tokens, float *stats_out, int32_t *dev_status,
+                                         turnopd_stream_t stream);
+turnopd_status turnopd_vocab_stats_merge(const float *parts, int32_t n_shards, const uint8_t *loss_mask,
+                                         int64_t num_tokens, float *merged_out, turnopd_stream_t stream);
+turnopd_status turnopd_vocab_shard_loss_grad(const void *z_student, const void *z_teacher, int32_t in_dtype,
+                                             int64_t ld, int64_t shard_vocab, int64_t num_rows,
+                                             const int32_t *row_of_token, const uint8_t *loss_mask,
+                                             const float *w, int64_t num_tokens, const float *merged_stats,
+                                             void *grad_shard, int32_t grad_dtype, uint32_t flags,
+                                             float *token_loss_out, double *loss_out, void *workspace,
+                                             size_t workspace_bytes, int32_t *dev_status,
+                                             turnopd_stream_t stream);
+
+/*
  * ---- Adaptive rollout-depth controller and loss-allocation diagnostics ----
  * (Sec. 4.1 "Adaptive Rollout-Depth Budgeting", Algorithm 1, and the
  * loss-allocation diagnostics of Sec. 3).  Host functions: every pointer is

@@ -27,6 +27,8 @@ __all__ = [
     "turnopd_depth_params", "turnopd_depth_state", "turnopd_depth_default_params",
     "turnopd_depth_init", "turnopd_depth_plan", "turnopd_depth_update", "turnopd_depth_efficiency",
     "turnopd_depth_coverage", "turnopd_turn_diagnostics",
+    "turnopd_vocab_stats_bytes", "turnopd_vocab_shard_stats", "turnopd_vocab_stats_merge",
+    "turnopd_vocab_shard_loss_grad",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -97,6 +99,10 @@ def load():
         "turnopd_depth_efficiency": [P, P, P, i32, D, P, P, P, P],
         "turnopd_depth_coverage": [P, P, i32, D, i32, i32, i32, P],
         "turnopd_turn_diagnostics": [P, P, P, i32, i32, P, P, P],
+        "turnopd_vocab_shard_stats": [P, P, i32, i64, i64, i64, P, P, i64, P, P, P],
+        "turnopd_vocab_stats_merge": [P, i32, P, i64, P, P],
+        "turnopd_vocab_shard_loss_grad": [P, P, i32, i64, i64, i64, P, P, P, i64, P, P, i32, u32, P, P, P,
+                                          sz, P, P],
     })
     for name, args in sig.items():
         fn = getattr(lib, name)
@@ -111,6 +117,8 @@ def load():
     lib.turnopd_alpha_schedule.argtypes = [i64, i64, f64, f64]
     lib.turnopd_alpha_schedule.restype = f64
     lib.turnopd_depth_default_params.restype = None
+    lib.turnopd_vocab_stats_bytes.argtypes = [i64]
+    lib.turnopd_vocab_stats_bytes.restype = sz
     lib.turnopd_status_string.argtypes = [ctypes.c_int]
     lib.turnopd_status_string.restype = ctypes.c_char_p
     _lib = lib
@@ -321,6 +329,77 @@ def turnopd_topk_loss_fwd_bwd(z_student, z_teacher, vocab, row_of_token, loss_ma
         _ptr(token_loss_out), _ptr(loss_out), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream)),
         "turnopd_topk_loss_fwd_bwd")
+
+
+# ---------------------------------------------------------------- vocabulary-parallel split
+
+def _shard_logits(z_student, z_teacher):
+    for name, z in (("z_student", z_student), ("z_teacher", z_teacher)):
+        if not z.is_cuda or z.dim() != 2 or z.stride(1) != 1:
+            raise ValueError(f"{name} must be a 2-D CUDA tensor with unit column stride")
+    if z_teacher.shape != z_student.shape or z_teacher.stride() != z_student.stride() \
+            or z_teacher.dtype != z_student.dtype:
+        raise ValueError("z_teacher must match z_student in shape, stride and dtype")
+    return z_student.stride(0), z_student.shape[1]
+
+
+def turnopd_vocab_stats_bytes(num_tokens: int) -> int:
+    return int(load().turnopd_vocab_stats_bytes(int(num_tokens)))
+
+
+def turnopd_vocab_shard_stats(z_student, z_teacher, row_of_token, loss_mask, stats_out, dev_status,
+                              stream=None):
+    """z_student, z_teacher: this rank's [num_rows, shard_vocab] column shard (row stride ld);
+    stats_out float32 [T, 6]."""
+    import torch
+
+    ld, Vr = _shard_logits(z_student, z_teacher)
+    T = loss_mask.numel()
+    _need(row_of_token, "row_of_token", torch.int32, T)
+    _need(loss_mask, "loss_mask", torch.uint8)
+    _need(stats_out, "stats_out", torch.float32, T * 6)
+    _need(dev_status, "dev_status", torch.int32, 1)
+    _check(load().turnopd_vocab_shard_stats(
+        _ptr(z_student), _ptr(z_teacher), _dtype_code(z_student, "z_student"), ld, Vr, z_student.shape[0],
+        _ptr(row_of_token), _ptr(loss_mask), T, _ptr(stats_out), _ptr(dev_status), _stream(stream)),
+        "turnopd_vocab_shard_stats")
+
+
+def turnopd_vocab_stats_merge(parts, loss_mask, merged_out, stream=None):
+    """parts float32 [n_shards, T, 6] (shard order) -> merged_out [T, 6]."""
+    import torch
+
+    T = loss_mask.numel()
+    _need(parts, "parts", torch.float32)
+    _need(loss_mask, "loss_mask", torch.uint8)
+    _need(merged_out, "merged_out", torch.float32, T * 6)
+    _check(load().turnopd_vocab_stats_merge(_ptr(parts), parts.shape[0], _ptr(loss_mask), T, _ptr(merged_out),
+                                            _stream(stream)), "turnopd_vocab_stats_merge")
+
+
+def turnopd_vocab_shard_loss_grad(z_student, z_teacher, row_of_token, loss_mask, w, merged_stats, grad_shard,
+                                  flags, token_loss_out, loss_out, workspace, dev_status, stream=None):
+    import torch
+
+    ld, Vr = _shard_logits(z_student, z_teacher)
+    T = loss_mask.numel()
+    if grad_shard is not None and (grad_shard.shape != z_student.shape or grad_shard.stride(0) != ld
+                                   or grad_shard.stride(1) != 1 or not grad_shard.is_cuda):
+        raise ValueError("grad_shard must match the logit shard in shape and row stride")
+    _need(row_of_token, "row_of_token", torch.int32, T)
+    _need(loss_mask, "loss_mask", torch.uint8)
+    _need(w, "w", torch.float32, T)
+    _need(merged_stats, "merged_stats", torch.float32, T * 6)
+    _need(token_loss_out, "token_loss_out", torch.float32, T)
+    _need(loss_out, "loss_out", torch.float64, 1)
+    _need(workspace, "workspace")
+    _need(dev_status, "dev_status", torch.int32, 1)
+    gdt = _dtype_code(grad_shard, "grad_shard") if grad_shard is not None else TURNOPD_F32
+    _check(load().turnopd_vocab_shard_loss_grad(
+        _ptr(z_student), _ptr(z_teacher), _dtype_code(z_student, "z_student"), ld, Vr, z_student.shape[0],
+        _ptr(row_of_token), _ptr(loss_mask), _ptr(w), T, _ptr(merged_stats), _ptr(grad_shard), gdt, int(flags),
+        _ptr(token_loss_out), _ptr(loss_out), _ptr(workspace), workspace.numel() * workspace.element_size(),
+        _ptr(dev_status), _stream(stream)), "turnopd_vocab_shard_loss_grad")
 
 
 # ---------------------------------------------------------------- rollout-depth controller (host)

@@ -92,6 +92,29 @@ void launch_zero_masked_f32(const uint8_t *mask, int64_t T, int64_t d, float *ou
 void launch_zero_masked_grad(const uint8_t *mask, const int32_t *row_of_token, int64_t T, int64_t num_rows,
                              int64_t ld, int64_t vocab, void *grad, int32_t grad_dtype, cudaStream_t stream);
 
+// Vocabulary-parallel split.
+struct VocabShardCall {
+    const void *zs, *zt;
+    int32_t in_dtype;
+    int64_t ld, vocab, num_rows;
+    const int32_t *row_of_token;
+    const uint8_t *mask;
+    const float *w;
+    int64_t T;
+    void *grad;
+    int32_t grad_dtype;
+    uint32_t flags;
+    float *token_loss;
+    double *loss;
+    void *workspace;
+    int32_t *status;
+};
+size_t vocab_stats_bytes(int64_t T);
+cudaError_t launch_vocab_shard_stats(const VocabShardCall &c, float *stats, cudaStream_t stream);
+cudaError_t launch_vocab_stats_merge(const float *parts, int n_shards, const uint8_t *mask, int64_t T,
+                                     float *merged, cudaStream_t stream);
+cudaError_t launch_vocab_shard_grad(const VocabShardCall &c, const float *merged, cudaStream_t stream);
+
 // Teacher top-K reverse KL.
 constexpr int kTopkMaxK = 1024;
 struct TopkCall {

@@ -252,6 +252,91 @@ turnopd_status turnopd_topk_loss_fwd_bwd(const void *z_student, const void *z_te
     return cuda_status(launch_topk(c, s));
 }
 
+size_t turnopd_vocab_stats_bytes(int64_t num_tokens) { return vocab_stats_bytes(num_tokens); }
+
+static turnopd_status vocab_common_checks(const void *z_student, const void *z_teacher, int32_t in_dtype, int64_t ld,
+                                          int64_t shard_vocab, int64_t num_rows, const int32_t *row_of_token,
+                                          const uint8_t *loss_mask, int64_t num_tokens, int32_t *dev_status)
+{
+    if (!dev_status || (num_tokens > 0 && (!z_student || !z_teacher || !loss_mask)))
+        return TURNOPD_ERR_NULL;
+    if (in_dtype != TURNOPD_F32 && in_dtype != TURNOPD_BF16)
+        return TURNOPD_ERR_UNSUPPORTED;
+    if (num_tokens < 0 || num_tokens > INT32_MAX || shard_vocab < 1 || shard_vocab > INT32_MAX ||
+        ld < shard_vocab || num_rows < 0 || (!row_of_token && num_rows < num_tokens))
+        return TURNOPD_ERR_SHAPE;
+    const size_t esz = in_dtype == TURNOPD_BF16 ? 2 : 4;
+    if (misaligned(z_student, esz) || misaligned(z_teacher, esz))
+        return TURNOPD_ERR_SHAPE;
+    return TURNOPD_OK;
+}
+
+turnopd_status turnopd_vocab_shard_stats(const void *z_student, const void *z_teacher, int32_t in_dtype, int64_t ld,
+                                         int64_t shard_vocab, int64_t num_rows, const int32_t *row_of_token,
+                                         const uint8_t *loss_mask, int64_t num_tokens, float *stats_out,
+                                         int32_t *dev_status, turnopd_stream_t stream)
+{
+    turnopd_status st = vocab_common_checks(z_student, z_teacher, in_dtype, ld, shard_vocab, num_rows, row_of_token,
+                                            loss_mask, num_tokens, dev_status);
+    if (st != TURNOPD_OK)
+        return st;
+    if (num_tokens > 0 && !stats_out)
+        return TURNOPD_ERR_NULL;
+    if (misaligned(stats_out, 4))
+        return TURNOPD_ERR_SHAPE;
+    if (num_tokens == 0)
+        return TURNOPD_OK;
+    VocabShardCall c{z_student, z_teacher, in_dtype, ld, shard_vocab, num_rows, row_of_token, loss_mask, nullptr,
+                     num_tokens, nullptr, TURNOPD_F32, 0u, nullptr, nullptr, nullptr, dev_status};
+    return cuda_status(launch_vocab_shard_stats(c, stats_out, (cudaStream_t)stream));
+}
+
+turnopd_status turnopd_vocab_stats_merge(const float *parts, int32_t n_shards, const uint8_t *loss_mask,
+                                         int64_t num_tokens, float *merged_out, turnopd_stream_t stream)
+{
+    if (num_tokens > 0 && (!parts || !loss_mask || !merged_out))
+        return TURNOPD_ERR_NULL;
+    if (n_shards < 1 || num_tokens < 0 || num_tokens > INT32_MAX)
+        return TURNOPD_ERR_SHAPE;
+    if (misaligned(parts, 4) || misaligned(merged_out, 4))
+        return TURNOPD_ERR_SHAPE;
+    if (num_tokens == 0)
+        return TURNOPD_OK;
+    return cuda_status(launch_vocab_stats_merge(parts, n_shards, loss_mask, num_tokens, merged_out,
+                                                (cudaStream_t)stream));
+}
+
+turnopd_status turnopd_vocab_shard_loss_grad(const void *z_student, const void *z_teacher, int32_t in_dtype,
+                                             int64_t ld, int64_t shard_vocab, int64_t num_rows,
+                                             const int32_t *row_of_token, const uint8_t *loss_mask, const float *w,
+                                             int64_t num_tokens, const float *merged_stats, void *grad_shard,
+                                             int32_t grad_dtype, uint32_t flags, float *token_loss_out,
+                                             double *loss_out, void *workspace, size_t workspace_bytes,
+                                             int32_t *dev_status, turnopd_stream_t stream)
+{
+    turnopd_status st = vocab_common_checks(z_student, z_teacher, in_dtype, ld, shard_vocab, num_rows, row_of_token,
+                                            loss_mask, num_tokens, dev_status);
+    if (st != TURNOPD_OK)
+        return st;
+    if (!loss_out || (num_tokens > 0 && (!w || !merged_stats || !token_loss_out)))
+        return TURNOPD_ERR_NULL;
+    if (grad_shard && grad_dtype != TURNOPD_F32 && grad_dtype != TURNOPD_BF16)
+        return TURNOPD_ERR_UNSUPPORTED;
+    if (flags & ~(uint32_t)TURNOPD_ZERO_MASKED_GRAD)
+        return TURNOPD_ERR_UNSUPPORTED;
+    if ((grad_shard && misaligned(grad_shard, grad_dtype == TURNOPD_BF16 ? 2 : 4)) || misaligned(loss_out, 8) ||
+        misaligned(merged_stats, 4))
+        return TURNOPD_ERR_SHAPE;
+    if (!workspace || misaligned(workspace, 256) || workspace_bytes < loss_workspace_bytes(num_tokens))
+        return TURNOPD_ERR_WORKSPACE;
+    cudaStream_t s = (cudaStream_t)stream;
+    if (num_tokens == 0)
+        return cuda_status(cudaMemsetAsync(loss_out, 0, sizeof(double), s));
+    VocabShardCall c{z_student, z_teacher, in_dtype, ld, shard_vocab, num_rows, row_of_token, loss_mask, w,
+                     num_tokens, grad_shard, grad_dtype, flags, token_loss_out, loss_out, workspace, dev_status};
+    return cuda_status(launch_vocab_shard_grad(c, merged_stats, s));
+}
+
 size_t turnopd_fused_workspace_bytes(int64_t num_tokens, int64_t vocab, int64_t d_s, int64_t d_t)
 {
     if (num_tokens < 0 || vocab < 1 || d_s < 1 || d_t < 1)
