@@ -506,6 +506,11 @@ def e2e_leg(args, step, zs, zt, grad, world, dist, device, R):
 
     h_zs = torch.empty(zs.shape, dtype=zs.dtype, pin_memory=True)
     h_zt = torch.empty(zt.shape, dtype=zt.dtype, pin_memory=True)
+    # Host-resident logits are written by the CPU; pinned pages that only a
+    # device->host DMA ever wrote copy back at half the rate on a GB300 host
+    # (measured 99 vs 211 GB/s), so the pages are touched from the CPU first.
+    h_zs.zero_()
+    h_zt.zero_()
     h_zs.copy_(zs)
     h_zt.copy_(zt)
     meta = [step.turn_id, step.loss_mask, step.traj_offsets, step.row_of_token]
