@@ -51,6 +51,9 @@ def parse():
     p.add_argument("--mode", default="full", choices=["full", "sampled", "topk"])
     p.add_argument("--k-top", type=int, default=50, help="support size of --mode topk")
     p.add_argument("--dw", action="store_true", help="fused workload: also the weight gradient dL/dW_s")
+    p.add_argument("--vocab-shards", type=int, default=0,
+                   help="time the vocabulary-parallel path with this many column shards of one GPU's logits "
+                        "standing in for ranks (stats, ordered merge, shard gradients)")
     p.add_argument("--alpha", type=float, default=0.5)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -176,6 +179,35 @@ def build_inputs(args, rank, device):
     return b, V, zs, zt, grad, step
 
 
+def vocab_parallel_loss_fn(step, zs, zt, grad, n_shards):
+    """One loss call of the vocabulary-parallel path with n_shards column shards of
+    this GPU's logits: every shard's statistics, the ordered merge, every shard's
+    gradient columns (the work all ranks of an n_shards-way split do together)."""
+    import torch
+
+    import paper_2607_05804_gb300 as P
+
+    V = step.vocab
+    T = step.T
+    cuts = [V * r // n_shards for r in range(n_shards + 1)]
+    if not hasattr(step, "_vp"):
+        step._vp = (torch.empty((n_shards, T, 6), dtype=torch.float32, device=zs.device),
+                    torch.empty((T, 6), dtype=torch.float32, device=zs.device))
+    parts, merged = step._vp
+
+    def call():
+        for r in range(n_shards):
+            P.turnopd_vocab_shard_stats(zs[:, cuts[r]:cuts[r + 1]], zt[:, cuts[r]:cuts[r + 1]], step.row_of_token,
+                                        step.loss_mask, parts[r], step.dev_status)
+        P.turnopd_vocab_stats_merge(parts, step.loss_mask, merged)
+        for r in range(n_shards):
+            P.turnopd_vocab_shard_loss_grad(zs[:, cuts[r]:cuts[r + 1]], zt[:, cuts[r]:cuts[r + 1]],
+                                            step.row_of_token, step.loss_mask, step.w[:T], merged,
+                                            grad[:, cuts[r]:cuts[r + 1]], 0, step.token_loss[:T], step.loss,
+                                            step.ws_l, step.dev_status)
+    return call
+
+
 def run_step(step, zs, zt, grad, world, dist, ev_pair=None):
     from paper_2607_05804_gb300 import dp
 
@@ -185,7 +217,10 @@ def run_step(step, zs, zt, grad, world, dist, ev_pair=None):
         step.weights()
     if ev_pair is not None:
         ev_pair[0].record()
-    step.loss_fwd_bwd(zs, zt, grad)
+    if getattr(step, "vp_call", None) is not None:
+        step.vp_call()
+    else:
+        step.loss_fwd_bwd(zs, zt, grad)
     if ev_pair is not None:
         ev_pair[1].record()
     step.turn_stats()
@@ -405,6 +440,10 @@ def main():
     P.load()
     b, V, zs, zt, grad, step = build_inputs(args, rank, device)
     R = b.num_valid
+    if args.vocab_shards:
+        if args.mode != "full":
+            raise SystemExit("--vocab-shards times the full-vocabulary mode")
+        step.vp_call = vocab_parallel_loss_fn(step, zs, zt, grad, args.vocab_shards)
     torch.cuda.synchronize()
 
     for _ in range(max(args.warmup, 3)):
@@ -448,6 +487,9 @@ def main():
     if args.mode == "topk":
         # teacher row read; the student logits at the K ids; K (id, value) outputs
         bytes_per_row = V * 2 + args.k_top * (2 + 4 + 4)
+    elif args.vocab_shards:
+        # statistics pass (two logit rows read), gradient pass (read again, gradient written)
+        bytes_per_row = 5 * V * 2
     else:
         bytes_per_row = 3 * V * 2  # two bf16 logit rows read + one bf16 gradient row written
     alg_bytes = R * bytes_per_row
@@ -475,6 +517,7 @@ def main():
                 "grad_dtype": "fp32 sparse (ids, values)" if args.mode == "topk" else "bf16",
                 "mode": args.mode, "alpha": args.alpha, "scope": "traj",
                 **({"k_top": args.k_top} if args.mode == "topk" else {}),
+                **({"vocab_shards": args.vocab_shards} if args.vocab_shards else {}),
                 "l2": "inputs larger than L2 (%.1f GB streamed per step), no flush" % (alg_bytes / 1e9),
                 "packed_tokens_per_s": b.num_tokens * world * args.steps / (ms / 1e3),
             },
@@ -483,12 +526,15 @@ def main():
                 "frac": achieved / peak, "peak_kind": peak_kind,
                 "kernel": ("turnopd_topk_loss_fwd_bwd launch sequence (k_topk_rows + compaction + loss sum)"
                            if args.mode == "topk" else
+                           f"vocabulary-parallel path, {args.vocab_shards} shards of one GPU "
+                           "(shard stats + merge + shard gradients)" if args.vocab_shards else
                            "turnopd_loss_fwd_bwd launch sequence (row kernel + compaction + loss sum)"),
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "launch_ms": loss_avg_ms,
-                "traffic": None if args.mode == "topk" else committed_traffic(args.workload),
+                "traffic": None if (args.mode == "topk" or args.vocab_shards) else committed_traffic(args.workload),
             },
-            "gpu_launches": KERNELS_PER_STEP * args.steps,
+            # vocabulary shards: counts(2) + weights(1) + per shard stats, gradient and loss sum + merge + stats(2)
+            "gpu_launches": (KERNELS_PER_STEP if not args.vocab_shards else 6 + 3 * args.vocab_shards) * args.steps,
             "clocks": clocks,
             "e2e": e2e,
             "cpu_baseline": cpu,
