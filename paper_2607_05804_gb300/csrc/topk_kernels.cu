@@ -36,7 +36,14 @@
 namespace turnopd {
 namespace {
 
-constexpr int kTkThreads = 256;   // 4 CTAs (rows) per SM
+#ifndef TURNOPD_TOPK_THREADS
+#define TURNOPD_TOPK_THREADS 256
+#endif
+#ifndef TURNOPD_TOPK_MINB
+#define TURNOPD_TOPK_MINB 3
+#endif
+constexpr int kTkThreads = TURNOPD_TOPK_THREADS;  // one row per CTA, 3 CTAs per SM
+constexpr int kTkMinBlocks = TURNOPD_TOPK_MINB;   // 80 registers: the 4-CTA cap (64) spills the load batch
 constexpr int kTkCap = 1024;      // candidate buffer (keys and student logits)
 // candidate groups whose loads a thread issues together (bf16 / fp32)
 template <bool BF16>
@@ -240,7 +247,7 @@ __host__ __device__ __forceinline__ int64_t topk_groups(int64_t V) { return (V +
 size_t topk_smem_bytes(int64_t V) { return kTkFixedSmem + align256(sizeof(uint16_t) * (size_t)topk_groups(V)); }
 
 template <bool BF16>
-__global__ void __launch_bounds__(kTkThreads, 4) k_topk_rows(TopkArgs a)
+__global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs a)
 {
     extern __shared__ uint64_t tk_smem[];
     uint64_t *s_cand = tk_smem;
