@@ -6,16 +6,18 @@
 //   l   = sum_{v in S} ps_v (log ps_v - log pt_v)
 //   g_v = w ps_v (log ps_v - log pt_v - l)  on S, 0 elsewhere (= w dl/dz_s).
 //
-// One CTA per row at a time (persistent).  Selection with 64-bit keys
+// Persistent CTAs, each with two rows in flight: streaming warps run pass A
+// of a row while two selector warps run the later phases of the previous row
+// (double-buffered buckets, named barriers).  Selection with 64-bit keys
 // (order-preserving logit bits << 32 | ~id, so larger key = larger logit,
 // then lower id):
 //   pass A   one read of the teacher row, warp-uniform: for every group of 16
 //            consecutive ids the largest logit is recorded in shared memory as
 //            a 16-bit ordered bucket (the top 16 bits of the order-preserving
 //            bits), and every thread keeps the largest logit it saw;
-//   bound    tau = the K-th largest of the 8 (or ceil(K/8)) largest lane
-//            maxima of every warp: K-th largest of distinct elements of the
-//            row, so a lower bound of the row's K-th largest logit;
+//   bound    tau = the K-th largest of the 8 (or ceil(K/warps)) largest lane
+//            maxima of every streaming warp: K-th largest of distinct elements
+//            of the row, so a lower bound of the row's K-th largest logit;
 //   collect  only the groups whose bucket reaches tau's are read again (a few
 //            dozen per row), and their elements >= tau go to a shared-memory
 //            candidate buffer; a buffer overflow (rows of many equal logits)
@@ -36,14 +38,21 @@
 namespace turnopd {
 namespace {
 
-#ifndef TURNOPD_TOPK_THREADS
-#define TURNOPD_TOPK_THREADS 256
+#ifndef TURNOPD_TOPK_STREAM_WARPS
+#define TURNOPD_TOPK_STREAM_WARPS 8
 #endif
 #ifndef TURNOPD_TOPK_MINB
 #define TURNOPD_TOPK_MINB 3
 #endif
-constexpr int kTkThreads = TURNOPD_TOPK_THREADS;  // one row per CTA, 3 CTAs per SM
-constexpr int kTkMinBlocks = TURNOPD_TOPK_MINB;   // 80 registers: the 4-CTA cap (64) spills the load batch
+constexpr int kTkStreamWarps = TURNOPD_TOPK_STREAM_WARPS;  // pass A, row after row
+constexpr int kTkSelThreads = 64;                           // two selector warps
+constexpr int kTkStreamThreads = kTkStreamWarps * 32;
+constexpr int kTkThreads = kTkStreamThreads + kTkSelThreads;
+constexpr int kTkMinBlocks = TURNOPD_TOPK_MINB;  // CTAs (rows in flight) per SM
+// named barriers: buffer b full (1 + b), buffer b free (3 + b), selectors only (5),
+// streaming warps only (6)
+constexpr int kBarFull = 1, kBarFree = 3, kBarSel = 5, kBarStream = 6;
+constexpr int kTkGroupCap = 1024;  // candidate groups listed per row by the streaming warps
 constexpr int kTkCap = 1024;      // candidate buffer (keys and student logits)
 // candidate groups whose loads a thread issues together (bf16 / fp32)
 template <bool BF16>
@@ -145,36 +154,46 @@ __device__ __forceinline__ void unpack_ords(const uint4 *v, uint32_t (&o)[kTkGro
     }
 }
 
-// Block-wide radix select: the K-th largest of the nonzero keys in keys[0, n)
-// (keys are unique; 0 marks an empty slot), deciding bytes hi_byte..lo_byte.
-// Returns t such that {keys >= t} holds the K largest keys when lo_byte = 0
-// (exactly K), or, when lo_byte > 0, the K-th largest key with its lower bytes
-// cleared (every key of equal upper bytes is >= t).  Returns 0 when fewer than
-// K keys are present.  Stops early once the chosen bin holds exactly the
-// remaining count.  All threads call it; it synchronises the block.
+__device__ __forceinline__ void named_sync(int id, int n)
+{
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+__device__ __forceinline__ void named_arrive(int id, int n)
+{
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory");
+}
+
+// Radix select over the selector warps: the K-th largest of the nonzero keys
+// in keys[0, n) (keys are unique; 0 marks an empty slot), deciding bytes
+// hi_byte..lo_byte.  Returns t such that {keys >= t} holds the K largest keys
+// when lo_byte = 0 (exactly K), or, when lo_byte > 0, the K-th largest key
+// with its lower bytes cleared (every key of equal upper bytes is >= t).
+// Returns 0 when fewer than K keys are present.  Stops early once the chosen
+// bin holds exactly the remaining count.  Every selector thread (stid =
+// 0 .. kTkSelThreads-1) calls it; it synchronises them on kBarSel.
 struct SelScratch {
     uint32_t hist[256];
     int bin, need;
 };
 
-__device__ uint64_t block_kth_largest(const uint64_t *keys, int n, int K, int hi_byte, int lo_byte,
-                                      SelScratch &sc)
+__device__ uint64_t sel_kth_largest(const uint64_t *keys, int n, int K, int hi_byte, int lo_byte,
+                                    SelScratch &sc, int stid)
 {
-    const int tid = threadIdx.x, lane = tid & 31;
+    const int lane = stid & 31;
     uint64_t prefix = 0, mask = 0;
     int need = K;
     for (int byte = hi_byte; byte >= lo_byte; --byte) {
-        for (int i = tid; i < 256; i += kTkThreads)
+        for (int i = stid; i < 256; i += kTkSelThreads)
             sc.hist[i] = 0;
-        __syncthreads();
+        named_sync(kBarSel, kTkSelThreads);
         const int sh = 8 * byte;
-        for (int i = tid; i < n; i += kTkThreads) {
+        for (int i = stid; i < n; i += kTkSelThreads) {
             const uint64_t k = keys[i];
             if (k != 0 && (k & mask) == prefix)
                 atomicAdd(&sc.hist[(k >> sh) & 255u], 1u);
         }
-        __syncthreads();
-        if (tid < 32) {
+        named_sync(kBarSel, kTkSelThreads);
+        if (stid < 32) {
             int c[8], tot = 0;
 #pragma unroll
             for (int e = 0; e < 8; ++e) {
@@ -207,9 +226,9 @@ __device__ uint64_t block_kth_largest(const uint64_t *keys, int n, int K, int hi
                 }
             }
         }
-        __syncthreads();
+        named_sync(kBarSel, kTkSelThreads);
         const int bin = sc.bin, nd = sc.need;
-        __syncthreads();
+        named_sync(kBarSel, kTkSelThreads);
         if (bin < 0)
             return 0;
         prefix |= (uint64_t)bin << sh;
@@ -236,127 +255,196 @@ struct TopkArgs {
     int32_t *status;
 };
 
-// Dynamic shared memory: candidate keys, selected keys, candidate student
-// logits, the selected student logits / gradients, then one 16-bit bucket per
-// group of 16 ids.
-constexpr size_t kTkFixedSmem =
-    sizeof(uint64_t) * (kTkCap + kTopkMaxK) + sizeof(float) * (kTkCap + kTopkMaxK);
+// Dynamic shared memory: candidate keys, the K selected keys, candidate student
+// logits, the K selected student logits / gradients, then two buffers of one
+// 16-bit bucket per group of 16 ids.
+__host__ __device__ __forceinline__ size_t topk_fixed_bytes(int K)
+{
+    return align256(sizeof(uint64_t) * (kTkCap + (size_t)K) + sizeof(float) * (kTkCap + (size_t)K));
+}
 
 __host__ __device__ __forceinline__ int64_t topk_groups(int64_t V) { return (V + kTkGroup - 1) / kTkGroup; }
 
-size_t topk_smem_bytes(int64_t V) { return kTkFixedSmem + align256(sizeof(uint16_t) * (size_t)topk_groups(V)); }
+__host__ __device__ __forceinline__ size_t topk_bucket_bytes(int64_t V)
+{
+    return align256(sizeof(uint16_t) * (size_t)topk_groups(V));
+}
 
+size_t topk_smem_bytes(int64_t V, int K) { return topk_fixed_bytes(K) + 2 * topk_bucket_bytes(V); }
+
+// One CTA holds two rows at a time: its streaming warps run pass A of row
+// i + 1 (into bucket buffer (i + 1) % 2) while its two selector warps run
+// bound, collect, select and the KL of row i from buffer i % 2, so the SM's
+// teacher stream does not pause for the latency-bound phases.
 template <bool BF16>
 __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs a)
 {
-    extern __shared__ uint64_t tk_smem[];
+    extern __shared__ __align__(128) uint64_t tk_smem[];
+    const int K = a.K;
     uint64_t *s_cand = tk_smem;
     uint64_t *s_top = s_cand + kTkCap;
-    float *s_cz = reinterpret_cast<float *>(s_top + kTopkMaxK);   // student logit of each candidate
-    float *s_g = s_cz + kTkCap;                                    // selected: student logit, then g
-    uint16_t *s_bucket = reinterpret_cast<uint16_t *>(s_g + kTopkMaxK);
+    float *s_cz = reinterpret_cast<float *>(s_top + K);   // student logit of each candidate
+    float *s_g = s_cz + kTkCap;                            // selected: student logit, then g
+    uint16_t *s_bucket0 = reinterpret_cast<uint16_t *>(reinterpret_cast<unsigned char *>(tk_smem) +
+                                                       topk_fixed_bytes(K));
     __shared__ SelScratch s_sel;
+    __shared__ int4 s_meta[2];      // per buffer: the row (token, row, -, weight bits)
+
     __shared__ int s_n, s_over;
-    __shared__ uint32_t s_wtop[kTkThreads];  // per-warp largest maxima (at most 32 per warp)
-    __shared__ uint32_t s_tau;
+    __shared__ uint32_t s_wtop[2][kTkStreamThreads];  // per buffer: the c largest lane maxima of each warp
+    __shared__ uint32_t s_tau[2];                     // per buffer: the bound (ordered logit)
+    __shared__ int s_ng[2];                           // per buffer: candidate groups found
+    __shared__ uint16_t s_glist[2][kTkGroupCap];      // per buffer: their indices
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int K = a.K;
     const int n_rows = *a.nvalid;
+    const int n_it = n_rows > (int)blockIdx.x ? (n_rows - (int)blockIdx.x + (int)gridDim.x - 1) / (int)gridDim.x : 0;
     const size_t esz = BF16 ? 2 : 4;
-    const int hi_val = BF16 ? 5 : 7;  // top byte of the ordered logit inside a key
     const bool vec_ok =
         ((reinterpret_cast<uintptr_t>(a.zt) | reinterpret_cast<uintptr_t>(a.zs) | (uintptr_t)(a.ld * esz)) & 15u) == 0;
     const int64_t ng = topk_groups(a.vocab);
+    const int ngv = vec_ok ? (int)(a.vocab / kTkGroup) : 0;  // whole groups read as vectors
+    const size_t bucket_elems = topk_bucket_bytes(a.vocab) / sizeof(uint16_t);
+    constexpr int VPG = BF16 ? 2 : 4;  // 16-byte vectors per group
+    // lower bound of the K-th largest logit: every streaming warp contributes the cw largest
+    // of its lanes' maxima (cw = max(ceil(K / warps), 8) <= 32); the K-th largest of these
+    // distinct elements cannot exceed the row's K-th largest.  No bound (admit everything)
+    // when cw would exceed 32.
+    const int cw = max((K + kTkStreamWarps - 1) / kTkStreamWarps, 8);
 
-    for (int j = blockIdx.x; j < n_rows; j += gridDim.x) {
-        const int4 m = a.rows[j];
-        const int tok = m.x;
-        const float w = __int_as_float(m.w);
-        const char *zt_row = static_cast<const char *>(a.zt) + (size_t)m.y * (size_t)a.ld * esz;
-        const char *zs_row = static_cast<const char *>(a.zs) + (size_t)m.y * (size_t)a.ld * esz;
-
-        // ---- pass A: group buckets and the thread's largest logit.  Whole groups of a
-        // 16-byte aligned row are read as vectors, 8 loads (128 B) in flight per thread.
-        uint32_t tmax = 0;
-        const int ngv = vec_ok ? (int)(a.vocab / kTkGroup) : 0;
-        constexpr int VPG = BF16 ? 2 : 4;  // 16-byte vectors per group
-        constexpr int U = 8 / VPG;         // groups per batch
-        const uint4 *rv = reinterpret_cast<const uint4 *>(zt_row);
-        for (int g0 = tid; g0 < ngv; g0 += U * kTkThreads) {
-            uint4 v[U * VPG];
+    if (warp < kTkStreamWarps) {
+        // ---- streaming warps: pass A, one row after another
+        constexpr int U = 8 / VPG;  // groups per batch
+        // one batch of whole groups: 8 loads (128 B) in flight per thread
+        uint4 v[U * VPG];
+        auto load_batch = [&](const uint4 *rv, int g0) {
 #pragma unroll
             for (int u = 0; u < U; ++u) {
-                const int g = g0 + u * kTkThreads;
+                const int g = g0 + u * kTkStreamThreads;
 #pragma unroll
                 for (int q = 0; q < VPG; ++q)
                     if (g < ngv)
                         v[u * VPG + q] = __ldg(rv + (size_t)g * VPG + q);
             }
+        };
+        auto row_vectors = [&](const int4 &mr) {
+            return reinterpret_cast<const uint4 *>(static_cast<const char *>(a.zt) + (size_t)mr.y * (size_t)a.ld * esz);
+        };
+        int4 m_next = n_it > 0 ? a.rows[blockIdx.x] : make_int4(0, 0, -1, 0);
+        if (n_it > 0)
+            load_batch(row_vectors(m_next), tid);  // the first batch of each row is loaded a row ahead
+        for (int it = 0; it < n_it; ++it) {
+            const int b = it & 1;
+            const int4 m = m_next;  // loaded one row ahead
+            if (it + 1 < n_it)
+                m_next = a.rows[blockIdx.x + (it + 1) * gridDim.x];
+            if (it >= 2)
+                named_sync(kBarFree + b, kTkThreads);  // the selectors are done with row it - 2
+            if (tid == 0) {
+                s_meta[b] = m;
+                s_tau[b] = 0;
+            }
+            const char *zt_row = static_cast<const char *>(a.zt) + (size_t)m.y * (size_t)a.ld * esz;
+            uint16_t *s_bucket = s_bucket0 + b * bucket_elems;
+            // group buckets and the thread's largest logit; whole groups of a 16-byte
+            // aligned row are read as vectors, a batch at a time
+            uint32_t tmax = 0;
+            const uint4 *rv = reinterpret_cast<const uint4 *>(zt_row);
+            for (int g0 = tid; g0 < ngv; g0 += U * kTkStreamThreads) {
+                if (g0 != tid)
+                    load_batch(rv, g0);
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
-                const int g = g0 + u * kTkThreads;
-                if (g >= ngv)
-                    break;
-                uint32_t o;
-                if (BF16) {
-                    const uint32_t o0 = bf16_max8_ord(v[u * 2]), o1 = bf16_max8_ord(v[u * 2 + 1]);
-                    o = max(o0, o1);
-                } else {
-                    float mx = -INFINITY;
+                for (int u = 0; u < U; ++u) {
+                    const int g = g0 + u * kTkStreamThreads;
+                    if (g >= ngv)
+                        break;
+                    uint32_t o;
+                    if (BF16) {
+                        const uint32_t o0 = bf16_max8_ord(v[u * 2]), o1 = bf16_max8_ord(v[u * 2 + 1]);
+                        o = max(o0, o1);
+                    } else {
+                        float mx = -INFINITY;
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        mx = fmaxf(mx, fmaxf(fmaxf(__uint_as_float(v[u * 4 + q].x), __uint_as_float(v[u * 4 + q].y)),
-                                             fmaxf(__uint_as_float(v[u * 4 + q].z), __uint_as_float(v[u * 4 + q].w))));
-                    o = ord32(__float_as_uint(mx));
+                        for (int q = 0; q < 4; ++q)
+                            mx = fmaxf(mx, fmaxf(fmaxf(__uint_as_float(v[u * 4 + q].x), __uint_as_float(v[u * 4 + q].y)),
+                                                 fmaxf(__uint_as_float(v[u * 4 + q].z), __uint_as_float(v[u * 4 + q].w))));
+                        o = ord32(__float_as_uint(mx));
+                    }
+                    s_bucket[g] = (uint16_t)bucket<BF16>(o);
+                    tmax = max(tmax, o);
                 }
+            }
+            // groups left: the partial last group, or every group of a misaligned row
+            for (int g = ngv + tid; g < (int)ng; g += kTkStreamThreads) {
+                const uint32_t o = group_max_ord_scalar<BF16>(zt_row, a.vocab, g);
                 s_bucket[g] = (uint16_t)bucket<BF16>(o);
                 tmax = max(tmax, o);
             }
-        }
-        // groups left: the partial last group, or every group of a misaligned row
-        for (int g = ngv + tid; g < (int)ng; g += kTkThreads) {
-            const uint32_t o = group_max_ord_scalar<BF16>(zt_row, a.vocab, g);
-            s_bucket[g] = (uint16_t)bucket<BF16>(o);
-            tmax = max(tmax, o);
-        }
-        // ---- lower bound of the K-th largest logit: every warp contributes the c largest
-        // of its lanes' maxima (c = max(ceil(K / warps), 8) <= 32); the K-th largest of
-        // these 16c distinct elements cannot exceed the row's K-th largest.  0 (admit
-        // everything) when c would exceed 32 or fewer than K maxima exist.
-        constexpr int kWarps = kTkThreads / 32;
-        const int cw = max((K + kWarps - 1) / kWarps, 8);
-        if (cw <= 32) {
-            bool taken = false;
-            for (int i = 0; i < cw; ++i) {
-                const uint32_t mx = __reduce_max_sync(0xffffffffu, taken ? 0u : tmax);
-                const unsigned who = __ballot_sync(0xffffffffu, !taken && tmax == mx);
-                if (who != 0u && lane == __ffs(who) - 1)
-                    taken = true;
-                if (lane == 0)
-                    s_wtop[warp * cw + i] = mx;
+            if (it + 1 < n_it)
+                load_batch(row_vectors(m_next), tid);  // in flight while the row is settled below
+            if (cw <= 32) {
+                bool taken = false;
+                for (int i = 0; i < cw; ++i) {
+                    const uint32_t mx = __reduce_max_sync(0xffffffffu, taken ? 0u : tmax);
+                    const unsigned who = __ballot_sync(0xffffffffu, !taken && tmax == mx);
+                    if (who != 0u && lane == __ffs(who) - 1)
+                        taken = true;
+                    if (lane == 0)
+                        s_wtop[b][warp * cw + i] = mx;
+                }
             }
+            if (tid == 0)
+                s_ng[b] = 0;
+            named_sync(kBarStream, kTkStreamThreads);
+            if (cw <= 32) {
+                const int nw = kTkStreamWarps * cw;
+                for (int u0 = tid; u0 < nw; u0 += kTkStreamThreads) {
+                    const uint32_t v = s_wtop[b][u0];
+                    int gt = 0, ge = 0;
+                    for (int u = 0; u < nw; ++u) {
+                        const uint32_t x = s_wtop[b][u];
+                        gt += x > v;
+                        ge += x >= v;
+                    }
+                    if (v != 0 && gt < K && ge >= K)
+                        s_tau[b] = v;  // every such thread writes the same value
+                }
+            }
+            named_sync(kBarStream, kTkStreamThreads);
+            // the whole groups that can hold an element >= tau: their bucket reaches tau's
+            const uint32_t tb = bucket<BF16>(s_tau[b]);
+            for (int g = tid; g < ngv; g += kTkStreamThreads)
+                if (s_bucket[g] >= tb) {
+                    const int p = atomicAdd(&s_ng[b], 1);
+                    if (p < kTkGroupCap)
+                        s_glist[b][p] = (uint16_t)g;
+                }
+            named_arrive(kBarFull + b, kTkThreads);  // row it is in buffer b
         }
-        if (tid == 0) {
+        return;
+    }
+
+    // ---- selector warps: the phases after pass A, one row behind the stream
+    const int stid = tid - kTkStreamThreads, swarp = stid >> 5;
+    const int hi_val = BF16 ? 5 : 7;  // top byte of the ordered logit inside a key
+    for (int it = 0; it < n_it; ++it) {
+        const int b = it & 1;
+        const int j = blockIdx.x + it * gridDim.x;
+        named_sync(kBarFull + b, kTkThreads);
+        const int4 m = s_meta[b];
+        const int tok = m.x;
+        const float w = __int_as_float(m.w);
+        const char *zt_row = static_cast<const char *>(a.zt) + (size_t)m.y * (size_t)a.ld * esz;
+        const char *zs_row = static_cast<const char *>(a.zs) + (size_t)m.y * (size_t)a.ld * esz;
+        const uint16_t *s_bucket = s_bucket0 + b * bucket_elems;
+        if (stid == 0) {
             s_n = 0;
             s_over = 0;
-            s_tau = 0;
         }
-        __syncthreads();
-        if (cw <= 32 && tid < kWarps * cw) {
-            const uint32_t v = s_wtop[tid];
-            int gt = 0, ge = 0;
-            for (int u = 0; u < kWarps * cw; ++u) {
-                const uint32_t x = s_wtop[u];
-                gt += x > v;
-                ge += x >= v;
-            }
-            if (v != 0 && gt < K && ge >= K)
-                s_tau = v;  // every such thread writes the same value
-        }
-        __syncthreads();
-        const uint32_t tau_ord = s_tau;
-        uint64_t tau = (uint64_t)tau_ord << 32;  // admits every id of logit >= tau_ord
+        named_sync(kBarSel, kTkSelThreads);
+        uint64_t tau = (uint64_t)s_tau[b] << 32;  // admits every id of logit >= tau's
+        const int n_listed = s_ng[b];
+
         auto append = [&](uint64_t k, float zsv) {
             const int p = atomicAdd(&s_n, 1);
             if (p < kTkCap) {
@@ -366,10 +454,30 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
                 s_over = 1;
             }
         };
+        const uint4 *rv = reinterpret_cast<const uint4 *>(zt_row);
         const uint4 *sv = reinterpret_cast<const uint4 *>(zs_row);
         // the candidate elements of up to kTkHits whole groups, teacher and student
         // vectors of all of them loaded before any is used
         constexpr int kTkHits = tk_hits<BF16>();
+        // the candidate elements of one whole group: teacher vectors vt, student vectors vs
+        auto scan_group = [&](const uint4 *vt, const uint4 *vs, int g) {
+            uint32_t o[kTkGroup];
+            unpack_ords<BF16>(vt, o);
+            const uint32_t e0 = (uint32_t)g * kTkGroup;
+#pragma unroll
+            for (int e = 0; e < kTkGroup; ++e) {
+                const uint64_t k = mkkey(o[e], e0 + e);
+                if (k >= tau) {
+                    const uint4 &x = vs[e / (16 / (int)esz)];
+                    const int wi = (e % (16 / (int)esz)) * (int)esz / 4;
+                    const uint32_t word = wi == 0 ? x.x : wi == 1 ? x.y : wi == 2 ? x.z : x.w;
+                    const float zsv = BF16 ? __uint_as_float(((e & 1) ? word >> 16 : word & 0xFFFFu) << 16)
+                                           : __uint_as_float(word);
+                    append(k, zsv);
+                }
+            }
+        };
+        // groups read from global memory, kTkHits at a time, all loads before any use
         auto take_groups = [&](const int (&hg)[kTkHits], int nh) {
             uint4 vt[kTkHits * VPG], vs[kTkHits * VPG];
 #pragma unroll
@@ -384,31 +492,21 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
             for (int h = 0; h < kTkHits; ++h) {
                 if (h >= nh)
                     break;
-                uint32_t o[kTkGroup];
-                unpack_ords<BF16>(&vt[h * VPG], o);
-                const uint32_t e0 = (uint32_t)hg[h] * kTkGroup;
-#pragma unroll
-                for (int e = 0; e < kTkGroup; ++e) {
-                    const uint64_t k = mkkey(o[e], e0 + e);
-                    if (k >= tau) {
-                        const uint4 &x = vs[h * VPG + e / (16 / (int)esz)];
-                        const int wi = (e % (16 / (int)esz)) * (int)esz / 4;
-                        const uint32_t word = wi == 0 ? x.x : wi == 1 ? x.y : wi == 2 ? x.z : x.w;
-                        const float zsv = BF16 ? __uint_as_float(((e & 1) ? word >> 16 : word & 0xFFFFu) << 16)
-                                               : __uint_as_float(word);
-                        append(k, zsv);
-                    }
-                }
+                scan_group(&vt[h * VPG], &vs[h * VPG], hg[h]);
             }
         };
-        // elements >= tau live in groups whose bucket reaches tau's
-        auto collect = [&]() {
+        // elements >= tau live in groups whose bucket reaches tau's: the groups the
+        // streaming warps listed, or (list overflow, raised tau) a scan of the buckets
+        auto collect = [&](bool listed) {
             const uint32_t tb = bucket<BF16>((uint32_t)(tau >> 32));
             int hg[kTkHits];
             int nh = 0;
-            for (int g = tid; g < ngv; g += kTkThreads) {
-                if (s_bucket[g] < tb)
+            const int n_scan = listed ? n_listed : ngv;
+            for (int i = stid; i < n_scan; i += kTkSelThreads) {
+                const int g = listed ? (int)s_glist[b][i] : i;
+                if (!listed && s_bucket[g] < tb)
                     continue;
+
                 hg[nh++] = g;
                 if (nh == kTkHits) {
                     take_groups(hg, nh);
@@ -418,7 +516,7 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
             if (nh > 0)
                 take_groups(hg, nh);
             // the partial last group and misaligned rows, element by element
-            for (int g = ngv + tid; g < (int)ng; g += kTkThreads) {
+            for (int g = ngv + stid; g < (int)ng; g += kTkSelThreads) {
                 if (s_bucket[g] < tb)
                     continue;
                 const int64_t e0 = (int64_t)g * kTkGroup;
@@ -430,113 +528,115 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
                 }
             }
         };
-        collect();
-        __syncthreads();
+        collect(n_listed <= kTkGroupCap);
+        named_sync(kBarSel, kTkSelThreads);
         // ---- overflow: raise tau to the K-th largest buffered key and collect again
         for (int round = 0; s_over && round < kTkRounds; ++round) {
-            tau = block_kth_largest(s_cand, kTkCap, K, 7, 0, s_sel);
-            if (tid == 0) {
+            tau = sel_kth_largest(s_cand, kTkCap, K, 7, 0, s_sel, stid);
+            if (stid == 0) {
                 s_n = 0;
                 s_over = 0;
             }
-            __syncthreads();
-            collect();
-            __syncthreads();
+            named_sync(kBarSel, kTkSelThreads);
+            collect(false);
+            named_sync(kBarSel, kTkSelThreads);
         }
         const bool failed = s_over != 0;
         const int nc = min(s_n, kTkCap);
-        __syncthreads();
+        named_sync(kBarSel, kTkSelThreads);
         if (failed) {
-            if (tid == 0) {
+            if (stid == 0) {
                 set_status(a.status, TURNOPD_ERR_UNSUPPORTED);
                 a.token_loss[tok] = 0.f;
                 a.row_wl[j] = 0.0;
             }
-            continue;
-        }
-        // ---- the K largest: each candidate's rank among the candidates is its position
-        // (keys are unique); a large buffer is first cut to the K largest by radix select
-        const uint64_t kth = nc <= kTkThreads ? 0 : block_kth_largest(s_cand, nc, K, hi_val, 0, s_sel);
-        for (int i = tid; i < nc; i += kTkThreads) {
-            const uint64_t k = s_cand[i];
-            if (k < kth)
-                continue;
-            int rank = 0;
-            int i2 = 0;
-            for (; i2 + 4 <= nc; i2 += 4)
-                rank += (s_cand[i2] > k) + (s_cand[i2 + 1] > k) + (s_cand[i2 + 2] > k) + (s_cand[i2 + 3] > k);
-            for (; i2 < nc; ++i2)
-                rank += s_cand[i2] > k;
-            if (rank < K) {
-                s_top[rank] = k;
-                s_g[rank] = s_cz[i];
+        } else {
+            // ---- the K largest: each candidate's rank among the candidates is its position
+            // (keys are unique); a large buffer is first cut to the K largest by radix select
+            const uint64_t kth = nc <= kTkSelThreads ? 0 : sel_kth_largest(s_cand, nc, K, hi_val, 0, s_sel, stid);
+            for (int i = stid; i < nc; i += kTkSelThreads) {
+                const uint64_t k = s_cand[i];
+                if (k < kth)
+                    continue;
+                int rank = 0;
+                int i2 = 0;
+                for (; i2 + 4 <= nc; i2 += 4)
+                    rank += (s_cand[i2] > k) + (s_cand[i2 + 1] > k) + (s_cand[i2 + 2] > k) + (s_cand[i2 + 3] > k);
+                for (; i2 < nc; ++i2)
+                    rank += s_cand[i2] > k;
+                if (rank < K) {
+                    s_top[rank] = k;
+                    s_g[rank] = s_cz[i];
+                }
             }
-        }
-        __syncthreads();
+            named_sync(kBarSel, kTkSelThreads);
 
-        // ---- KL over S (one warp, fp32)
-        if (warp == 0) {
-            float m_s = -INFINITY, m_t = -INFINITY;
-            for (int r = lane; r < K; r += 32) {
-                const float zt_v = key_value<BF16>(s_top[r]);
-                const float zs_v = s_g[r];  // student logit, carried with the candidate
-                m_s = fmaxf(m_s, zs_v);
-                m_t = fmaxf(m_t, zt_v);
+            // ---- KL over S (one warp, fp32)
+            if (swarp == 0) {
+                float m_s = -INFINITY, m_t = -INFINITY;
+                for (int r = lane; r < K; r += 32) {
+                    const float zt_v = key_value<BF16>(s_top[r]);
+                    const float zs_v = s_g[r];  // student logit, carried with the candidate
+                    m_s = fmaxf(m_s, zs_v);
+                    m_t = fmaxf(m_t, zt_v);
+                }
+                m_s = warp_max_f(m_s);
+                m_t = warp_max_f(m_t);
+                float s_s = 0.f, s_t = 0.f, a_sd = 0.f;
+                for (int r = lane; r < K; r += 32) {
+                    const float zs_v = s_g[r], zt_v = key_value<BF16>(s_top[r]);
+                    const float es = expf(zs_v - m_s);
+                    s_s += es;
+                    s_t += expf(zt_v - m_t);
+                    a_sd = fmaf(es, zs_v - zt_v, a_sd);
+                }
+                s_s = warp_sum_f(s_s);
+                s_t = warp_sum_f(s_t);
+                a_sd = warp_sum_f(a_sd);
+                const float ep = a_sd / s_s;                              // E_p[z_s - z_t]
+                const float c = (m_s - m_t) + logf(s_s / s_t);            // LSE_s - LSE_t
+                const float ell = ep - c;
+                for (int r = lane; r < K; r += 32) {
+                    const float zs_v = s_g[r], zt_v = key_value<BF16>(s_top[r]);
+                    const float p = expf(zs_v - m_s) / s_s;
+                    const float g = w * p * ((zs_v - zt_v) - ep);
+                    s_g[r] = g;
+                    if (a.topk_ids)
+                        a.topk_ids[(size_t)tok * K + r] = (int32_t)key_id(s_top[r]);
+                    if (a.topk_grad)
+                        a.topk_grad[(size_t)tok * K + r] = g;
+                }
+                if (lane == 0) {
+                    if (!isfinite(ell))
+                        set_status(a.status, TURNOPD_ERR_NONFINITE);
+                    a.token_loss[tok] = ell;
+                    a.row_wl[j] = (double)w * (double)ell;
+                }
             }
-            m_s = warp_max_f(m_s);
-            m_t = warp_max_f(m_t);
-            float s_s = 0.f, s_t = 0.f, a_sd = 0.f;
-            for (int r = lane; r < K; r += 32) {
-                const float zs_v = s_g[r], zt_v = key_value<BF16>(s_top[r]);
-                const float es = expf(zs_v - m_s);
-                s_s += es;
-                s_t += expf(zt_v - m_t);
-                a_sd = fmaf(es, zs_v - zt_v, a_sd);
-            }
-            s_s = warp_sum_f(s_s);
-            s_t = warp_sum_f(s_t);
-            a_sd = warp_sum_f(a_sd);
-            const float ep = a_sd / s_s;                              // E_p[z_s - z_t]
-            const float c = (m_s - m_t) + logf(s_s / s_t);            // LSE_s - LSE_t
-            const float ell = ep - c;
-            for (int r = lane; r < K; r += 32) {
-                const float zs_v = s_g[r], zt_v = key_value<BF16>(s_top[r]);
-                const float p = expf(zs_v - m_s) / s_s;
-                const float g = w * p * ((zs_v - zt_v) - ep);
-                s_g[r] = g;
-                if (a.topk_ids)
-                    a.topk_ids[(size_t)tok * K + r] = (int32_t)key_id(s_top[r]);
-                if (a.topk_grad)
-                    a.topk_grad[(size_t)tok * K + r] = g;
-            }
-            if (lane == 0) {
-                if (!isfinite(ell))
-                    set_status(a.status, TURNOPD_ERR_NONFINITE);
-                a.token_loss[tok] = ell;
-                a.row_wl[j] = (double)w * (double)ell;
+            // ---- dense gradient row: zeros, then the K entries
+            if (a.grad) {
+                const size_t gesz = a.grad_dtype == TURNOPD_BF16 ? 2 : 4;
+                char *grow = static_cast<char *>(a.grad) + (size_t)m.y * (size_t)a.ld * gesz;
+                const int64_t bytes = a.vocab * (int64_t)gesz;
+                const bool g_ok = ((reinterpret_cast<uintptr_t>(grow)) & 15u) == 0;
+                const int64_t nv16 = g_ok ? bytes / 16 : 0;
+                for (int64_t q = stid; q < nv16; q += kTkSelThreads)
+                    reinterpret_cast<uint4 *>(grow)[q] = make_uint4(0, 0, 0, 0);
+                for (int64_t q = nv16 * 16 + stid; q < bytes; q += kTkSelThreads)
+                    grow[q] = 0;
+                named_sync(kBarSel, kTkSelThreads);
+                for (int r = stid; r < K; r += kTkSelThreads) {
+                    const uint32_t id = key_id(s_top[r]);
+                    if (a.grad_dtype == TURNOPD_BF16)
+                        reinterpret_cast<__nv_bfloat16 *>(grow)[id] = __float2bfloat16_rn(s_g[r]);
+                    else
+                        reinterpret_cast<float *>(grow)[id] = s_g[r];
+                }
             }
         }
-        // ---- dense gradient row: zeros, then the K entries
-        if (a.grad) {
-            const size_t gesz = a.grad_dtype == TURNOPD_BF16 ? 2 : 4;
-            char *grow = static_cast<char *>(a.grad) + (size_t)m.y * (size_t)a.ld * gesz;
-            const int64_t bytes = a.vocab * (int64_t)gesz;
-            const bool g_ok = ((reinterpret_cast<uintptr_t>(grow)) & 15u) == 0;
-            const int64_t nv16 = g_ok ? bytes / 16 : 0;
-            for (int64_t q = tid; q < nv16; q += kTkThreads)
-                reinterpret_cast<uint4 *>(grow)[q] = make_uint4(0, 0, 0, 0);
-            for (int64_t b = nv16 * 16 + tid; b < bytes; b += kTkThreads)
-                grow[b] = 0;
-            __syncthreads();
-            for (int r = tid; r < K; r += kTkThreads) {
-                const uint32_t id = key_id(s_top[r]);
-                if (a.grad_dtype == TURNOPD_BF16)
-                    reinterpret_cast<__nv_bfloat16 *>(grow)[id] = __float2bfloat16_rn(s_g[r]);
-                else
-                    reinterpret_cast<float *>(grow)[id] = s_g[r];
-            }
-        }
-        __syncthreads();
+        named_sync(kBarSel, kTkSelThreads);  // buffer b and the candidate arrays are free
+        if (it + 2 < n_it)
+            named_arrive(kBarFree + b, kTkThreads);
     }
 }
 
@@ -586,7 +686,7 @@ cudaError_t launch_topk(const TopkCall &c, cudaStream_t stream)
         return e;
     const int ti = c.in_dtype == TURNOPD_BF16 ? 0 : 1;
     auto kern = c.in_dtype == TURNOPD_BF16 ? k_topk_rows<true> : k_topk_rows<false>;
-    const size_t smem = topk_smem_bytes(c.vocab);
+    const size_t smem = topk_smem_bytes(c.vocab, c.K);
     static size_t attr_smem[64][2] = {};
     const int di = dev < 64 ? dev : 0;
     if (attr_smem[di][ti] < smem) {
