@@ -413,13 +413,17 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
                 } else {  // sampled token: g = w l (e_y - p)
                     const uint4 a = vs[q];
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
+                    for (int j = 0; j < 4; ++j)
                         g[j] = fmul2(ex2x2(ffma2(unpack2(word(a, j)), L2, NLW)), SGL);
-                        const int e = ((v0 + q) * 8 + 2 * j) - y;
-                        if (e == 0)
-                            g[j].x += wl;
-                        else if (e == -1)
-                            g[j].y += wl;
+                    if (v0 + q == (y >> 3)) {  // the vector holding y
+                        const int yi = y & 7;
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            if (yi == 2 * j)
+                                g[j].x += wl;
+                            if (yi == 2 * j + 1)
+                                g[j].y += wl;
+                        }
                     }
                 }
                 if (G32) {
