@@ -54,6 +54,10 @@ def parse():
     p.add_argument("--vocab-shards", type=int, default=0,
                    help="time the vocabulary-parallel path with this many column shards of one GPU's logits "
                         "standing in for ranks (stats, ordered merge, shard gradients)")
+    p.add_argument("--layout", default="compact", choices=["compact", "dense"],
+                   help="logit rows: one per supervised token, or one per token (row i = token i)")
+    p.add_argument("--zero-masked", action="store_true",
+                   help="dense layout with TURNOPD_ZERO_MASKED_GRAD: masked tokens' gradient rows written as zeros")
     p.add_argument("--alpha", type=float, default=0.5)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -149,6 +153,10 @@ class ClockSampler:
                 "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(self.rows)}
 
 
+def dense_layout(args):
+    return args.layout == "dense" or args.zero_masked
+
+
 def build_inputs(args, rank, device):
     import torch
 
@@ -160,20 +168,26 @@ def build_inputs(args, rank, device):
         b = W.packed(seed=rank, num_traj=args.num_traj or 8, traj_len=args.traj_len or 4096)
     else:
         b = W.CONFIGS[args.workload](seed=rank)
+    from paper_2607_05804_gb300 import TURNOPD_ZERO_MASKED_GRAD
+
     V = W.V_QWEN
-    R = b.num_valid
-    zs, zt = W.make_logits(R, V, "agent", torch.bfloat16, seed=1000 + rank, device=device)
+    dense = dense_layout(args)
+    rows = b.num_tokens if dense else b.num_valid
+    zs, zt = W.make_logits(rows, V, "agent", torch.bfloat16, seed=1000 + rank, device=device)
     mode = TURNOPD_SAMPLED_TOKEN if args.mode == "sampled" else TURNOPD_FULL_VOCAB
     y = None
     if mode == TURNOPD_SAMPLED_TOKEN:
         y_c = W.sample_ids(zs, seed=2000 + rank)  # per row; expand to per token
-        y = torch.zeros(b.num_tokens, dtype=torch.int32, device=device)
-        idx = torch.from_numpy(b.loss_mask.nonzero()[0]).to(device)
-        y[idx] = y_c
-    tid, msk, off, rot = to_device(b, device, compact=True)
+        if dense:
+            y = y_c
+        else:
+            y = torch.zeros(b.num_tokens, dtype=torch.int32, device=device)
+            idx = torch.from_numpy(b.loss_mask.nonzero()[0]).to(device)
+            y[idx] = y_c
+    tid, msk, off, rot = to_device(b, device, compact=not dense)
     k_top = args.k_top if args.mode == "topk" else 0
     step = LossStep(tid, msk, off, b.max_turns, V, row_of_token=rot, sampled_ids=y, mode=mode,
-                    alpha=args.alpha, k_top=k_top)
+                    alpha=args.alpha, k_top=k_top, flags=TURNOPD_ZERO_MASKED_GRAD if args.zero_masked else 0)
     # the top-K mode returns its gradient sparse: (ids, values) per token
     grad = None if k_top else torch.empty_like(zs)
     return b, V, zs, zt, grad, step
@@ -228,24 +242,29 @@ def run_step(step, zs, zt, grad, world, dist, ev_pair=None):
         dp.reduce_step(step.loss, step.turn_sum, step.turn_cnt, step.turn_surv)
 
 
-def cpu_baseline(b, zs, zt, V, alpha, mode, rows_override=0, budget_s=15.0, k_top=0):
+def cpu_baseline(b, zs, zt, V, alpha, mode, rows_override=0, budget_s=15.0, k_top=0, dense=False):
     """Time the fp64 CPU oracle on a bounded sample of the same workload: supervised
     rows in order, in chunks of 512 (so the oracle's fp64 gradient stays a few GB),
     until about `budget_s` seconds of oracle time or `rows_override` rows."""
     import numpy as np
+    import torch
 
     import oracle
     import workloads as W
 
     oracle.build()
-    R = zs.shape[0]
     w = oracle.weights(b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns, alpha).astype(np.float32)
     valid = np.nonzero(b.loss_mask)[0]
+    R = valid.size
     limit = min(R, rows_override) if rows_override else R
     done, spent, chunk = 0, 0.0, 512
     while done < limit and (rows_override or spent < budget_s):
         n = min(chunk, limit - done)
-        zsn, ztn = W.bf16_bits(zs[done:done + n]), W.bf16_bits(zt[done:done + n])
+        if dense:  # the supervised tokens' own rows
+            sel = torch.from_numpy(valid[done:done + n]).to(zs.device)
+            zsn, ztn = W.bf16_bits(zs.index_select(0, sel)), W.bf16_bits(zt.index_select(0, sel))
+        else:
+            zsn, ztn = W.bf16_bits(zs[done:done + n]), W.bf16_bits(zt[done:done + n])
         t0 = time.perf_counter()
         if k_top:
             oracle.topk_loss(zsn, ztn, V, np.ones(n, np.uint8), w[valid[done:done + n]], k_top)
@@ -441,8 +460,8 @@ def main():
     b, V, zs, zt, grad, step = build_inputs(args, rank, device)
     R = b.num_valid
     if args.vocab_shards:
-        if args.mode != "full":
-            raise SystemExit("--vocab-shards times the full-vocabulary mode")
+        if args.mode != "full" or dense_layout(args):
+            raise SystemExit("--vocab-shards times the full-vocabulary mode on compact rows")
         step.vp_call = vocab_parallel_loss_fn(step, zs, zt, grad, args.vocab_shards)
     torch.cuda.synchronize()
 
@@ -493,6 +512,10 @@ def main():
     else:
         bytes_per_row = 3 * V * 2  # two bf16 logit rows read + one bf16 gradient row written
     alg_bytes = R * bytes_per_row
+    masked_rows = b.num_tokens - R
+    if args.zero_masked:
+        # per masked token: a zero gradient row, or (top-K) K ids of -1 and K zero values
+        alg_bytes += masked_rows * (args.k_top * (4 + 4) if args.mode == "topk" else V * 2)
     loss_avg_ms = statistics.mean(loss_ms)
     achieved = alg_bytes / (loss_avg_ms / 1e3) / 1e9
 
@@ -503,7 +526,7 @@ def main():
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(b, zs, zt, V, args.alpha, 0, args.cpu_sample_rows,
-                           k_top=args.k_top if args.mode == "topk" else 0)
+                           k_top=args.k_top if args.mode == "topk" else 0, dense=dense_layout(args))
 
     if rank == 0:
         out = {
@@ -513,7 +536,9 @@ def main():
             "config": {
                 "workload": f"{b.name}_V{V}", "tokens": b.num_tokens, "supervised_tokens": R,
                 "tokens_counted": "supervised (assistant) tokens", "vocab": V,
-                "layout": "compact rows (one per supervised token)",
+                "layout": ("dense rows (row i = token i)" if dense_layout(args)
+                           else "compact rows (one per supervised token)"),
+                **({"zero_masked_grad": True, "masked_rows": masked_rows} if args.zero_masked else {}),
                 "grad_dtype": "fp32 sparse (ids, values)" if args.mode == "topk" else "bf16",
                 "mode": args.mode, "alpha": args.alpha, "scope": "traj",
                 **({"k_top": args.k_top} if args.mode == "topk" else {}),
@@ -531,10 +556,12 @@ def main():
                            "turnopd_loss_fwd_bwd launch sequence (row kernel + compaction + loss sum)"),
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "launch_ms": loss_avg_ms,
-                "traffic": None if (args.mode == "topk" or args.vocab_shards) else committed_traffic(args.workload),
+                "traffic": (None if (args.mode == "topk" or args.vocab_shards or dense_layout(args))
+                            else committed_traffic(args.workload)),
             },
             # vocabulary shards: counts(2) + weights(1) + per shard stats, gradient and loss sum + merge + stats(2)
-            "gpu_launches": (KERNELS_PER_STEP if not args.vocab_shards else 6 + 3 * args.vocab_shards) * args.steps,
+            "gpu_launches": ((KERNELS_PER_STEP + (1 if args.zero_masked else 0)) if not args.vocab_shards
+                             else 6 + 3 * args.vocab_shards) * args.steps,
             "clocks": clocks,
             "e2e": e2e,
             "cpu_baseline": cpu,

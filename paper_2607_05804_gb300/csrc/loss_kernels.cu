@@ -279,8 +279,18 @@ __global__ void k_zero_masked(const uint8_t *__restrict__ mask, const int32_t *_
         const int64_t r = rot ? (int64_t)rot[i] : i;
         if (r < 0 || r >= num_rows)
             continue;
+        // zeros are all-zero bits in both output types: 16-byte stores between an
+        // element-wise head (up to the first 16-byte boundary) and tail
         TOut *g = grad + r * ld;
-        for (int64_t v = threadIdx.x; v < vocab; v += blockDim.x)
+        const int64_t to16 = (int64_t)(((16u - (reinterpret_cast<uintptr_t>(g) & 15u)) & 15u) / sizeof(TOut));
+        const int64_t head = to16 < vocab ? to16 : vocab;
+        for (int64_t v = threadIdx.x; v < head; v += blockDim.x)
+            g[v] = from_float<TOut>(0.f);
+        uint4 *body = reinterpret_cast<uint4 *>(g + head);
+        const int64_t nvec = (vocab - head) * (int64_t)sizeof(TOut) / 16;
+        for (int64_t q = threadIdx.x; q < nvec; q += blockDim.x)
+            body[q] = make_uint4(0u, 0u, 0u, 0u);
+        for (int64_t v = head + nvec * (int64_t)(16 / sizeof(TOut)) + threadIdx.x; v < vocab; v += blockDim.x)
             g[v] = from_float<TOut>(0.f);
     }
 }
