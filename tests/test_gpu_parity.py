@@ -296,13 +296,16 @@ def test_random_structures_with_empty_trajectories(P, oracle):
         run_chain(P, oracle, b, 40, zs, zt, mode=k % 2, alpha=0.3 * (k % 4))
 
 
-def test_zero_masked_grad_and_untouched_rows(P, oracle):
+@pytest.mark.parametrize("ld,gdt", [(1024, torch.bfloat16), (1003, torch.bfloat16), (1001, torch.float32)])
+def test_zero_masked_grad_and_untouched_rows(P, oracle, ld, gdt):
+    """Masked rows are zeroed only with the flag; odd row strides put the row starts off
+    16-byte boundaries (the zero fill's element-wise head and tail)."""
     b = W.packed(seed=4, num_traj=2, traj_len=512)
     V = 1000
-    zs, zt = W.make_logits(b.num_tokens, V, "agent", torch.bfloat16, seed=4, device="cuda", ld=1024)
+    zs, zt = W.make_logits(b.num_tokens, V, "agent", torch.bfloat16, seed=4, device="cuda", ld=ld)
     for flags in (0, ZERO_MASKED):
         step = make_step(P, b, V, compact=False, flags=flags)
-        grad = torch.full(zs.shape, 3.0, dtype=torch.bfloat16, device="cuda")
+        grad = torch.full(zs.shape, 3.0, dtype=gdt, device="cuda")
         step.run(zs, zt, grad)
         torch.cuda.synchronize()
         masked = torch.from_numpy(b.loss_mask == 0).cuda()
