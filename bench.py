@@ -35,7 +35,9 @@ sys.path.insert(0, ROOT)
 
 METRIC = "loss fwd+bwd tokens/s at V=151936 bf16 on 1 GB300; achieved HBM GB/s vs peak"
 UNIT = "tokens/s"
-KERNELS_PER_STEP = 9  # counts(2) + weights(1) + compaction(2) + row kernel + loss sum + stats(2)
+# counts(2) + weights(1) + compaction(2) + row kernel + loss sum + stats(2); the full and
+# sampled modes add the helper grid that runs beside the cluster grid
+KERNELS_PER_STEP = 9
 ROW_KERNEL_SOURCES = ["paper_2607_05804_gb300/csrc/rowkl_cluster.cu",
                       "paper_2607_05804_gb300/csrc/loss_kernels.cu",
                       "paper_2607_05804_gb300/csrc/common.cuh"]
@@ -553,14 +555,16 @@ def main():
                            if args.mode == "topk" else
                            f"vocabulary-parallel path, {args.vocab_shards} shards of one GPU "
                            "(shard stats + merge + shard gradients)" if args.vocab_shards else
-                           "turnopd_loss_fwd_bwd launch sequence (row kernel + compaction + loss sum)"),
+                           "turnopd_loss_fwd_bwd launch sequence (cluster row kernel beside the helper grid "
+                           "+ compaction + loss sum)"),
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "launch_ms": loss_avg_ms,
                 "traffic": (None if (args.mode == "topk" or args.vocab_shards or dense_layout(args))
                             else committed_traffic(args.workload)),
             },
             # vocabulary shards: counts(2) + weights(1) + per shard stats, gradient and loss sum + merge + stats(2)
-            "gpu_launches": ((KERNELS_PER_STEP + (1 if args.zero_masked else 0)) if not args.vocab_shards
+            "gpu_launches": ((KERNELS_PER_STEP + (1 if args.zero_masked else 0) + (0 if args.mode == "topk" else 1))
+                             if not args.vocab_shards
                              else 6 + 3 * args.vocab_shards) * args.steps,
             "clocks": clocks,
             "e2e": e2e,

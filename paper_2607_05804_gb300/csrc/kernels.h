@@ -77,6 +77,9 @@ struct RowIn {
     const int4 *rows;
     const int32_t *nvalid;
     int32_t *status;
+    // split_den > 0: the cluster kernel takes rows [0, nvalid split_num / split_den) of the
+    // row list and the helper kernel the rest (set by launch_row_cluster)
+    int32_t split_num, split_den;
 };
 
 int device_sm_count();

@@ -382,7 +382,7 @@ cudaError_t launch_loss(const LossArgs &a, const LossWorkspace &ws, cudaStream_t
                                 stream);
 
     RowIn p{a.zs, a.zt, a.ld, a.vocab, a.row_of_token, a.sampled_ids, a.w, a.mode, a.grad,
-            a.token_loss, ws.row_wl, ws.rows, ws.nvalid, a.status};
+            a.token_loss, ws.row_wl, ws.rows, ws.nvalid, a.status, 0, 0};
     bool done = false;
     if (a.in_dtype == TURNOPD_BF16 && !(a.flags & TURNOPD_FORCE_PORTABLE)) {
         e = launch_row_cluster(p, a.grad_dtype == TURNOPD_F32, stream, &done);

@@ -24,6 +24,9 @@
 // Each thread reads its vectors of a row from shared memory twice: once into
 // registers for the maxima and sums, once for the gradient (3 exponentials
 // per element in all).
+// Clusters of 8 fill 120 of the 152 SMs; with a bf16 gradient (or none) a helper
+// grid of one 512-thread CTA per free SM takes the last share of the rows, each
+// row read from HBM once and again from L2 (k_row_helper below).
 // Waits are bounded: on timeout the kernel records TURNOPD_ERR_TIMEOUT, stops
 // computing and runs its remaining barriers without waiting, so it terminates.
 
@@ -167,8 +170,12 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
     }
     __syncthreads();
     cluster_sync();  // peers' barriers are initialised before any record is sent
+    // Every CTA of this grid is resident: a helper grid launched after this one may
+    // start now, on the SMs the clusters left free.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-    const int nvalid = *p.nvalid;
+    const int nv_all = *p.nvalid;
+    const int nvalid = p.split_den ? (int)((int64_t)nv_all * p.split_num / p.split_den) : nv_all;
     const int n = nvalid > cid ? (nvalid - cid + ncl - 1) / ncl : 0;  // same for the whole cluster
     if (n == 0)
         return;
@@ -487,6 +494,175 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
     cluster_sync();  // no CTA leaves while a peer may still address its shared memory
 }
 
+// Helper for the SMs the clusters leave free (15 eight-CTA clusters cover 120 of
+// 152): one CTA per row at a time, rows j0 + blockIdx.x, j0 + blockIdx.x +
+// gridDim.x, ... of the row list, j0 = the cluster kernel's share.  The
+// statistics pass streams both rows from HBM with a running maximum per thread
+// (one rescale per batch of kHelpU vectors when the maximum moves); the gradient
+// pass reads them again from L2, where the pass before left them (the clusters'
+// own copies are evict-first).  bf16 logits, bf16 gradient or none; like the
+// bf16 cluster path it keeps no reference difference.  Launched as a dependent
+// of the cluster grid (it starts once every cluster is resident) and completes
+// only after it, so stream order after it covers both grids.
+constexpr int kHelpThreads = 512;
+constexpr int kHelpU = 4;  // vectors of each model in flight per thread
+
+__device__ __forceinline__ uint32_t hmax4(const uint4 &v) { return hmax2u(hmax2u(v.x, v.y), hmax2u(v.z, v.w)); }
+
+__global__ void __launch_bounds__(kHelpThreads, 1) k_row_helper(RowIn p)
+{
+    constexpr int NW = kHelpThreads / 32;
+    constexpr uint32_t kFill = 0xff7fff7fu;  // lowest finite bf16 pair: adds 0, never the max
+    __shared__ float red[NW][8];
+    __shared__ float bc[8];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int nvalid = *p.nvalid;
+    const int j0 = p.split_den ? (int)((int64_t)nvalid * p.split_num / p.split_den) : 0;
+    const int nvec = (int)(p.vocab / 8);
+    const __nv_bfloat16 *zs = static_cast<const __nv_bfloat16 *>(p.zs);
+    const __nv_bfloat16 *zt = static_cast<const __nv_bfloat16 *>(p.zt);
+    const float2 L2 = splat(kLog2e);
+    for (int j = j0 + (int)blockIdx.x; j < nvalid; j += gridDim.x) {
+        const int4 m = p.rows[j];
+        const size_t off = (size_t)m.y * (size_t)p.ld;
+        const uint4 *vs = reinterpret_cast<const uint4 *>(zs + off);
+        const uint4 *vt = reinterpret_cast<const uint4 *>(zt + off);
+        float ms = -INFINITY, mt = -INFINITY;
+        float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
+        for (int q0 = tid; q0 < nvec; q0 += kHelpU * kHelpThreads) {
+            uint4 a[kHelpU], b[kHelpU];
+#pragma unroll
+            for (int u = 0; u < kHelpU; ++u) {
+                const int q = q0 + u * kHelpThreads;
+                if (q < nvec) {
+                    a[u] = __ldg(vs + q);
+                    b[u] = __ldg(vt + q);
+                } else {
+                    a[u] = b[u] = make_uint4(kFill, kFill, kFill, kFill);
+                }
+            }
+            uint32_t bs = hmax4(a[0]), bt = hmax4(b[0]);
+#pragma unroll
+            for (int u = 1; u < kHelpU; ++u) {
+                bs = hmax2u(bs, hmax4(a[u]));
+                bt = hmax2u(bt, hmax4(b[u]));
+            }
+            const float nms = fmaxf(ms, fmaxf(bf16lo(bs), bf16hi(bs)));
+            const float nmt = fmaxf(mt, fmaxf(bf16lo(bt), bf16hi(bt)));
+            if (nms > ms) {
+                const float2 f = splat(ex2((ms - nms) * kLog2e));
+                S2 = fmul2(S2, f);
+                A2 = fmul2(A2, f);
+                ms = nms;
+            }
+            if (nmt > mt) {
+                T2 = fmul2(T2, splat(ex2((mt - nmt) * kLog2e)));
+                mt = nmt;
+            }
+            const float2 NS = splat(-ms * kLog2e), NTT = splat(-mt * kLog2e);
+#pragma unroll
+            for (int u = 0; u < kHelpU; ++u)
+#pragma unroll
+                for (int w = 0; w < 4; ++w) {
+                    const float2 a2 = unpack2(word(a[u], w)), b2 = unpack2(word(b[u], w));
+                    const float2 es = ex2x2(ffma2(a2, L2, NS));
+                    S2 = fadd2(S2, es);
+                    A2 = ffma2(es, fsub2(a2, b2), A2);
+                    T2 = fadd2(T2, ex2x2(ffma2(b2, L2, NTT)));
+                }
+        }
+        Student S = Student{ms, S2.x + S2.y, A2.x + A2.y, 0.f};
+        Teacher U = Teacher{mt, T2.x + T2.y};
+        lane_merge<32, false>(S, U);
+        if (lane == 0) {
+            red[warp][0] = S.m, red[warp][1] = S.s, red[warp][2] = S.a;
+            red[warp][3] = U.m, red[warp][4] = U.s;
+        }
+        __syncthreads();
+        if (warp == 0) {
+            Student A = student_empty();
+            Teacher B = teacher_empty();
+            if (lane < NW) {
+                A = Student{red[lane][0], red[lane][1], red[lane][2], 0.f};
+                B = Teacher{red[lane][3], red[lane][4]};
+            }
+            lane_merge<NW, false>(A, B);
+            if (lane == 0) {
+                const RowConst rc = row_const(A, B);
+                const int y = m.z;  // in [0, V) or -1: the compaction drops other rows
+                const float e = y >= 0 ? (to_float(zs[off + y]) - to_float(zt[off + y])) - rc.dl : rc.kl;
+                const float wi = __int_as_float(m.w), wl = wi * e;
+                const float sg = wi < 0.f ? -1.f : 1.f;
+                if (!isfinite(rc.lse_s) || !isfinite(rc.lse_t) || !isfinite(e))
+                    set_status(p.status, TURNOPD_ERR_NONFINITE);
+                p.token_loss[m.x] = e;
+                p.row_wl[j] = (double)wi * (double)e;
+                // the gradient constants of the cluster kernel's bf16 path
+                bc[0] = -rc.lse_s * kLog2e + log2f(fabsf(y < 0 ? wi : wl));  // nlw
+                bc[1] = sg;
+                bc[2] = -sg * (rc.d + rc.cp);
+                bc[3] = wl > 0.f ? -1.f : 1.f;
+                bc[4] = wl;
+            }
+        }
+        __syncthreads();
+        if (p.grad) {
+            const float2 NLW = splat(bc[0]), SG = splat(bc[1]), NC = splat(bc[2]), SGL = splat(bc[3]);
+            const float wl = bc[4];
+            const int y = m.z;
+            uint4 *gr = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.grad) + off);
+            for (int q0 = tid; q0 < nvec; q0 += kHelpU * kHelpThreads) {
+                uint4 a[kHelpU], b[kHelpU];
+#pragma unroll
+                for (int u = 0; u < kHelpU; ++u) {
+                    const int q = q0 + u * kHelpThreads;
+                    if (q < nvec) {
+                        a[u] = __ldg(vs + q);
+                        if (y < 0)
+                            b[u] = __ldg(vt + q);
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < kHelpU; ++u) {
+                    const int q = q0 + u * kHelpThreads;
+                    if (q >= nvec)
+                        break;
+                    float2 g[4];
+                    if (y < 0) {  // full vocabulary: g = w p ((z_s - z_t) - d - cp)
+#pragma unroll
+                        for (int w = 0; w < 4; ++w) {
+                            const float2 a2 = unpack2(word(a[u], w)), b2 = unpack2(word(b[u], w));
+                            g[w] = fmul2(ex2x2(ffma2(a2, L2, NLW)), ffma2(fsub2(a2, b2), SG, NC));
+                        }
+                    } else {  // sampled token: g = w l (e_y - p)
+#pragma unroll
+                        for (int w = 0; w < 4; ++w)
+                            g[w] = fmul2(ex2x2(ffma2(unpack2(word(a[u], w)), L2, NLW)), SGL);
+                        if (q == (y >> 3)) {  // the vector holding y
+                            const int yi = y & 7;
+#pragma unroll
+                            for (int w = 0; w < 4; ++w) {
+                                if (yi == 2 * w)
+                                    g[w].x += wl;
+                                if (yi == 2 * w + 1)
+                                    g[w].y += wl;
+                            }
+                        }
+                    }
+                    uint4 o;
+                    o.x = pack_bf16x2(g[0].x, g[0].y);
+                    o.y = pack_bf16x2(g[1].x, g[1].y);
+                    o.z = pack_bf16x2(g[2].x, g[2].y);
+                    o.w = pack_bf16x2(g[3].x, g[3].y);
+                    __stcs(gr + q, o);
+                }
+            }
+        }
+        __syncthreads();  // red and bc are reused by the next row
+    }
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // complete only after the cluster grid
+}
+
 // Threads per row group and groups per CTA (tuning knobs).
 #ifndef TURNOPD_ROW_THREADS
 #define TURNOPD_ROW_THREADS 512
@@ -500,6 +676,10 @@ constexpr int kG = TURNOPD_ROW_GROUPS;
 constexpr int kMaxSlice = 2400;                      // vectors per CTA: 3 stages fit 227 KB
 constexpr int kVPT = (kMaxSlice + kNT - 1) / kNT;    // vectors per thread
 constexpr int64_t kMinVocab = 32768;  // below this the portable kernel is faster
+// The helper's rows per SM and second against the clusters' (packed 8 x 4096,
+// V = 151,936: the split that finishes both grids together was 0.86 of the rows
+// to 120 cluster SMs with 32 helper SMs).
+constexpr double kHelperRate = 0.61;
 
 size_t cluster_smem_bytes(int slice_vec)
 {
@@ -510,6 +690,9 @@ size_t cluster_smem_bytes(int slice_vec)
            kG * 16 * sizeof(float);                 // broadcast row constants
 }
 
+// The cluster grid (as many clusters as are co-resident, cached per device) and,
+// for a bf16 or no gradient, the helper grid on the SMs the clusters leave free,
+// with the row list split so that both finish together.
 template <bool G32>
 cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaStream_t stream)
 {
@@ -551,8 +734,28 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
             return cudaErrorInvalidConfiguration;
         grid_cache[dev][gi] = ncl;
     }
+    RowIn pl = p;
+    const int free_sm = device_sm_count() - grid_cache[dev][gi] * kCS;
+    if (!G32 && free_sm > 0) {
+        const double cl = (double)(grid_cache[dev][gi] * kCS);
+        pl.split_den = 1 << 20;
+        pl.split_num = (int32_t)(pl.split_den * cl / (cl + kHelperRate * free_sm) + 0.5);
+    }
     cfg.gridDim = dim3(grid_cache[dev][gi] * kCS);
-    return cudaLaunchKernelEx(&cfg, kern, p, slice_vec, nvec);
+    e = cudaLaunchKernelEx(&cfg, kern, pl, slice_vec, nvec);
+    if (e != cudaSuccess || pl.split_den == 0)
+        return e;
+    // the helper grid on the free SMs, a dependent of the cluster grid
+    cudaLaunchConfig_t hc = {};
+    cudaLaunchAttribute ha[1];
+    ha[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    ha[0].val.programmaticStreamSerializationAllowed = 1;
+    hc.attrs = ha;
+    hc.numAttrs = 1;
+    hc.gridDim = dim3(free_sm);
+    hc.blockDim = dim3(kHelpThreads);
+    hc.stream = stream;
+    return cudaLaunchKernelEx(&hc, k_row_helper, pl);
 }
 
 }  // namespace
