@@ -272,13 +272,16 @@ __global__ void k_turn_stats_index(const double *__restrict__ traj_turn_sum,
 
 // ---------------------------------------------------------------- launchers
 
+// One CTA per trajectory: 32 warps, so a 4096-token trajectory takes 4 load steps per warp.
+constexpr int kTrajThreads = 1024;
+
 cudaError_t launch_turn_counts(const int32_t *turn_id, const uint8_t *mask, const int64_t *off,
                                int32_t B, int64_t T, int32_t Tmax, int32_t *n_bt,
                                int64_t *counts, int32_t *status, cudaStream_t stream)
 {
     if (B > 0) {
-        k_traj_counts<<<B, 256, sizeof(int32_t) * Tmax, stream>>>(turn_id, mask, off, B, T, Tmax,
-                                                                   n_bt, status);
+        k_traj_counts<<<B, kTrajThreads, sizeof(int32_t) * Tmax, stream>>>(turn_id, mask, off, B, T, Tmax,
+                                                                            n_bt, status);
     }
     k_counts_reduce<<<1, 256, 0, stream>>>(n_bt, B, Tmax, counts);
     return cudaGetLastError();
@@ -290,8 +293,8 @@ cudaError_t launch_weights(const int32_t *turn_id, const uint8_t *mask, const in
                            float *w_out, int32_t *status, cudaStream_t stream)
 {
     if (B > 0)
-        k_weights<<<B, 256, 0, stream>>>(turn_id, mask, off, B, T, Tmax, alpha, scope, n_min, n_bt,
-                                         counts, w_out, status);
+        k_weights<<<B, kTrajThreads, 0, stream>>>(turn_id, mask, off, B, T, Tmax, alpha, scope, n_min, n_bt,
+                                                  counts, w_out, status);
     return cudaGetLastError();
 }
 
@@ -300,7 +303,7 @@ int turn_stats_warps(int32_t Tmax)
     // per-warp bins: Tmax * (8 + 4) bytes; keep the block under 160 KB
     const size_t per_warp = (size_t)Tmax * 12;
     int nw = (int)((160u * 1024u) / per_warp);
-    return nw > 8 ? 8 : nw;
+    return nw > kTrajThreads / 32 ? kTrajThreads / 32 : nw;
 }
 
 cudaError_t launch_turn_stats(const float *token_loss, const int32_t *turn_id,
