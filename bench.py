@@ -86,23 +86,31 @@ def load_peaks():
         return 6800.0, "fallback"
 
 
-def source_hash():
+TOPK_KERNEL_SOURCES = ["paper_2607_05804_gb300/csrc/topk_kernels.cu",
+                       "paper_2607_05804_gb300/csrc/common.cuh"]
+
+
+def source_hash(sources=None):
     h = hashlib.sha256()
-    for rel in ROW_KERNEL_SOURCES:
+    for rel in (ROW_KERNEL_SOURCES if sources is None else sources):
         with open(os.path.join(ROOT, rel), "rb") as fh:
             h.update(fh.read())
     return h.hexdigest()[:16]
 
 
-def committed_traffic(workload):
-    """DRAM bytes per row-kernel launch from the committed ncu summary, if it was
-    taken on the current kernel source."""
-    path = os.path.join(ROOT, "profiles", "row_kernel_traffic.json")
+def committed_traffic(workload, rows=None, kind="row"):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the
+    current kernel source: the row kernels' per-workload figure, or (kind "topk")
+    the top-K kernel's bytes per row times `rows`."""
+    name, sources = (("topk_traffic.json", TOPK_KERNEL_SOURCES) if kind == "topk"
+                     else ("row_kernel_traffic.json", ROW_KERNEL_SOURCES))
     try:
-        with open(path) as fh:
+        with open(os.path.join(ROOT, "profiles", name)) as fh:
             d = json.load(fh)
-        if d.get("source_hash") != source_hash():
+        if d.get("source_hash") != source_hash(sources):
             return None
+        if kind == "topk":
+            return d["bytes_per_row"] * rows
         return d.get("bytes_per_launch", {}).get(workload)
     except Exception:
         return None
@@ -559,7 +567,8 @@ def main():
                            "+ compaction + loss sum)"),
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "launch_ms": loss_avg_ms,
-                "traffic": (None if (args.mode == "topk" or args.vocab_shards or dense_layout(args))
+                "traffic": (None if (args.vocab_shards or dense_layout(args))
+                            else committed_traffic(args.workload, R, "topk") if args.mode == "topk"
                             else committed_traffic(args.workload)),
             },
             # vocabulary shards: counts(2) + weights(1) + per shard stats, gradient and loss sum + merge + stats(2)

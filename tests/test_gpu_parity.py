@@ -140,6 +140,27 @@ def test_cluster_kernel_all_rows(P, oracle, V, mode, gdt):
               grad_dtype=torch.bfloat16 if gdt == "bf16" else torch.float32)
 
 
+@pytest.mark.parametrize("V", [50000, W.V_QWEN])
+@pytest.mark.parametrize("mode", [0, 1], ids=["full", "sampled"])
+def test_forward_only_all_rows(P, oracle, V, mode):
+    """No gradient buffer: the loss and every token's l through both row grids (the
+    clusters' share of the rows and the helper grid's)."""
+    b = W.packed(seed=17, num_traj=2, traj_len=512)
+    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=17, device="cuda")
+    y = per_token_ids(b, W.sample_ids(zs, 3, V), True) if mode == 1 else None
+    step = make_step(P, b, V, compact=True, mode=mode, alpha=0.5, y=y)
+    step.run(zs, zt, None)
+    torch.cuda.synchronize()
+    assert step.status() == 0
+    T = b.num_tokens
+    w_ref = oracle.weights(b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns, 0.5)
+    _, tl_ref, loss_ref = oracle.loss_fwd_bwd(
+        bits_or_f32(zs), bits_or_f32(zt), V, b.loss_mask, w_ref.astype(np.float32), mode=mode,
+        row_of_token=b.compact_rows(), sampled_ids=y.cpu().numpy() if y is not None else None, grad=False)
+    assert_token_loss(step.token_loss[:T].cpu().numpy(), tl_ref, b.loss_mask)
+    assert_loss(step.loss.item(), loss_ref)
+
+
 def test_cluster_matches_portable(P, oracle):
     """Both kernels agree with each other to within the oracle tolerances."""
     b = W.packed(seed=13, num_traj=2, traj_len=512)
