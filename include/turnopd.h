@@ -451,6 +451,20 @@ turnopd_status turnopd_turn_stats(const float *token_loss, const int32_t *turn_i
  */
 double turnopd_alpha_schedule(int64_t k, int64_t K, double s, double e);
 
+/*
+ * turnopd_selftest_wait_timeout -- diagnostic of the device-side timeout path.
+ * Every wait of the library's kernels on an mbarrier or a flag is a bounded poll
+ * loop: when the limit runs out the kernel records TURNOPD_ERR_TIMEOUT in
+ * *dev_status, stops waiting and returns, so the context stays usable.  This
+ * entry launches one CTA that polls, in the same way, a barrier that nothing
+ * arrives on, so the path can be exercised without any failure of the GPU.
+ * poll_limit: polls before giving up, in [1, 2^24].
+ * dev_status: device int32 (caller-zeroed); receives TURNOPD_ERR_TIMEOUT.
+ * Errors: TURNOPD_ERR_NULL, TURNOPD_ERR_SHAPE (limit out of range), TURNOPD_ERR_CUDA.
+ */
+turnopd_status turnopd_selftest_wait_timeout(uint32_t poll_limit, int32_t *dev_status,
+                                             turnopd_stream_t stream);
+
 /* Human-readable name of a status code (static string, never NULL). */
 const char *turnopd_status_string(turnopd_status status);
 

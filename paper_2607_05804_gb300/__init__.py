@@ -22,6 +22,7 @@ __all__ = [
     "turnopd_turn_counts", "turnopd_weights", "turnopd_weights_workspace_bytes",
     "turnopd_loss_fwd_bwd", "turnopd_loss_workspace_bytes", "turnopd_turn_stats",
     "turnopd_alpha_schedule", "turnopd_status_string", "turnopd_loss_fwd_bwd_static",
+    "turnopd_selftest_wait_timeout",
     "TURNOPD_STATIC_MAX_TOKENS", "turnopd_fused_lmhead_fwd_bwd", "turnopd_fused_workspace_bytes",
     "turnopd_topk_loss_fwd_bwd", "TURNOPD_TOPK_MAX", "TURNOPD_TOPK_MAX_VOCAB",
     "turnopd_depth_params", "turnopd_depth_state", "turnopd_depth_default_params",
@@ -101,6 +102,7 @@ def load():
         "turnopd_turn_diagnostics": [P, P, P, i32, i32, P, P, P],
         "turnopd_vocab_shard_stats": [P, P, i32, i64, i64, i64, P, P, i64, P, P, P],
         "turnopd_vocab_stats_merge": [P, i32, P, i64, P, P],
+        "turnopd_selftest_wait_timeout": [u32, P, P],
         "turnopd_vocab_shard_loss_grad": [P, P, i32, i64, i64, i64, P, P, P, i64, P, P, i32, u32, P, P, P,
                                           sz, P, P],
     })
@@ -173,6 +175,16 @@ def _check(code, where):
 
 def turnopd_status_string(code: int) -> str:
     return load().turnopd_status_string(int(code)).decode()
+
+
+def turnopd_selftest_wait_timeout(poll_limit: int, dev_status, stream=None):
+    """One CTA polls a barrier that nothing arrives on; after poll_limit polls it
+    records TURNOPD_ERR_TIMEOUT in dev_status (device int32[1])."""
+    import torch
+
+    _need(dev_status, "dev_status", torch.int32, 1)
+    _check(load().turnopd_selftest_wait_timeout(int(poll_limit), _ptr(dev_status), _stream(stream)),
+           "turnopd_selftest_wait_timeout")
 
 
 def turnopd_alpha_schedule(k: int, K: int, s: float = 0.0, e: float = 1.0) -> float:

@@ -66,7 +66,7 @@ def build(force: bool = False, verbose: bool = False) -> str:
         with cf.ThreadPoolExecutor(max_workers=min(8, os.cpu_count() or 4)) as ex:
             objs = list(ex.map(compile_one, sources()))
         out = os.path.join(tmp, "libturnopd.so")
-        cmd = [nvcc, *ARCH, "-shared", "-cudart", "static", "-o", out, *objs]
+        cmd = [nvcc, *ARCH, "-shared", "-cudart", "static", "-o", out, *objs, "-ldl"]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"nvcc link failed:\n{r.stdout}\n{r.stderr}")

@@ -83,6 +83,7 @@ struct RowIn {
 };
 
 int device_sm_count();
+cudaError_t launch_wait_selftest(uint32_t limit, int32_t *status, cudaStream_t stream);
 
 // Pieces of the loss path reused by the fused LM-head path.
 cudaError_t launch_compaction(const LossArgs &a, int4 *rows, int32_t *blk_count, int32_t *nvalid,

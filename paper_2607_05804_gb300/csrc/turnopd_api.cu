@@ -5,6 +5,8 @@
 #include <cmath>
 #include <cstring>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "common.cuh"
 #include "kernels.h"
 
@@ -33,6 +35,15 @@ int device_sm_count()
 namespace {
 
 bool misaligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) != 0; }
+
+// An NVTX range around one entry point (shows the library's calls on a profiler
+// timeline; without a profiler attached it costs a function-pointer check).
+struct NvtxRange {
+    explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+    ~NvtxRange() { nvtxRangePop(); }
+    NvtxRange(const NvtxRange &) = delete;
+    NvtxRange &operator=(const NvtxRange &) = delete;
+};
 
 turnopd_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TURNOPD_OK : TURNOPD_ERR_CUDA; }
 
@@ -84,6 +95,15 @@ double turnopd_alpha_schedule(int64_t k, int64_t K, double s, double e)
     return a < 0.0 ? 0.0 : (a > 1.0 ? 1.0 : a);
 }
 
+turnopd_status turnopd_selftest_wait_timeout(uint32_t poll_limit, int32_t *dev_status, turnopd_stream_t stream)
+{
+    if (!dev_status)
+        return TURNOPD_ERR_NULL;
+    if (poll_limit < 1 || poll_limit > (1u << 24))
+        return TURNOPD_ERR_SHAPE;
+    return cuda_status(launch_wait_selftest(poll_limit, dev_status, (cudaStream_t)stream));
+}
+
 size_t turnopd_weights_workspace_bytes(int32_t num_traj, int32_t max_turns)
 {
     if (num_traj < 0 || max_turns < 1)
@@ -104,6 +124,7 @@ turnopd_status turnopd_turn_counts(const int32_t *turn_id, const uint8_t *loss_m
                                    int32_t *traj_turn_cnt, int64_t *counts,
                                    int32_t *dev_status, turnopd_stream_t stream)
 {
+    NvtxRange nvtx("turnopd_turn_counts");
     turnopd_status st = check_structure(turn_id, loss_mask, traj_offsets, num_traj, num_tokens,
                                         max_turns, dev_status);
     if (st != TURNOPD_OK)
@@ -122,6 +143,7 @@ turnopd_status turnopd_weights(const int32_t *turn_id, const uint8_t *loss_mask,
                                float *w_out, void *workspace, size_t workspace_bytes,
                                int32_t *dev_status, turnopd_stream_t stream)
 {
+    NvtxRange nvtx("turnopd_weights");
     turnopd_status st = check_structure(turn_id, loss_mask, traj_offsets, num_traj, num_tokens,
                                         max_turns, dev_status);
     if (st != TURNOPD_OK)
@@ -160,6 +182,7 @@ turnopd_status turnopd_loss_fwd_bwd(const void *z_student, const void *z_teacher
                                     void *workspace, size_t workspace_bytes,
                                     int32_t *dev_status, turnopd_stream_t stream)
 {
+    NvtxRange nvtx("turnopd_loss_fwd_bwd");
     if (!loss_out || !dev_status)
         return TURNOPD_ERR_NULL;
     if (num_tokens > 0 && (!z_student || !z_teacher || !loss_mask || !w || !token_loss_out))
@@ -203,6 +226,7 @@ turnopd_status turnopd_topk_loss_fwd_bwd(const void *z_student, const void *z_te
                                          double *loss_out, void *workspace, size_t workspace_bytes,
                                          int32_t *dev_status, turnopd_stream_t stream)
 {
+    NvtxRange nvtx("turnopd_topk_loss_fwd_bwd");
     if (!loss_out || !dev_status)
         return TURNOPD_ERR_NULL;
     if (num_tokens > 0 && (!z_student || !z_teacher || !loss_mask || !w || !token_loss_out))
@@ -276,6 +300,7 @@ turnopd_status turnopd_vocab_shard_stats(const void *z_student, const void *z_te
                                          const uint8_t *loss_mask, int64_t num_tokens, float *stats_out,
                                          int32_t *dev_status, turnopd_stream_t stream)
 {
+    NvtxRange nvtx("turnopd_vocab_shard_stats");
     turnopd_status st = vocab_common_checks(z_student, z_teacher, in_dtype, ld, shard_vocab, num_rows, row_of_token,
                                             loss_mask, num_tokens, dev_status);
     if (st != TURNOPD_OK)
@@ -294,6 +319,7 @@ turnopd_status turnopd_vocab_shard_stats(const void *z_student, const void *z_te
 turnopd_status turnopd_vocab_stats_merge(const float *parts, int32_t n_shards, const uint8_t *loss_mask,
                                          int64_t num_tokens, float *merged_out, turnopd_stream_t stream)
 {
+    NvtxRange nvtx("turnopd_vocab_stats_merge");
     if (num_tokens > 0 && (!parts || !loss_mask || !merged_out))
         return TURNOPD_ERR_NULL;
     if (n_shards < 1 || num_tokens < 0 || num_tokens > INT32_MAX)
@@ -314,6 +340,7 @@ turnopd_status turnopd_vocab_shard_loss_grad(const void *z_student, const void *
                                              double *loss_out, void *workspace, size_t workspace_bytes,
                                              int32_t *dev_status, turnopd_stream_t stream)
 {
+    NvtxRange nvtx("turnopd_vocab_shard_loss_grad");
     turnopd_status st = vocab_common_checks(z_student, z_teacher, in_dtype, ld, shard_vocab, num_rows, row_of_token,
                                             loss_mask, num_tokens, dev_status);
     if (st != TURNOPD_OK)
@@ -353,6 +380,7 @@ turnopd_status turnopd_fused_lmhead_fwd_bwd(const void *h_s, const void *W_s, in
                                             size_t workspace_bytes, int32_t *dev_status,
                                             turnopd_stream_t stream)
 {
+    NvtxRange nvtx("turnopd_fused_lmhead_fwd_bwd");
     if (!loss_out || !dev_status || !W_s || !W_t)
         return TURNOPD_ERR_NULL;
     if (num_tokens > 0 && (!h_s || !h_t || !loss_mask || !w || !token_loss_out))
@@ -390,6 +418,7 @@ turnopd_status turnopd_turn_stats(const float *token_loss, const int32_t *turn_i
                                   double *turn_sum, int64_t *turn_cnt, int32_t *turn_surv,
                                   int32_t *dev_status, turnopd_stream_t stream)
 {
+    NvtxRange nvtx("turnopd_turn_stats");
     turnopd_status st = check_structure(turn_id, loss_mask, traj_offsets, num_traj, num_tokens,
                                         max_turns, dev_status);
     if (st != TURNOPD_OK)

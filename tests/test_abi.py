@@ -143,3 +143,10 @@ def test_topk_host_validation(lib):
     assert call(flags=0x100) == 6                     # only TURNOPD_ZERO_MASKED_GRAD
     assert call(ws=None) == 10
     assert call(wsb=ws_need - 1) == 10
+
+
+def test_selftest_wait_timeout_host_validation(lib):
+    f = lib.turnopd_selftest_wait_timeout
+    assert f(100, None, None) == 1                # TURNOPD_ERR_NULL
+    assert f(0, FAKE, None) == 2                  # TURNOPD_ERR_SHAPE: no polls
+    assert f((1 << 24) + 1, FAKE, None) == 2      # TURNOPD_ERR_SHAPE: beyond the cap
