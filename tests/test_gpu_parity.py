@@ -161,6 +161,23 @@ def test_forward_only_all_rows(P, oracle, V, mode):
     assert_loss(step.loss.item(), loss_ref)
 
 
+@pytest.mark.parametrize("n_sup", [1, 2, 3, 7])
+@pytest.mark.parametrize("mode", [0, 1], ids=["full", "sampled"])
+def test_few_rows_split_between_grids(P, oracle, n_sup, mode):
+    """A handful of supervised rows at the full vocabulary: the row list's cut leaves
+    the cluster grid none or a few of them and the helper grid the rest."""
+    T = 40
+    turn_id = np.full(T, -1, np.int32)
+    mask = np.zeros(T, np.uint8)
+    idx = np.linspace(3, T - 2, n_sup).astype(int)
+    mask[idx] = 1
+    turn_id[idx] = np.arange(n_sup) % 3
+    b = W.Batch("few", turn_id, mask, np.array([0, T], np.int64), 3)
+    V = FULL_V
+    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=40 + n_sup, device="cuda")
+    run_chain(P, oracle, b, V, zs, zt, mode=mode, alpha=0.5, compact=True)
+
+
 def test_cluster_matches_portable(P, oracle):
     """Both kernels agree with each other to within the oracle tolerances."""
     b = W.packed(seed=13, num_traj=2, traj_len=512)
