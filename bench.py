@@ -60,6 +60,7 @@ def parse():
                    help="logit rows: one per supervised token, or one per token (row i = token i)")
     p.add_argument("--zero-masked", action="store_true",
                    help="dense layout with TURNOPD_ZERO_MASKED_GRAD: masked tokens' gradient rows written as zeros")
+    p.add_argument("--fp32-grad", action="store_true", help="full/sampled modes: an fp32 gradient instead of bf16")
     p.add_argument("--alpha", type=float, default=0.5)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -199,7 +200,8 @@ def build_inputs(args, rank, device):
     step = LossStep(tid, msk, off, b.max_turns, V, row_of_token=rot, sampled_ids=y, mode=mode,
                     alpha=args.alpha, k_top=k_top, flags=TURNOPD_ZERO_MASKED_GRAD if args.zero_masked else 0)
     # the top-K mode returns its gradient sparse: (ids, values) per token
-    grad = None if k_top else torch.empty_like(zs)
+    grad = None if k_top else torch.empty(zs.shape, dtype=torch.float32 if args.fp32_grad else zs.dtype,
+                                          device=zs.device)
     return b, V, zs, zt, grad, step
 
 
@@ -520,7 +522,8 @@ def main():
         # statistics pass (two logit rows read), gradient pass (read again, gradient written)
         bytes_per_row = 5 * V * 2
     else:
-        bytes_per_row = 3 * V * 2  # two bf16 logit rows read + one bf16 gradient row written
+        # two bf16 logit rows read + one gradient row written (bf16, or fp32)
+        bytes_per_row = 2 * V * 2 + V * (4 if args.fp32_grad else 2)
     alg_bytes = R * bytes_per_row
     masked_rows = b.num_tokens - R
     if args.zero_masked:
@@ -549,7 +552,8 @@ def main():
                 "layout": ("dense rows (row i = token i)" if dense_layout(args)
                            else "compact rows (one per supervised token)"),
                 **({"zero_masked_grad": True, "masked_rows": masked_rows} if args.zero_masked else {}),
-                "grad_dtype": "fp32 sparse (ids, values)" if args.mode == "topk" else "bf16",
+                "grad_dtype": ("fp32 sparse (ids, values)" if args.mode == "topk"
+                               else "fp32" if args.fp32_grad else "bf16"),
                 "mode": args.mode, "alpha": args.alpha, "scope": "traj",
                 **({"k_top": args.k_top} if args.mode == "topk" else {}),
                 **({"vocab_shards": args.vocab_shards} if args.vocab_shards else {}),

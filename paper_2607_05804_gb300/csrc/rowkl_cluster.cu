@@ -24,9 +24,9 @@
 // Each thread reads its vectors of a row from shared memory twice: once into
 // registers for the maxima and sums, once for the gradient (3 exponentials
 // per element in all).
-// Clusters of 8 fill 120 of the 152 SMs; with a bf16 gradient (or none) a helper
-// grid of one 512-thread CTA per free SM takes the last share of the rows, each
-// row read from HBM once and again from L2 (k_row_helper below).
+// Clusters of 8 fill 120 of the 152 SMs; a helper grid of one 512-thread CTA per
+// free SM takes the last share of the rows, each row read from HBM once and again
+// from L2 (k_row_helper below).
 // Waits are bounded: on timeout the kernel records TURNOPD_ERR_TIMEOUT, stops
 // computing and runs its remaining barriers without waiting, so it terminates.
 
@@ -500,8 +500,10 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
 // statistics pass streams both rows from HBM with a running maximum per thread
 // (one rescale per batch of kHelpU vectors when the maximum moves); the gradient
 // pass reads them again from L2, where the pass before left them (the clusters'
-// own copies are evict-first).  bf16 logits, bf16 gradient or none; like the
-// bf16 cluster path it keeps no reference difference.  Launched as a dependent
+// own copies are evict-first).  bf16 logits; a bf16 or fp32 gradient or none.
+// Like the cluster kernel, the fp32 gradient also keeps A relative to the
+// reference difference d at the thread's running student argmax (re-referenced,
+// A <- (A + S (d - d')) f, when the maximum moves).  Launched as a dependent
 // of the cluster grid (it starts once every cluster is resident) and completes
 // only after it, so stream order after it covers both grids.
 constexpr int kHelpThreads = 512;
@@ -509,6 +511,7 @@ constexpr int kHelpU = 4;  // vectors of each model in flight per thread
 
 __device__ __forceinline__ uint32_t hmax4(const uint4 &v) { return hmax2u(hmax2u(v.x, v.y), hmax2u(v.z, v.w)); }
 
+template <bool G32>
 __global__ void __launch_bounds__(kHelpThreads, 1) k_row_helper(RowIn p)
 {
     constexpr int NW = kHelpThreads / 32;
@@ -527,7 +530,7 @@ __global__ void __launch_bounds__(kHelpThreads, 1) k_row_helper(RowIn p)
         const size_t off = (size_t)m.y * (size_t)p.ld;
         const uint4 *vs = reinterpret_cast<const uint4 *>(zs + off);
         const uint4 *vt = reinterpret_cast<const uint4 *>(zt + off);
-        float ms = -INFINITY, mt = -INFINITY;
+        float ms = -INFINITY, mt = -INFINITY, dd = 0.f;  // dd: reference difference (fp32 gradient)
         float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
         for (int q0 = tid; q0 < nvec; q0 += kHelpU * kHelpThreads) {
             uint4 a[kHelpU], b[kHelpU];
@@ -551,15 +554,36 @@ __global__ void __launch_bounds__(kHelpThreads, 1) k_row_helper(RowIn p)
             const float nmt = fmaxf(mt, fmaxf(bf16lo(bt), bf16hi(bt)));
             if (nms > ms) {
                 const float2 f = splat(ex2((ms - nms) * kLog2e));
+                if (G32) {  // d at the first element of the batch equal to the new maximum
+                    float xd = 0.f;
+                    bool found = false;
+#pragma unroll
+                    for (int u = 0; u < kHelpU; ++u)
+#pragma unroll
+                        for (int w = 0; w < 4; ++w) {
+                            const float2 x = unpack2(word(a[u], w)), y = unpack2(word(b[u], w));
+                            if (!found && x.x == nms) {
+                                xd = x.x - y.x;
+                                found = true;
+                            }
+                            if (!found && x.y == nms) {
+                                xd = x.y - y.y;
+                                found = true;
+                            }
+                        }
+                    A2 = fmul2(ffma2(S2, splat(dd - xd), A2), f);
+                    dd = xd;
+                } else {
+                    A2 = fmul2(A2, f);
+                }
                 S2 = fmul2(S2, f);
-                A2 = fmul2(A2, f);
                 ms = nms;
             }
             if (nmt > mt) {
                 T2 = fmul2(T2, splat(ex2((mt - nmt) * kLog2e)));
                 mt = nmt;
             }
-            const float2 NS = splat(-ms * kLog2e), NTT = splat(-mt * kLog2e);
+            const float2 NS = splat(-ms * kLog2e), NTT = splat(-mt * kLog2e), D = splat(dd);
 #pragma unroll
             for (int u = 0; u < kHelpU; ++u)
 #pragma unroll
@@ -567,26 +591,26 @@ __global__ void __launch_bounds__(kHelpThreads, 1) k_row_helper(RowIn p)
                     const float2 a2 = unpack2(word(a[u], w)), b2 = unpack2(word(b[u], w));
                     const float2 es = ex2x2(ffma2(a2, L2, NS));
                     S2 = fadd2(S2, es);
-                    A2 = ffma2(es, fsub2(a2, b2), A2);
+                    A2 = ffma2(es, G32 ? fsub2(fsub2(a2, b2), D) : fsub2(a2, b2), A2);
                     T2 = fadd2(T2, ex2x2(ffma2(b2, L2, NTT)));
                 }
         }
-        Student S = Student{ms, S2.x + S2.y, A2.x + A2.y, 0.f};
+        Student S = Student{ms, S2.x + S2.y, A2.x + A2.y, dd};
         Teacher U = Teacher{mt, T2.x + T2.y};
-        lane_merge<32, false>(S, U);
+        lane_merge<32, G32>(S, U);
         if (lane == 0) {
             red[warp][0] = S.m, red[warp][1] = S.s, red[warp][2] = S.a;
-            red[warp][3] = U.m, red[warp][4] = U.s;
+            red[warp][3] = U.m, red[warp][4] = U.s, red[warp][5] = S.d;
         }
         __syncthreads();
         if (warp == 0) {
             Student A = student_empty();
             Teacher B = teacher_empty();
             if (lane < NW) {
-                A = Student{red[lane][0], red[lane][1], red[lane][2], 0.f};
+                A = Student{red[lane][0], red[lane][1], red[lane][2], red[lane][5]};
                 B = Teacher{red[lane][3], red[lane][4]};
             }
-            lane_merge<NW, false>(A, B);
+            lane_merge<NW, G32>(A, B);
             if (lane == 0) {
                 const RowConst rc = row_const(A, B);
                 const int y = m.z;  // in [0, V) or -1: the compaction drops other rows
@@ -597,20 +621,22 @@ __global__ void __launch_bounds__(kHelpThreads, 1) k_row_helper(RowIn p)
                     set_status(p.status, TURNOPD_ERR_NONFINITE);
                 p.token_loss[m.x] = e;
                 p.row_wl[j] = (double)wi * (double)e;
-                // the gradient constants of the cluster kernel's bf16 path
+                // the gradient constants of the cluster kernel
                 bc[0] = -rc.lse_s * kLog2e + log2f(fabsf(y < 0 ? wi : wl));  // nlw
                 bc[1] = sg;
-                bc[2] = -sg * (rc.d + rc.cp);
+                bc[2] = -sg * (rc.d + rc.cp);  // bf16 output: one rounding of d + cp
                 bc[3] = wl > 0.f ? -1.f : 1.f;
                 bc[4] = wl;
+                bc[5] = -sg * rc.d;            // fp32 output
+                bc[6] = -sg * rc.cp;
             }
         }
         __syncthreads();
         if (p.grad) {
             const float2 NLW = splat(bc[0]), SG = splat(bc[1]), NC = splat(bc[2]), SGL = splat(bc[3]);
+            const float2 ND = splat(bc[5]), NCP = splat(bc[6]);
             const float wl = bc[4];
             const int y = m.z;
-            uint4 *gr = reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.grad) + off);
             for (int q0 = tid; q0 < nvec; q0 += kHelpU * kHelpThreads) {
                 uint4 a[kHelpU], b[kHelpU];
 #pragma unroll
@@ -632,7 +658,8 @@ __global__ void __launch_bounds__(kHelpThreads, 1) k_row_helper(RowIn p)
 #pragma unroll
                         for (int w = 0; w < 4; ++w) {
                             const float2 a2 = unpack2(word(a[u], w)), b2 = unpack2(word(b[u], w));
-                            g[w] = fmul2(ex2x2(ffma2(a2, L2, NLW)), ffma2(fsub2(a2, b2), SG, NC));
+                            const float2 pw = ex2x2(ffma2(a2, L2, NLW)), x = fsub2(a2, b2);
+                            g[w] = G32 ? fmul2(pw, fadd2(ffma2(x, SG, ND), NCP)) : fmul2(pw, ffma2(x, SG, NC));
                         }
                     } else {  // sampled token: g = w l (e_y - p)
 #pragma unroll
@@ -649,12 +676,18 @@ __global__ void __launch_bounds__(kHelpThreads, 1) k_row_helper(RowIn p)
                             }
                         }
                     }
-                    uint4 o;
-                    o.x = pack_bf16x2(g[0].x, g[0].y);
-                    o.y = pack_bf16x2(g[1].x, g[1].y);
-                    o.z = pack_bf16x2(g[2].x, g[2].y);
-                    o.w = pack_bf16x2(g[3].x, g[3].y);
-                    __stcs(gr + q, o);
+                    if (G32) {
+                        float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(p.grad) + off) + 2 * (size_t)q;
+                        __stcs(dst, make_float4(g[0].x, g[0].y, g[1].x, g[1].y));
+                        __stcs(dst + 1, make_float4(g[2].x, g[2].y, g[3].x, g[3].y));
+                    } else {
+                        uint4 o;
+                        o.x = pack_bf16x2(g[0].x, g[0].y);
+                        o.y = pack_bf16x2(g[1].x, g[1].y);
+                        o.z = pack_bf16x2(g[2].x, g[2].y);
+                        o.w = pack_bf16x2(g[3].x, g[3].y);
+                        __stcs(reinterpret_cast<uint4 *>(static_cast<__nv_bfloat16 *>(p.grad) + off) + q, o);
+                    }
                 }
             }
         }
@@ -690,9 +723,9 @@ size_t cluster_smem_bytes(int slice_vec)
            kG * 16 * sizeof(float);                 // broadcast row constants
 }
 
-// The cluster grid (as many clusters as are co-resident, cached per device) and,
-// for a bf16 or no gradient, the helper grid on the SMs the clusters leave free,
-// with the row list split so that both finish together.
+// The cluster grid (as many clusters as are co-resident, cached per device) and
+// the helper grid on the SMs the clusters leave free, with the row list split so
+// that both finish together.
 template <bool G32>
 cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaStream_t stream)
 {
@@ -736,7 +769,7 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
     }
     RowIn pl = p;
     const int free_sm = device_sm_count() - grid_cache[dev][gi] * kCS;
-    if (!G32 && free_sm > 0) {
+    if (free_sm > 0) {
         const double cl = (double)(grid_cache[dev][gi] * kCS);
         pl.split_den = 1 << 20;
         pl.split_num = (int32_t)(pl.split_den * cl / (cl + kHelperRate * free_sm) + 0.5);
@@ -755,7 +788,7 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
     hc.gridDim = dim3(free_sm);
     hc.blockDim = dim3(kHelpThreads);
     hc.stream = stream;
-    return cudaLaunchKernelEx(&hc, k_row_helper, pl);
+    return cudaLaunchKernelEx(&hc, k_row_helper<G32>, pl);
 }
 
 }  // namespace
