@@ -34,6 +34,7 @@
 
 #include "common.cuh"
 #include "kernels.h"
+#include "packed.cuh"
 #include "ptx.cuh"
 
 namespace turnopd {
@@ -42,33 +43,6 @@ namespace {
 constexpr int kStages = 3;
 constexpr uint32_t kCopyChunk = 65536;       // bytes per bulk copy instruction
 constexpr uint32_t kWaitLimit = 1u << 22;    // mbarrier polls before giving up
-
-// ---- packed f32x2 arithmetic (two fp32 lanes per instruction) -----------
-// The sm_100-family paired-fp32 builtins; subtraction as an exact fma by -1.
-
-__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) { return __ffma2_rn(a, b, c); }
-__device__ __forceinline__ float2 fadd2(float2 a, float2 b) { return __fadd2_rn(a, b); }
-__device__ __forceinline__ float2 fmul2(float2 a, float2 b) { return __fmul2_rn(a, b); }
-__device__ __forceinline__ float2 fsub2(float2 a, float2 b)
-{
-    return __ffma2_rn(b, make_float2(-1.f, -1.f), a);
-}
-
-__device__ __forceinline__ float2 unpack2(uint32_t u) { return make_float2(bf16lo(u), bf16hi(u)); }
-__device__ __forceinline__ float2 splat(float x) { return make_float2(x, x); }
-__device__ __forceinline__ float2 ex2x2(float2 x) { return make_float2(ex2(x.x), ex2(x.y)); }
-
-__device__ __forceinline__ uint32_t hmax2u(uint32_t a, uint32_t b)
-{
-    uint32_t d;
-    asm("max.bf16x2 %0, %1, %2;" : "=r"(d) : "r"(a), "r"(b));
-    return d;
-}
-
-__device__ __forceinline__ uint32_t word(const uint4 &v, int j)
-{
-    return j == 0 ? v.x : (j == 1 ? v.y : (j == 2 ? v.z : v.w));
-}
 
 // Merge per-lane partial statistics across the first `width` lanes of a warp
 // (lanes beyond hold empty partials): exact max by butterfly, one rescale
@@ -508,8 +482,6 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
 // only after it, so stream order after it covers both grids.
 constexpr int kHelpThreads = 512;
 constexpr int kHelpU = 4;  // vectors of each model in flight per thread
-
-__device__ __forceinline__ uint32_t hmax4(const uint4 &v) { return hmax2u(hmax2u(v.x, v.y), hmax2u(v.z, v.w)); }
 
 template <bool G32>
 __global__ void __launch_bounds__(kHelpThreads, 1) k_row_helper(RowIn p)

@@ -16,7 +16,10 @@
 #include <algorithm>
 
 #include "common.cuh"
+#include <type_traits>
+
 #include "kernels.h"
+#include "packed.cuh"
 #include "row_math.cuh"
 
 namespace turnopd {
@@ -24,6 +27,7 @@ namespace {
 
 constexpr int kVpThreads = 256;
 constexpr int kStatWords = 6;  // m_s, S_s, A, d, m_t, S_t
+constexpr int kVpU = 4;        // bf16 rows: vectors of each model in flight per thread
 
 struct ShardIn {
     const void *zs, *zt;
@@ -51,6 +55,80 @@ __device__ __forceinline__ void fold_row(const TIn *rs, const TIn *rt, int64_t V
         float a = to_float(rs[v]), b = to_float(rt[v]);
         accumulate<1>(s, t, &a, &b);
     }
+}
+
+// The same statistics for an aligned bf16 row in 16-byte vectors, kVpU vectors of
+// each model in flight per thread: a running maximum rescaled once per batch when it
+// moves, A kept relative to d at the thread's running student argmax (re-referenced,
+// A <- (A + S (d - d')) f, with the maximum), packed f32x2 sums.
+__device__ __forceinline__ void fold_row_bf16(const uint4 *vs, const uint4 *vt, int64_t nvec, Student &s,
+                                              Teacher &t)
+{
+    constexpr uint32_t kFill = 0xff7fff7fu;  // lowest finite bf16 pair: adds 0, never the max
+    const float2 L2 = splat(kLog2e);
+    float ms = -INFINITY, mt = -INFINITY, dd = 0.f;
+    float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
+    for (int64_t q0 = threadIdx.x; q0 < nvec; q0 += kVpU * kVpThreads) {
+        uint4 a[kVpU], b[kVpU];
+#pragma unroll
+        for (int u = 0; u < kVpU; ++u) {
+            const int64_t q = q0 + u * kVpThreads;
+            if (q < nvec) {
+                a[u] = __ldg(vs + q);
+                b[u] = __ldg(vt + q);
+            } else {
+                a[u] = b[u] = make_uint4(kFill, kFill, kFill, kFill);
+            }
+        }
+        uint32_t bs = hmax4(a[0]), bt = hmax4(b[0]);
+#pragma unroll
+        for (int u = 1; u < kVpU; ++u) {
+            bs = hmax2u(bs, hmax4(a[u]));
+            bt = hmax2u(bt, hmax4(b[u]));
+        }
+        const float nms = fmaxf(ms, fmaxf(bf16lo(bs), bf16hi(bs)));
+        const float nmt = fmaxf(mt, fmaxf(bf16lo(bt), bf16hi(bt)));
+        if (nms > ms) {
+            float xd = 0.f;  // d at the first element of the batch equal to the new maximum
+            bool found = false;
+#pragma unroll
+            for (int u = 0; u < kVpU; ++u)
+#pragma unroll
+                for (int w = 0; w < 4; ++w) {
+                    const float2 x = unpack2(word(a[u], w)), y = unpack2(word(b[u], w));
+                    if (!found && x.x == nms) {
+                        xd = x.x - y.x;
+                        found = true;
+                    }
+                    if (!found && x.y == nms) {
+                        xd = x.y - y.y;
+                        found = true;
+                    }
+                }
+            const float2 f = splat(ex2((ms - nms) * kLog2e));
+            A2 = fmul2(ffma2(S2, splat(dd - xd), A2), f);
+            S2 = fmul2(S2, f);
+            dd = xd;
+            ms = nms;
+        }
+        if (nmt > mt) {
+            T2 = fmul2(T2, splat(ex2((mt - nmt) * kLog2e)));
+            mt = nmt;
+        }
+        const float2 NS = splat(-ms * kLog2e), NTT = splat(-mt * kLog2e), D = splat(dd);
+#pragma unroll
+        for (int u = 0; u < kVpU; ++u)
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+                const float2 a2 = unpack2(word(a[u], w)), b2 = unpack2(word(b[u], w));
+                const float2 es = ex2x2(ffma2(a2, L2, NS));
+                S2 = fadd2(S2, es);
+                A2 = ffma2(es, fsub2(fsub2(a2, b2), D), A2);
+                T2 = fadd2(T2, ex2x2(ffma2(b2, L2, NTT)));
+            }
+    }
+    s = ms == -INFINITY ? student_empty() : Student{ms, S2.x + S2.y, A2.x + A2.y, dd};
+    t = mt == -INFINITY ? teacher_empty() : Teacher{mt, T2.x + T2.y};
 }
 
 // Block reduction of the per-thread accumulators (result in thread 0).
@@ -101,7 +179,17 @@ __global__ void __launch_bounds__(kVpThreads) k_shard_stats(ShardIn p, float *__
             continue;
         Student s = student_empty();
         Teacher t = teacher_empty();
-        fold_row<TIn, VEC>(zs + r * p.ld, zt + r * p.ld, p.vocab, s, t);
+        if constexpr (VEC && std::is_same<TIn, __nv_bfloat16>::value) {
+            const int64_t nvec = p.vocab / 8;
+            fold_row_bf16(reinterpret_cast<const uint4 *>(zs + r * p.ld), reinterpret_cast<const uint4 *>(zt + r * p.ld),
+                          nvec, s, t);
+            for (int64_t v = nvec * 8 + threadIdx.x; v < p.vocab; v += kVpThreads) {  // ragged tail
+                float a = to_float(zs[r * p.ld + v]), b = to_float(zt[r * p.ld + v]);
+                accumulate<1>(s, t, &a, &b);
+            }
+        } else {
+            fold_row<TIn, VEC>(zs + r * p.ld, zt + r * p.ld, p.vocab, s, t);
+        }
         block_merge(s, t, red_s, red_t);
         if (threadIdx.x == 0) {
             float *o = stats + i * kStatWords;
@@ -169,7 +257,38 @@ k_shard_grad(ShardIn p, const float *__restrict__ merged, const float *__restric
             const TIn *rs = zs + r * p.ld;
             const TIn *rt = zt + r * p.ld;
             TOut *gr = grad + r * p.ld;
-            if (VEC) {
+            if constexpr (VEC && std::is_same<TIn, __nv_bfloat16>::value) {
+                // kVpU vector pairs in flight per thread, packed arithmetic
+                const uint4 *vs = reinterpret_cast<const uint4 *>(rs), *vt = reinterpret_cast<const uint4 *>(rt);
+                const float2 L2 = splat(kLog2e), NL = splat(nl), D = splat(d), CP = splat(cp), WI = splat(wi);
+                for (int64_t q0 = threadIdx.x; q0 < nvec; q0 += kVpU * kVpThreads) {
+                    uint4 a[kVpU], b[kVpU];
+#pragma unroll
+                    for (int u = 0; u < kVpU; ++u) {
+                        const int64_t q = q0 + u * kVpThreads;
+                        if (q < nvec) {
+                            a[u] = __ldg(vs + q);
+                            b[u] = __ldg(vt + q);
+                        }
+                    }
+#pragma unroll
+                    for (int u = 0; u < kVpU; ++u) {
+                        const int64_t q = q0 + u * kVpThreads;
+                        if (q >= nvec)
+                            break;
+                        float g[8];
+#pragma unroll
+                        for (int w = 0; w < 4; ++w) {
+                            const float2 a2 = unpack2(word(a[u], w)), b2 = unpack2(word(b[u], w));
+                            const float2 x = fsub2(fsub2(fsub2(a2, b2), D), CP);
+                            const float2 gg = fmul2(fmul2(ex2x2(ffma2(a2, L2, NL)), WI), x);
+                            g[2 * w] = gg.x;
+                            g[2 * w + 1] = gg.y;
+                        }
+                        store_vec<TOut, 8>(gr + q * 8, g);
+                    }
+                }
+            } else if (VEC) {
                 for (int64_t qv = threadIdx.x; qv < nvec; qv += kVpThreads) {
                     float a[N], b[N], g[N];
                     Vec<TIn>::load(rs + qv * N, a);
@@ -191,6 +310,18 @@ k_shard_grad(ShardIn p, const float *__restrict__ merged, const float *__restric
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// The grids are persistent (each CTA strides over the rows), so they are sized to
+// the CTAs that are co-resident: a larger grid would run its surplus as a late
+// second wave that ends the kernel with a tail.
+template <typename K>
+int resident_grid(K kern, int64_t rows)
+{
+    int nb = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&nb, kern, kVpThreads, 0) != cudaSuccess || nb < 1)
+        nb = 1;
+    return (int)std::min<int64_t>(std::max<int64_t>(rows, 1), (int64_t)device_sm_count() * nb);
+}
+
 }  // namespace
 
 size_t vocab_stats_bytes(int64_t T) { return sizeof(float) * kStatWords * (size_t)std::max<int64_t>(T, 0); }
@@ -200,18 +331,9 @@ cudaError_t launch_vocab_shard_stats(const VocabShardCall &c, float *stats, cuda
     ShardIn p{c.zs, c.zt, c.ld, c.vocab, c.num_rows, c.row_of_token, c.mask, c.T, c.status};
     const size_t esz = c.in_dtype == TURNOPD_BF16 ? 2 : 4;
     const bool vec = aligned16(c.zs) && aligned16(c.zt) && (c.ld * esz) % 16 == 0;
-    const int grid = (int)std::min<int64_t>(std::max<int64_t>(c.T, 1), (int64_t)device_sm_count() * 8);
-    if (c.in_dtype == TURNOPD_BF16) {
-        if (vec)
-            k_shard_stats<__nv_bfloat16, true><<<grid, kVpThreads, 0, stream>>>(p, stats);
-        else
-            k_shard_stats<__nv_bfloat16, false><<<grid, kVpThreads, 0, stream>>>(p, stats);
-    } else {
-        if (vec)
-            k_shard_stats<float, true><<<grid, kVpThreads, 0, stream>>>(p, stats);
-        else
-            k_shard_stats<float, false><<<grid, kVpThreads, 0, stream>>>(p, stats);
-    }
+    auto kern = c.in_dtype == TURNOPD_BF16 ? (vec ? k_shard_stats<__nv_bfloat16, true> : k_shard_stats<__nv_bfloat16, false>)
+                                           : (vec ? k_shard_stats<float, true> : k_shard_stats<float, false>);
+    kern<<<resident_grid(kern, c.T), kVpThreads, 0, stream>>>(p, stats);
     return cudaGetLastError();
 }
 
@@ -224,15 +346,11 @@ cudaError_t launch_vocab_stats_merge(const float *parts, int n_shards, const uin
 }
 
 template <typename TIn, typename TOut>
-static void shard_grad_kernel(const ShardIn &p, bool vec, int grid, const float *merged, const float *w, void *grad,
-                              float *tl, double *wl, int32_t *nv, cudaStream_t stream)
+static void shard_grad_kernel(const ShardIn &p, bool vec, int64_t rows, const float *merged, const float *w,
+                              void *grad, float *tl, double *wl, int32_t *nv, cudaStream_t stream)
 {
-    if (vec)
-        k_shard_grad<TIn, TOut, true><<<grid, kVpThreads, 0, stream>>>(p, merged, w, static_cast<TOut *>(grad), tl,
-                                                                      wl, nv);
-    else
-        k_shard_grad<TIn, TOut, false><<<grid, kVpThreads, 0, stream>>>(p, merged, w, static_cast<TOut *>(grad), tl,
-                                                                       wl, nv);
+    auto kern = vec ? k_shard_grad<TIn, TOut, true> : k_shard_grad<TIn, TOut, false>;
+    kern<<<resident_grid(kern, rows), kVpThreads, 0, stream>>>(p, merged, w, static_cast<TOut *>(grad), tl, wl, nv);
 }
 
 cudaError_t launch_vocab_shard_grad(const VocabShardCall &c, const float *merged, cudaStream_t stream)
@@ -245,7 +363,7 @@ cudaError_t launch_vocab_shard_grad(const VocabShardCall &c, const float *merged
                      (!c.grad || (aligned16(c.grad) && (c.ld * gesz) % 16 == 0));
     if (c.grad && (c.flags & TURNOPD_ZERO_MASKED_GRAD))
         launch_zero_masked_grad(c.mask, c.row_of_token, c.T, c.num_rows, c.ld, c.vocab, c.grad, c.grad_dtype, stream);
-    const int grid = (int)std::min<int64_t>(std::max<int64_t>(c.T, 1), (int64_t)device_sm_count() * 8);
+    const int64_t grid = c.T;  // rows to spread over the resident grid
     const bool bf_in = c.in_dtype == TURNOPD_BF16, bf_out = c.grad_dtype == TURNOPD_BF16;
     if (bf_in && bf_out)
         shard_grad_kernel<__nv_bfloat16, __nv_bfloat16>(p, vec, grid, merged, c.w, c.grad, c.token_loss, ws.row_wl,
