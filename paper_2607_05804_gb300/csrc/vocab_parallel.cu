@@ -25,7 +25,7 @@
 namespace turnopd {
 namespace {
 
-constexpr int kVpThreads = 256;
+constexpr int kVpThreads = 128;  // several rows in flight per SM: one row's merge overlaps the others' loads
 constexpr int kStatWords = 6;  // m_s, S_s, A, d, m_t, S_t
 constexpr int kVpU = 4;        // bf16 rows: vectors of each model in flight per thread
 
