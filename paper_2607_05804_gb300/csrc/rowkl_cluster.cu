@@ -483,9 +483,10 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
 constexpr int kHelpThreads = 512;
 constexpr int kHelpU = 4;  // vectors of each model in flight per thread
 
-template <bool G32>
-__global__ void __launch_bounds__(kHelpThreads, 1) k_row_helper(RowIn p)
+template <bool G32, int NTH = kHelpThreads, int MINB = 1>
+__global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
 {
+    constexpr int kHelpThreads = NTH;
     constexpr int NW = kHelpThreads / 32;
     constexpr uint32_t kFill = 0xff7fff7fu;  // lowest finite bf16 pair: adds 0, never the max
     __shared__ float red[NW][8];
@@ -680,15 +681,24 @@ constexpr int kNT = TURNOPD_ROW_THREADS;
 constexpr int kG = TURNOPD_ROW_GROUPS;
 constexpr int kMaxSlice = 2400;                      // vectors per CTA: 3 stages fit 227 KB
 constexpr int kVPT = (kMaxSlice + kNT - 1) / kNT;    // vectors per thread
-constexpr int64_t kMinVocab = 32768;  // below this the portable kernel is faster
-// The helper's rows per SM and second against the clusters' (packed 8 x 4096,
-// V = 151,936: the split that finishes both grids together was 0.86 of the rows
-// to 120 cluster SMs with 32 helper SMs).
-constexpr double kHelperRate = 0.61;
-
-size_t cluster_smem_bytes(int slice_vec)
+// Below this many columns the clusters' slices are too short to hide the per-row
+// record exchange: the helper kernel alone, on every SM, is faster (V = 65,536:
+// 0.72 of the copy bandwidth against 0.58; V = 100,000: 0.68 against 0.73).
+constexpr int64_t kClusterMinVocab = 81920;
+constexpr int kSmallRowVec = 7168;  // up to this many vectors per row: 256-thread helpers, 2 per SM
+// The helper's rows per SM and second against the clusters', which decides the
+// split of the row list.  It depends on the clusters' slice length: 0.61 for
+// slices of 2048 vectors or more (V = 151,936 in clusters of 8, 262,144 in
+// clusters of 16), about 0.9 for 1563 (V = 100,000 / 200,000); linear between.
+double helper_rate(int slice_vec)
 {
-    return (size_t)kStages * 2 * slice_vec * 16 + 2 * kG * kCS * 8 * sizeof(float) +
+    const double r = 0.61 + (2048 - slice_vec) * 0.0006;
+    return r < 0.61 ? 0.61 : (r > 1.0 ? 1.0 : r);
+}
+
+size_t cluster_smem_bytes(int slice_vec, int cs)
+{
+    return (size_t)kStages * 2 * slice_vec * 16 + 2 * kG * cs * 8 * sizeof(float) +
            kStages * sizeof(int4) + (2 * kStages + 2 * kG) * sizeof(uint64_t) +
            kG * (kNT / 32) * 8 * sizeof(float) +  // per-group warp partials
            4 * sizeof(int) +                        // row held by each stage
@@ -698,22 +708,24 @@ size_t cluster_smem_bytes(int slice_vec)
 // The cluster grid (as many clusters as are co-resident, cached per device) and
 // the helper grid on the SMs the clusters leave free, with the row list split so
 // that both finish together.
-template <bool G32>
+template <bool G32, int CS>
 cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaStream_t stream)
 {
-    auto kern = k_row_cluster<kCS, kNT, kVPT, kG, G32>;
+    auto kern = k_row_cluster<CS, kNT, kVPT, kG, G32>;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess)
         return e;
     static int grid_cache[64][2];
     static size_t smem_cache[64][2];
-    const int gi = G32 ? 1 : 0;
+    const int gi = G32 ? 1 : 0;  // per instantiation (cluster size and gradient type)
     if (dev >= 64)
         return cudaErrorInvalidDevice;
     if (smem_cache[dev][gi] < smem) {
         e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
         if (e != cudaSuccess)
+            return e;
+        if (CS > 8 && (e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) != cudaSuccess)
             return e;
         smem_cache[dev][gi] = smem;
         grid_cache[dev][gi] = 0;
@@ -721,7 +733,7 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = kCS;
+    attr[0].val.clusterDim.x = CS;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
@@ -730,7 +742,7 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
     cfg.dynamicSmemBytes = smem;
     cfg.stream = stream;
     if (grid_cache[dev][gi] == 0) {
-        cfg.gridDim = dim3(kCS);
+        cfg.gridDim = dim3(CS);
         int ncl = 0;
         e = cudaOccupancyMaxActiveClusters(&ncl, kern, &cfg);
         if (e != cudaSuccess)
@@ -740,13 +752,13 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
         grid_cache[dev][gi] = ncl;
     }
     RowIn pl = p;
-    const int free_sm = device_sm_count() - grid_cache[dev][gi] * kCS;
+    const int free_sm = device_sm_count() - grid_cache[dev][gi] * CS;
     if (free_sm > 0) {
-        const double cl = (double)(grid_cache[dev][gi] * kCS);
+        const double cl = (double)(grid_cache[dev][gi] * CS);
         pl.split_den = 1 << 20;
-        pl.split_num = (int32_t)(pl.split_den * cl / (cl + kHelperRate * free_sm) + 0.5);
+        pl.split_num = (int32_t)(pl.split_den * cl / (cl + helper_rate(slice_vec) * free_sm) + 0.5);
     }
-    cfg.gridDim = dim3(grid_cache[dev][gi] * kCS);
+    cfg.gridDim = dim3(grid_cache[dev][gi] * CS);
     e = cudaLaunchKernelEx(&cfg, kern, pl, slice_vec, nvec);
     if (e != cudaSuccess || pl.split_den == 0)
         return e;
@@ -769,14 +781,32 @@ cudaError_t launch_row_cluster(const RowIn &p, bool fp32_grad, cudaStream_t stre
 {
     *used = false;
     auto al16 = [](const void *q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
-    if (p.vocab < kMinVocab || p.vocab % 8 != 0 || p.ld % 8 != 0 || !al16(p.zs) || !al16(p.zt) ||
-        (p.grad && !al16(p.grad)))
+    if (p.vocab % 8 != 0 || p.ld % 8 != 0 || !al16(p.zs) || !al16(p.zt) || (p.grad && !al16(p.grad)))
         return cudaSuccess;
+    // clusters of 8, or of 16 (non-portable size) when an eighth of the row does not fit three stages
     const int nvec = (int)(p.vocab / 8);
-    const int slice_vec = (nvec + kCS - 1) / kCS;
-    if (slice_vec > kMaxSlice)
-        return cudaSuccess;
-    const size_t smem = cluster_smem_bytes(slice_vec);
+    const int cs = (nvec + kCS - 1) / kCS <= kMaxSlice ? kCS : 2 * kCS;
+    const int slice_vec = (nvec + cs - 1) / cs;
+    // short rows, or a slice too long even for clusters of 16: the helper kernel alone, every row, every SM
+    if (p.vocab < kClusterMinVocab || slice_vec > kMaxSlice) {
+        RowIn pl = p;
+        pl.split_den = 0;
+        const int sms = device_sm_count();
+        *used = true;
+        if (p.vocab / 8 <= kSmallRowVec) {
+            if (fp32_grad)
+                k_row_helper<true, 256, 2><<<sms * 2, 256, 0, stream>>>(pl);
+            else
+                k_row_helper<false, 256, 2><<<sms * 2, 256, 0, stream>>>(pl);
+        } else {
+            if (fp32_grad)
+                k_row_helper<true><<<sms, kHelpThreads, 0, stream>>>(pl);
+            else
+                k_row_helper<false><<<sms, kHelpThreads, 0, stream>>>(pl);
+        }
+        return cudaGetLastError();
+    }
+    const size_t smem = cluster_smem_bytes(slice_vec, cs);
     int dev = 0, optin = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess)
@@ -787,8 +817,11 @@ cudaError_t launch_row_cluster(const RowIn &p, bool fp32_grad, cudaStream_t stre
     if (smem + 64 > (size_t)optin)  // room for the kernel's static shared memory
         return cudaSuccess;
     *used = true;
-    return fp32_grad ? launch_t<true>(p, slice_vec, nvec, smem, stream)
-                     : launch_t<false>(p, slice_vec, nvec, smem, stream);
+    if (cs == kCS)
+        return fp32_grad ? launch_t<true, kCS>(p, slice_vec, nvec, smem, stream)
+                         : launch_t<false, kCS>(p, slice_vec, nvec, smem, stream);
+    return fp32_grad ? launch_t<true, 2 * kCS>(p, slice_vec, nvec, smem, stream)
+                     : launch_t<false, 2 * kCS>(p, slice_vec, nvec, smem, stream);
 }
 
 }  // namespace turnopd

@@ -128,12 +128,13 @@ def test_scopes_and_floor(P, oracle, scope, n_min):
 
 # ---------------------------------------------------------------- cluster kernel, all rows
 
-@pytest.mark.parametrize("V", [50000, W.V_QWEN])
+@pytest.mark.parametrize("V", [50000, W.V_QWEN, 262144])
 @pytest.mark.parametrize("mode", [0, 1], ids=["full", "sampled"])
 @pytest.mark.parametrize("gdt", ["bf16", "f32"])
 def test_cluster_kernel_all_rows(P, oracle, V, mode, gdt):
-    """The cluster-resident kernel (vocabularies >= 32768, multiple of 8) on every row:
-    V = 50,000 gives a ragged last slice (6250 vectors over 8 CTAs)."""
+    """The bf16 row path on every row (vocabulary a multiple of 8): V = 50,000 takes the
+    helper kernel alone, V = 151,936 clusters of 8 beside it (ragged last slice), and
+    V = 262,144 clusters of 16 beside it."""
     b = W.packed(seed=11, num_traj=2, traj_len=256)
     zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=12, device="cuda")
     run_chain(P, oracle, b, V, zs, zt, mode=mode, alpha=0.5, compact=True,
