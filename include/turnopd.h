@@ -277,8 +277,8 @@ size_t turnopd_fused_workspace_bytes(int64_t num_tokens, int64_t vocab, int64_t 
  * Inputs (device, row-major): z_student, z_teacher [num_rows, ld] of in_dtype
  *   (TURNOPD_BF16 or TURNOPD_F32), ld >= vocab; loss_mask uint8[num_tokens];
  *   w float32[num_tokens]; 1 <= k_top <= min(vocab, TURNOPD_TOPK_MAX);
- *   vocab <= TURNOPD_TOPK_MAX_VOCAB (the kernel keeps one 16-bit bucket per 16
- *   vocabulary ids of a row in shared memory).
+ *   vocab <= TURNOPD_TOPK_MAX_VOCAB (the kernel keeps, for each of the two rows it
+ *   holds at a time, one 16-bit bucket per 16 vocabulary ids in shared memory).
  * Outputs (each nullable except token_loss_out and loss_out):
  *   topk_ids_out  int32 [num_tokens, k_top]: S_i in order (largest teacher
  *                 logit first); topk_grad_out float32 [num_tokens, k_top]: g_i
@@ -297,7 +297,7 @@ size_t turnopd_fused_workspace_bytes(int64_t num_tokens, int64_t vocab, int64_t 
  *   kernel's bounded rounds (only rows with thousands of equal top logits).
  */
 #define TURNOPD_TOPK_MAX 1024
-#define TURNOPD_TOPK_MAX_VOCAB (1 << 20)
+#define TURNOPD_TOPK_MAX_VOCAB 737280  /* 720 * 1024 */
 turnopd_status turnopd_topk_loss_fwd_bwd(const void *z_student, const void *z_teacher,
                                          int32_t in_dtype, int64_t ld, int64_t vocab,
                                          int64_t num_rows, const int32_t *row_of_token,

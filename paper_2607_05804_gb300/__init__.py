@@ -43,7 +43,7 @@ TURNOPD_FORCE_PORTABLE = 0x100
 TURNOPD_MAX_TURNS = 4096
 TURNOPD_STATIC_MAX_TOKENS = 65536
 TURNOPD_TOPK_MAX = 1024
-TURNOPD_TOPK_MAX_VOCAB = 1 << 20
+TURNOPD_TOPK_MAX_VOCAB = 737280
 
 STATUS_NAMES = {
     0: "TURNOPD_OK", 1: "TURNOPD_ERR_NULL", 2: "TURNOPD_ERR_SHAPE", 3: "TURNOPD_ERR_OFFSETS",

@@ -15,16 +15,23 @@
 //            consecutive ids the largest logit is recorded in shared memory as
 //            a 16-bit ordered bucket (the top 16 bits of the order-preserving
 //            bits), and every thread keeps the largest logit it saw;
-//   bound    tau = the K-th largest of the 8 (or ceil(K/warps)) largest lane
-//            maxima of every streaming warp: K-th largest of distinct elements
-//            of the row, so a lower bound of the row's K-th largest logit;
-//   collect  only the groups whose bucket reaches tau's are read again (a few
-//            dozen per row), and their elements >= tau go to a shared-memory
-//            candidate buffer; a buffer overflow (rows of many equal logits)
-//            raises tau to the K-th largest buffered key and collects again
-//            (bounded rounds);
-//   select   the exact K-th largest buffered key by radix select, then each
-//            selected key's rank among the selected gives its position.
+//   bound    (streaming warps) for K <= 64, tau = the K-th largest of the 8
+//            largest lane maxima of every streaming warp: K-th largest of
+//            distinct elements of the row, so a lower bound of the row's K-th
+//            largest logit; above, the K-th largest group bucket (K groups each
+//            hold an element that large), by binary search on its value; then
+//            the groups whose bucket reaches tau's are listed;
+//   collect  (selector warps) only the listed groups are read again, in step
+//            across the lanes (a few dozen per row at K = 50), and their
+//            elements >= tau go to a shared-memory candidate buffer (1,024
+//            entries, 2,048 above K = 512); when it overflows (rows of many
+//            equal logits, sorted rows) a radix select over the row's keys >=
+//            tau, one key byte per pass, raises tau until the keys above it fit
+//            the buffer, then collects again (at most 6 passes for bf16 keys,
+//            8 for fp32);
+//   select   up to 256 candidates: the exact K-th largest by radix select, then
+//            each selected key's rank among the candidates is its position;
+//            more: a bitonic sort of the buffer.
 // The KL over S is evaluated by one warp in fp32 with
 // l = E_p[z_s - z_t] - (LSE_s - LSE_t) and g_v = w p_v ((z_s - z_t)_v - E_p[.]).
 
@@ -52,13 +59,22 @@ constexpr int kTkMinBlocks = TURNOPD_TOPK_MINB;  // CTAs (rows in flight) per SM
 // named barriers: buffer b full (1 + b), buffer b free (3 + b), selectors only (5),
 // streaming warps only (6)
 constexpr int kBarFull = 1, kBarFree = 3, kBarSel = 5, kBarStream = 6;
-constexpr int kTkGroupCap = 1024;  // candidate groups listed per row by the streaming warps
-constexpr int kTkCap = 1024;      // candidate buffer (keys and student logits)
-// candidate groups whose loads a thread issues together (bf16 / fp32)
-template <bool BF16>
-__host__ __device__ constexpr int tk_hits() { return BF16 ? 2 : 1; }
-constexpr int kTkRounds = 16;     // bound on overflow rounds
+constexpr int kTkGroupCap = 2048;  // candidate groups listed per row by the streaming warps
+// candidate buffer (keys and student logits): 1,024 entries, 2,048 above K = 512
+// (a power of two: the bitonic sort of a large buffer runs in place)
+__host__ __device__ constexpr int topk_cap(int K) { return K <= 512 ? 1024 : 2048; }
+// K up to which the streaming warps' lane maxima give the bound (the 8 largest
+// of each warp's 32); the group buckets give it above
+constexpr int kTkLaneTop = 8;
+constexpr int kTkLaneBoundMaxK = kTkStreamWarps * kTkLaneTop;
+// candidates above which the selection sorts the buffer instead of ranking
+constexpr int kTkRankMax = 256;
+constexpr uint32_t kTkQueue = 64;  // ring of group indices per selector warp (at most 63 held)
 constexpr int kTkGroup = 16;      // ids per recorded bucket
+static_assert(kTkQueue >= 64 && (kTkQueue & (kTkQueue - 1)) == 0, "group ring");
+static_assert(TURNOPD_TOPK_MAX_VOCAB / kTkGroup <= 65536, "group indices are 16-bit");
+static_assert(TURNOPD_TOPK_MAX_VOCAB <= (1 << 20) && topk_cap(TURNOPD_TOPK_MAX) <= 2048,
+              "a sorted key holds a 20-bit id and an 11-bit buffer position");
 
 __device__ __forceinline__ uint32_t ord16(uint32_t u)
 {
@@ -163,6 +179,51 @@ __device__ __forceinline__ void named_arrive(int id, int n)
     asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(n) : "memory");
 }
 
+// Radix-select scratch of the selector warps: a 256-bin histogram of one key
+// byte and the bin chosen from it.
+struct SelScratch {
+    uint32_t hist[256];
+    int bin, need;
+};
+
+// The bin of the need-th largest key of a 256-bin histogram sc.hist (bin 255
+// holds the largest keys): sc.bin = that bin, or -1 when the histogram holds
+// fewer than need keys; sc.need = the count still needed inside the bin,
+// negated when the bin holds exactly that many.  Run by one warp (lane 0..31).
+__device__ __forceinline__ void pick_bin(SelScratch &sc, int need, int lane)
+{
+    int c[8], tot = 0;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        c[e] = (int)sc.hist[255 - 8 * lane - e];
+        tot += c[e];
+    }
+    int incl = tot;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, off);
+        if (lane >= off)
+            incl += y;
+    }
+    const int excl = incl - tot;
+    const unsigned hit = __ballot_sync(0xffffffffu, excl < need && incl >= need);
+    if (hit == 0u) {
+        if (lane == 0)
+            sc.bin = -1;
+    } else if (lane == __ffs(hit) - 1) {
+        int cum = excl;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            if (cum + c[e] >= need) {
+                sc.bin = 255 - 8 * lane - e;
+                sc.need = (cum + c[e] == need) ? -(need - cum) : need - cum;
+                break;
+            }
+            cum += c[e];
+        }
+    }
+}
+
 // Radix select over the selector warps: the K-th largest of the nonzero keys
 // in keys[0, n) (keys are unique; 0 marks an empty slot), deciding bytes
 // hi_byte..lo_byte.  Returns t such that {keys >= t} holds the K largest keys
@@ -171,15 +232,9 @@ __device__ __forceinline__ void named_arrive(int id, int n)
 // Returns 0 when fewer than K keys are present.  Stops early once the chosen
 // bin holds exactly the remaining count.  Every selector thread (stid =
 // 0 .. kTkSelThreads-1) calls it; it synchronises them on kBarSel.
-struct SelScratch {
-    uint32_t hist[256];
-    int bin, need;
-};
-
 __device__ uint64_t sel_kth_largest(const uint64_t *keys, int n, int K, int hi_byte, int lo_byte,
                                     SelScratch &sc, int stid)
 {
-    const int lane = stid & 31;
     uint64_t prefix = 0, mask = 0;
     int need = K;
     for (int byte = hi_byte; byte >= lo_byte; --byte) {
@@ -193,39 +248,8 @@ __device__ uint64_t sel_kth_largest(const uint64_t *keys, int n, int K, int hi_b
                 atomicAdd(&sc.hist[(k >> sh) & 255u], 1u);
         }
         named_sync(kBarSel, kTkSelThreads);
-        if (stid < 32) {
-            int c[8], tot = 0;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) {
-                c[e] = (int)sc.hist[255 - 8 * lane - e];
-                tot += c[e];
-            }
-            int incl = tot;
-#pragma unroll
-            for (int off = 1; off < 32; off <<= 1) {
-                const int y = __shfl_up_sync(0xffffffffu, incl, off);
-                if (lane >= off)
-                    incl += y;
-            }
-            const int excl = incl - tot;
-            const unsigned hit = __ballot_sync(0xffffffffu, excl < need && incl >= need);
-            if (hit == 0u) {
-                if (lane == 0)
-                    sc.bin = -1;
-            } else if (lane == __ffs(hit) - 1) {
-                int cum = excl;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    if (cum + c[e] >= need) {
-                        sc.bin = 255 - 8 * lane - e;
-                        // remaining count inside the bin; negative marks "the bin is exactly it"
-                        sc.need = (cum + c[e] == need) ? -(need - cum) : need - cum;
-                        break;
-                    }
-                    cum += c[e];
-                }
-            }
-        }
+        if (stid < 32)
+            pick_bin(sc, need, stid);
         named_sync(kBarSel, kTkSelThreads);
         const int bin = sc.bin, nd = sc.need;
         named_sync(kBarSel, kTkSelThreads);
@@ -238,6 +262,48 @@ __device__ uint64_t sel_kth_largest(const uint64_t *keys, int n, int K, int hi_b
         need = nd;
     }
     return prefix;
+}
+
+// Buckets of the 16-bit pair x at or above m.
+__device__ __forceinline__ int count_ge2(uint32_t x, uint32_t m)
+{
+    return (int)((x & 0xFFFFu) >= m) + (int)((x >> 16) >= m);
+}
+
+// Sorts keys[0, n) (n a power of two >= 2 kTkSelThreads, distinct keys but for 0
+// padding) in descending order: bitonic network over the selector threads, each
+// thread loading U pairs before it compares and stores any, synchronised on
+// kBarSel after every step.
+template <int U>
+__device__ void sort_desc(uint64_t *keys, int n, int stid)
+{
+    const int np = n / 2;  // pairs per step
+    for (int k = 2; k <= n; k <<= 1)
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            for (int i0 = stid; i0 < np; i0 += U * kTkSelThreads) {
+                uint64_t x[U], y[U];
+                int l[U];
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    const int i = i0 + u * kTkSelThreads;
+                    l[u] = 2 * i - (i & (j - 1));
+                    if (i < np) {
+                        x[u] = keys[l[u]];
+                        y[u] = keys[l[u] + j];
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    // blocks with (l & k) == 0 descending, the others ascending; the last merge
+                    // (k = n) is descending throughout
+                    if (i0 + u * kTkSelThreads < np && (x[u] < y[u]) == ((l[u] & k) == 0)) {
+                        keys[l[u]] = y[u];
+                        keys[l[u] + j] = x[u];
+                    }
+                }
+            }
+            named_sync(kBarSel, kTkSelThreads);
+        }
 }
 
 struct TopkArgs {
@@ -260,7 +326,7 @@ struct TopkArgs {
 // 16-bit bucket per group of 16 ids.
 __host__ __device__ __forceinline__ size_t topk_fixed_bytes(int K)
 {
-    return align256(sizeof(uint64_t) * (kTkCap + (size_t)K) + sizeof(float) * (kTkCap + (size_t)K));
+    return align256((sizeof(uint64_t) + sizeof(float)) * ((size_t)topk_cap(K) + (size_t)K));
 }
 
 __host__ __device__ __forceinline__ int64_t topk_groups(int64_t V) { return (V + kTkGroup - 1) / kTkGroup; }
@@ -282,19 +348,22 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
     extern __shared__ __align__(128) uint64_t tk_smem[];
     const int K = a.K;
     uint64_t *s_cand = tk_smem;
-    uint64_t *s_top = s_cand + kTkCap;
+    const int cap = topk_cap(K);
+    uint64_t *s_top = s_cand + cap;
     float *s_cz = reinterpret_cast<float *>(s_top + K);   // student logit of each candidate
-    float *s_g = s_cz + kTkCap;                            // selected: student logit, then g
+    float *s_g = s_cz + cap;                               // selected: student logit, then g
     uint16_t *s_bucket0 = reinterpret_cast<uint16_t *>(reinterpret_cast<unsigned char *>(tk_smem) +
                                                        topk_fixed_bytes(K));
     __shared__ SelScratch s_sel;
     __shared__ int4 s_meta[2];      // per buffer: the row (token, row, -, weight bits)
 
     __shared__ int s_n, s_over;
-    __shared__ uint32_t s_wtop[2][kTkStreamThreads];  // per buffer: the c largest lane maxima of each warp
+    __shared__ uint32_t s_wtop[2][kTkLaneBoundMaxK];  // per buffer: the 8 largest lane maxima of each warp
     __shared__ uint32_t s_tau[2];                     // per buffer: the bound (ordered logit)
     __shared__ int s_ng[2];                           // per buffer: candidate groups found
     __shared__ uint16_t s_glist[2][kTkGroupCap];      // per buffer: their indices
+    __shared__ uint16_t s_wq[2][kTkQueue];            // per selector warp: groups found, not yet read
+    __shared__ int s_scnt[kTkStreamWarps];            // per streaming warp: a count of buckets
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int n_rows = *a.nvalid;
@@ -306,11 +375,11 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
     const int ngv = vec_ok ? (int)(a.vocab / kTkGroup) : 0;  // whole groups read as vectors
     const size_t bucket_elems = topk_bucket_bytes(a.vocab) / sizeof(uint16_t);
     constexpr int VPG = BF16 ? 2 : 4;  // 16-byte vectors per group
-    // lower bound of the K-th largest logit: every streaming warp contributes the cw largest
-    // of its lanes' maxima (cw = max(ceil(K / warps), 8) <= 32); the K-th largest of these
-    // distinct elements cannot exceed the row's K-th largest.  No bound (admit everything)
-    // when cw would exceed 32.
-    const int cw = max((K + kTkStreamWarps - 1) / kTkStreamWarps, 8);
+    // lower bound of the K-th largest logit: for K <= 64 every streaming warp contributes
+    // the 8 largest of its lanes' maxima, and the K-th largest of these distinct elements
+    // cannot exceed the row's K-th largest; above, the selectors take the K-th largest
+    // group bucket.
+    const bool lane_bound = K <= kTkLaneBoundMaxK;
 
     if (warp < kTkStreamWarps) {
         // ---- streaming warps: pass A, one row after another
@@ -382,22 +451,23 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
             }
             if (it + 1 < n_it)
                 load_batch(row_vectors(m_next), tid);  // in flight while the row is settled below
-            if (cw <= 32) {
+            if (lane_bound) {
                 bool taken = false;
-                for (int i = 0; i < cw; ++i) {
+#pragma unroll
+                for (int i = 0; i < kTkLaneTop; ++i) {
                     const uint32_t mx = __reduce_max_sync(0xffffffffu, taken ? 0u : tmax);
                     const unsigned who = __ballot_sync(0xffffffffu, !taken && tmax == mx);
                     if (who != 0u && lane == __ffs(who) - 1)
                         taken = true;
                     if (lane == 0)
-                        s_wtop[b][warp * cw + i] = mx;
+                        s_wtop[b][warp * kTkLaneTop + i] = mx;
                 }
             }
             if (tid == 0)
                 s_ng[b] = 0;
             named_sync(kBarStream, kTkStreamThreads);
-            if (cw <= 32) {
-                const int nw = kTkStreamWarps * cw;
+            if (lane_bound) {
+                constexpr int nw = kTkStreamWarps * kTkLaneTop;
                 for (int u0 = tid; u0 < nw; u0 += kTkStreamThreads) {
                     const uint32_t v = s_wtop[b][u0];
                     int gt = 0, ge = 0;
@@ -409,6 +479,38 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
                     if (v != 0 && gt < K && ge >= K)
                         s_tau[b] = v;  // every such thread writes the same value
                 }
+            } else if (a.vocab > cap) {
+                // the K-th largest group bucket, by binary search on its value with counts of
+                // the buckets at or above it: K groups each hold an element that large (no
+                // bound, tau = 0, when the row has fewer than K groups)
+                const uint4 *b4 = reinterpret_cast<const uint4 *>(s_bucket);
+                const int n4 = (int)ng / 8;
+                uint32_t lo = 0, hi = 0xFFFFu;  // count(>= lo) >= K or lo = 0; the answer is in [lo, hi]
+                while (lo < hi) {
+                    const uint32_t mid = (lo + hi + 1) >> 1;
+                    int c = 0;
+                    for (int i = tid; i < n4; i += kTkStreamThreads) {
+                        const uint4 q = b4[i];
+                        c += count_ge2(q.x, mid) + count_ge2(q.y, mid) + count_ge2(q.z, mid) + count_ge2(q.w, mid);
+                    }
+                    for (int g = n4 * 8 + tid; g < (int)ng; g += kTkStreamThreads)
+                        c += (uint32_t)s_bucket[g] >= mid;
+                    c = __reduce_add_sync(0xffffffffu, c);
+                    if (lane == 0)
+                        s_scnt[warp] = c;
+                    named_sync(kBarStream, kTkStreamThreads);
+                    int tot = 0;
+#pragma unroll
+                    for (int w = 0; w < kTkStreamWarps; ++w)
+                        tot += s_scnt[w];
+                    named_sync(kBarStream, kTkStreamThreads);
+                    if (tot >= K)
+                        lo = mid;
+                    else
+                        hi = mid - 1;
+                }
+                if (tid == 0)
+                    s_tau[b] = BF16 ? lo : lo << 16;
             }
             named_sync(kBarStream, kTkStreamThreads);
             // the whole groups that can hold an element >= tau: their bucket reaches tau's
@@ -447,7 +549,7 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
 
         auto append = [&](uint64_t k, float zsv) {
             const int p = atomicAdd(&s_n, 1);
-            if (p < kTkCap) {
+            if (p < cap) {
                 s_cand[p] = k;
                 s_cz[p] = zsv;
             } else {
@@ -456,9 +558,6 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
         };
         const uint4 *rv = reinterpret_cast<const uint4 *>(zt_row);
         const uint4 *sv = reinterpret_cast<const uint4 *>(zs_row);
-        // the candidate elements of up to kTkHits whole groups, teacher and student
-        // vectors of all of them loaded before any is used
-        constexpr int kTkHits = tk_hits<BF16>();
         // the candidate elements of one whole group: teacher vectors vt, student vectors vs
         auto scan_group = [&](const uint4 *vt, const uint4 *vs, int g) {
             uint32_t o[kTkGroup];
@@ -477,44 +576,58 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
                 }
             }
         };
-        // groups read from global memory, kTkHits at a time, all loads before any use
-        auto take_groups = [&](const int (&hg)[kTkHits], int nh) {
-            uint4 vt[kTkHits * VPG], vs[kTkHits * VPG];
-#pragma unroll
-            for (int h = 0; h < kTkHits; ++h)
-#pragma unroll
-                for (int q = 0; q < VPG; ++q)
-                    if (h < nh) {
-                        vt[h * VPG + q] = __ldg(rv + (size_t)hg[h] * VPG + q);
-                        vs[h * VPG + q] = __ldg(sv + (size_t)hg[h] * VPG + q);
-                    }
-#pragma unroll
-            for (int h = 0; h < kTkHits; ++h) {
-                if (h >= nh)
-                    break;
-                scan_group(&vt[h * VPG], &vs[h * VPG], hg[h]);
-            }
-        };
         // elements >= tau live in groups whose bucket reaches tau's: the groups the
         // streaming warps listed, or (list overflow, raised tau) a scan of the buckets
-        auto collect = [&](bool listed) {
-            const uint32_t tb = bucket<BF16>((uint32_t)(tau >> 32));
-            int hg[kTkHits];
-            int nh = 0;
-            const int n_scan = listed ? n_listed : ngv;
-            for (int i = stid; i < n_scan; i += kTkSelThreads) {
-                const int g = listed ? (int)s_glist[b][i] : i;
-                if (!listed && s_bucket[g] < tb)
-                    continue;
-
-                hg[nh++] = g;
-                if (nh == kTkHits) {
-                    take_groups(hg, nh);
-                    nh = 0;
+        // visit(g, ok) for the whole groups (g < ngv) whose bucket reaches tb, one per lane
+        // and call, the lanes converged.  Each warp walks its share of the buckets in step,
+        // queues the groups that pass (ballot) in its ring in shared memory, and visits 32 at a
+        // time, so the lanes' loads are in flight together (a lane that visited its groups
+        // alone would hold the warp for one memory round trip per group).
+        auto walk_groups = [&](uint32_t tb, auto &&visit) {
+            uint16_t *q = s_wq[swarp];
+            uint32_t head = 0, tail = 0;  // warp-uniform
+            for (int g0 = swarp * 32; g0 < ngv; g0 += kTkSelThreads) {
+                const int g = g0 + lane;
+                const bool pass = g < ngv && s_bucket[g] >= tb;
+                const unsigned m = __ballot_sync(0xffffffffu, pass);
+                if (pass)
+                    q[(tail + __popc(m & ((1u << lane) - 1u))) & (kTkQueue - 1)] = (uint16_t)g;
+                tail += __popc(m);
+                __syncwarp();
+                if (tail - head >= 32) {
+                    const int gq = q[(head + lane) & (kTkQueue - 1)];
+                    __syncwarp();
+                    head += 32;
+                    visit(gq, true);
                 }
             }
-            if (nh > 0)
-                take_groups(hg, nh);
+            if (head != tail) {  // fewer than 32 left
+                const bool ok = lane < (int)(tail - head);
+                const int gq = ok ? q[(head + lane) & (kTkQueue - 1)] : 0;
+                __syncwarp();
+                visit(gq, ok);
+            }
+        };
+        // the candidate elements of group g (ok): teacher and student vectors loaded together
+        auto take_one = [&](int g, bool ok) {
+            if (!ok)
+                return;
+            uint4 vt[VPG], vs[VPG];
+#pragma unroll
+            for (int q = 0; q < VPG; ++q) {
+                vt[q] = __ldg(rv + (size_t)g * VPG + q);
+                vs[q] = __ldg(sv + (size_t)g * VPG + q);
+            }
+            scan_group(vt, vs, g);
+        };
+        auto collect = [&](bool listed) {
+            const uint32_t tb = bucket<BF16>((uint32_t)(tau >> 32));
+            if (listed) {
+                for (int i = stid; i < n_listed; i += kTkSelThreads)
+                    take_one((int)s_glist[b][i], true);
+            } else {
+                walk_groups(tb, take_one);
+            }
             // the partial last group and misaligned rows, element by element
             for (int g = ngv + stid; g < (int)ng; g += kTkSelThreads) {
                 if (s_bucket[g] < tb)
@@ -528,11 +641,72 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
                 }
             }
         };
+        // f(k) for every key >= lo of the row: the whole groups whose bucket reaches
+        // lo's are read again (teacher only, a group per lane in step), the partial
+        // last group and misaligned rows element by element
+        auto each_key = [&](uint64_t lo, auto &&f) {
+            const uint32_t tb = bucket<BF16>((uint32_t)(lo >> 32));
+            walk_groups(tb, [&](int g, bool ok) {
+                if (!ok)
+                    return;
+                uint4 vt[VPG];
+#pragma unroll
+                for (int q = 0; q < VPG; ++q)
+                    vt[q] = __ldg(rv + (size_t)g * VPG + q);
+                uint32_t o[kTkGroup];
+                unpack_ords<BF16>(vt, o);
+                const uint32_t e0 = (uint32_t)g * kTkGroup;
+#pragma unroll
+                for (int e = 0; e < kTkGroup; ++e) {
+                    const uint64_t k = mkkey(o[e], e0 + e);
+                    if (k >= lo)
+                        f(k);
+                }
+            });
+            for (int g = ngv + stid; g < (int)ng; g += kTkSelThreads) {
+                if (s_bucket[g] < tb)
+                    continue;
+                const int64_t e0 = (int64_t)g * kTkGroup;
+                for (int64_t e = e0; e < e0 + kTkGroup && e < a.vocab; ++e) {
+                    const uint64_t k = mkkey(elem_ord<BF16>(zt_row, e), (uint32_t)e);
+                    if (k >= lo)
+                        f(k);
+                }
+            }
+        };
         collect(n_listed <= kTkGroupCap);
         named_sync(kBarSel, kTkSelThreads);
-        // ---- overflow: raise tau to the K-th largest buffered key and collect again
-        for (int round = 0; s_over && round < kTkRounds; ++round) {
-            tau = sel_kth_largest(s_cand, kTkCap, K, 7, 0, s_sel, stid);
+        if (s_over) {
+            // ---- overflow: radix select over the row's keys >= tau, one key byte per
+            // pass from the top, until the keys >= the chosen prefix fit the buffer.
+            // Keys above the prefix number K - need; those with the prefix, cnt.
+            uint64_t prefix = 0, pmask = 0;
+            int need = K;
+            for (int byte = hi_val; byte >= 0; --byte) {
+                const int sh = 8 * byte;
+                for (int i = stid; i < 256; i += kTkSelThreads)
+                    s_sel.hist[i] = 0;
+                named_sync(kBarSel, kTkSelThreads);
+                each_key(max(tau, prefix), [&](uint64_t k) {
+                    if ((k & pmask) == prefix)
+                        atomicAdd(&s_sel.hist[(k >> sh) & 255u], 1u);
+                });
+                named_sync(kBarSel, kTkSelThreads);
+                if (stid < 32)
+                    pick_bin(s_sel, need, stid);
+                named_sync(kBarSel, kTkSelThreads);
+                const int bin = s_sel.bin, nd = s_sel.need;
+                const int cnt = bin >= 0 ? (int)s_sel.hist[bin] : 0;
+                named_sync(kBarSel, kTkSelThreads);
+                if (bin < 0)
+                    break;  // fewer than K keys >= tau: not reached, tau is a lower bound
+                prefix |= (uint64_t)bin << sh;
+                pmask |= (uint64_t)255u << sh;
+                if (nd < 0 || K - nd + cnt <= cap)
+                    break;
+                need = nd;
+            }
+            tau = max(tau, prefix);
             if (stid == 0) {
                 s_n = 0;
                 s_over = 0;
@@ -542,7 +716,7 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
             named_sync(kBarSel, kTkSelThreads);
         }
         const bool failed = s_over != 0;
-        const int nc = min(s_n, kTkCap);
+        const int nc = min(s_n, cap);
         named_sync(kBarSel, kTkSelThreads);
         if (failed) {
             if (stid == 0) {
@@ -551,22 +725,43 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
                 a.row_wl[j] = 0.0;
             }
         } else {
-            // ---- the K largest: each candidate's rank among the candidates is its position
-            // (keys are unique); a large buffer is first cut to the K largest by radix select
-            const uint64_t kth = nc <= kTkSelThreads ? 0 : sel_kth_largest(s_cand, nc, K, hi_val, 0, s_sel, stid);
-            for (int i = stid; i < nc; i += kTkSelThreads) {
-                const uint64_t k = s_cand[i];
-                if (k < kth)
-                    continue;
-                int rank = 0;
-                int i2 = 0;
-                for (; i2 + 4 <= nc; i2 += 4)
-                    rank += (s_cand[i2] > k) + (s_cand[i2 + 1] > k) + (s_cand[i2 + 2] > k) + (s_cand[i2 + 3] > k);
-                for (; i2 < nc; ++i2)
-                    rank += s_cand[i2] > k;
-                if (rank < K) {
-                    s_top[rank] = k;
-                    s_g[rank] = s_cz[i];
+            if (nc > kTkRankMax) {
+                // ---- the K largest of a large buffer: sort it (padded with 0 keys to a power
+                // of two, at most the buffer's size) and take the first K
+                // Each key carries its buffer position in its low 11 bits, below the id's 20:
+                // ids are below 2^20, so ~id's upper 12 bits are ones and the order is kept.
+                int n2 = kTkRankMax;
+                while (n2 < nc)
+                    n2 <<= 1;
+                for (int i = stid; i < n2; i += kTkSelThreads) {
+                    const uint64_t k = s_cand[i];
+                    s_cand[i] = i < nc ? (k & 0xFFFFFFFF00000000ull) | ((k & 0xFFFFFull) << 11) | (uint64_t)i : 0ull;
+                }
+                named_sync(kBarSel, kTkSelThreads);
+                sort_desc<BF16 ? 4 : 2>(s_cand, n2, stid);
+                for (int r = stid; r < K; r += kTkSelThreads) {
+                    const uint64_t p = s_cand[r];
+                    s_top[r] = (p & 0xFFFFFFFF00000000ull) | 0xFFF00000ull | ((p >> 11) & 0xFFFFFull);
+                    s_g[r] = s_cz[p & 0x7FFu];
+                }
+            } else {
+                // ---- the K largest: each candidate's rank among the candidates is its position
+                // (keys are unique); a buffer above 64 is first cut to the K largest by radix select
+                const uint64_t kth = nc <= kTkSelThreads ? 0 : sel_kth_largest(s_cand, nc, K, hi_val, 0, s_sel, stid);
+                for (int i = stid; i < nc; i += kTkSelThreads) {
+                    const uint64_t k = s_cand[i];
+                    if (k < kth)
+                        continue;
+                    int rank = 0;
+                    int i2 = 0;
+                    for (; i2 + 4 <= nc; i2 += 4)
+                        rank += (s_cand[i2] > k) + (s_cand[i2 + 1] > k) + (s_cand[i2 + 2] > k) + (s_cand[i2 + 3] > k);
+                    for (; i2 < nc; ++i2)
+                        rank += s_cand[i2] > k;
+                    if (rank < K) {
+                        s_top[rank] = k;
+                        s_g[rank] = s_cz[i];
+                    }
                 }
             }
             named_sync(kBarSel, kTkSelThreads);

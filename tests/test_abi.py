@@ -134,7 +134,7 @@ def test_topk_host_validation(lib):
     assert call(k=0) == 2
     assert call(k=1025) == 2
     assert call(k=51, vocab=50, ld=64) == 2          # k_top > vocab
-    assert call(vocab=(1 << 20) + 1, ld=(1 << 20) + 1) == 2
+    assert call(vocab=737280 + 1, ld=737280 + 8) == 2
     assert call(ld=100, vocab=101) == 2
     assert call(rows=10) == 2
     assert call(ids=ctypes.c_void_p(0x10002)) == 2   # misaligned int32 output

@@ -205,6 +205,49 @@ def test_full_vocab_packed_sampled_rows_and_properties(P, oracle):
         <= 1e-6 * abs(loss)
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32])
+@pytest.mark.parametrize("K", [65, 200, 256, 257, 513, 1024])
+def test_large_k_full_vocab(P, oracle, dtype, K):
+    """K above 64: the bound is the K-th largest group bucket; above 256
+    candidates the buffer is sorted, and above K = 512 it holds 2,048."""
+    V, T = W.V_QWEN, 6
+    zs, zt = W.make_logits(T, V, "agent", dtype, seed=17 + K, device="cuda")
+    mask = torch.ones(T, dtype=torch.uint8, device="cuda")
+    w = torch.linspace(0.1, 1.0, T, dtype=torch.float32, device="cuda")
+    ids, gk, tl, loss, st = run_topk(P, zs, zt, V, mask, w, K)
+    assert st == 0
+    check_against_oracle(oracle, zs, zt, V, mask, w, K, ids, gk, tl, loss)
+
+
+@pytest.mark.parametrize("K", [50, 256, 1024])
+def test_sorted_rows(P, oracle, K):
+    """Teacher rows in ascending and descending id order, and a row with the
+    top ids spread by a stride: orders that defeat sampling-based bounds."""
+    V, T = W.V_QWEN, 3
+    base = torch.linspace(-8.0, 8.0, V, dtype=torch.float32)
+    zt = torch.stack([base, base.flip(0), base[torch.randperm(V, generator=torch.Generator().manual_seed(9))]])
+    zt = zt.to(torch.bfloat16).cuda()
+    zs = (torch.randn(T, V, generator=torch.Generator().manual_seed(10)) * 2).to(torch.bfloat16).cuda()
+    mask = torch.ones(T, dtype=torch.uint8, device="cuda")
+    w = torch.ones(T, dtype=torch.float32, device="cuda")
+    ids, gk, tl, loss, st = run_topk(P, zs, zt, V, mask, w, K)
+    assert st == 0
+    check_against_oracle(oracle, zs, zt, V, mask, w, K, ids, gk, tl, loss)
+
+
+def test_largest_vocabulary_and_largest_k(P, oracle):
+    """V = TURNOPD_TOPK_MAX_VOCAB with K = TURNOPD_TOPK_MAX: the shared-memory layout at its
+    largest (two rows of buckets, the K-sized arrays)."""
+    V, K = P.TURNOPD_TOPK_MAX_VOCAB, P.TURNOPD_TOPK_MAX
+    T = 3
+    zs, zt = W.make_logits(T, V, "agent", torch.bfloat16, seed=31, device="cuda")
+    mask = torch.ones(T, dtype=torch.uint8, device="cuda")
+    w = torch.full((T,), 0.25, dtype=torch.float32, device="cuda")
+    ids, gk, tl, loss, st = run_topk(P, zs, zt, V, mask, w, K)
+    assert st == 0
+    check_against_oracle(oracle, zs, zt, V, mask, w, K, ids, gk, tl, loss)
+
+
 def test_empty_and_all_masked(P):
     V, K = 512, 8
     zs = torch.zeros((4, V), dtype=torch.bfloat16, device="cuda")
