@@ -373,8 +373,15 @@ def fused_bench(args, world, rank, local):
     import paper_2607_05804_gb300 as P
     from paper_2607_05804_gb300.step import LossStep, to_device
 
+    from paper_2607_05804_gb300 import dp
+
     device = torch.device("cuda", local)
     torch.cuda.set_device(device)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl", device_id=device)
     P.load()
     b = W.fused(seed=rank, num_traj=args.num_traj or 8, traj_len=args.traj_len or 2048)
     d_s, d_t, V = 4096, 5120, W.V_QWEN
@@ -387,7 +394,7 @@ def fused_bench(args, world, rank, local):
     dW = torch.empty((V, d_s), dtype=torch.float32, device=device) if args.dw else None
 
     def one(ev=None):
-        step.weights()
+        step.weights(dp.global_counts(step.local_counts()) if world > 1 else None)
         if ev is not None:
             ev[0].record()
         P.turnopd_fused_lmhead_fwd_bwd(h_s, W_s, h_t, W_t, msk, step.w[:T], 0, dh,
@@ -395,6 +402,8 @@ def fused_bench(args, world, rank, local):
         if ev is not None:
             ev[1].record()
         step.turn_stats()
+        if world > 1:
+            dp.reduce_step(step.loss, step.turn_sum, step.turn_cnt, step.turn_surv)
 
     for _ in range(max(args.warmup, 3)):
         one()
@@ -405,6 +414,8 @@ def fused_bench(args, world, rank, local):
            for _ in range(args.steps)]
     a, z = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     sampler = ClockSampler(local)
+    if world > 1:
+        dist.barrier()
     torch.cuda.synchronize()
     sampler.start()
     a.record()
@@ -412,10 +423,20 @@ def fused_bench(args, world, rank, local):
         one(evs[k])
     z.record()
     torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
     clocks = sampler.stop()
     ms = a.elapsed_time(z)
     call_ms = statistics.mean(x.elapsed_time(y) for x, y in evs)
     Tv = b.num_valid
+    tot_valid = Tv
+    if world > 1:
+        t = torch.tensor([ms, call_ms], device=device, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms, call_ms = float(t[0].item()), float(t[1].item())
+        n = torch.tensor([Tv], device=device, dtype=torch.int64)
+        dist.all_reduce(n)
+        tot_valid = int(n.item())
     flops = 2.0 * Tv * V * (d_s + d_t) * 2 + 2.0 * Tv * V * d_s  # forward, recompute, dH
     if args.dw:
         flops += 2.0 * Tv * V * d_s  # dW_s
@@ -430,7 +451,7 @@ def fused_bench(args, world, rank, local):
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = fused_cpu_baseline(b, (h_s, W_s, h_t, W_t), step.w[:T])
-    out = {"metric": "fused LM-head loss fwd+bwd supervised tokens/s", "value": Tv * args.steps / (ms / 1e3),
+    out = {"metric": "fused LM-head loss fwd+bwd supervised tokens/s", "value": tot_valid * args.steps / (ms / 1e3),
            "unit": "tokens/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
            "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
@@ -444,7 +465,10 @@ def fused_bench(args, world, rank, local):
            "gpu_launches": (FUSED_KERNELS_PER_STEP + (1 if args.dw else 0)) * args.steps, "clocks": clocks,
            "e2e": None,
            "cpu_baseline": cpu}
-    print(json.dumps(out), flush=True)
+    if rank == 0:
+        print(json.dumps(out), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
 
 
 def main():
