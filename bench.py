@@ -224,7 +224,7 @@ def vocab_parallel_loss_fn(step, zs, zt, grad, n_shards):
     def call():
         for r in range(n_shards):
             P.turnopd_vocab_shard_stats(zs[:, cuts[r]:cuts[r + 1]], zt[:, cuts[r]:cuts[r + 1]], step.row_of_token,
-                                        step.loss_mask, parts[r], step.dev_status)
+                                        step.loss_mask, parts[r], step.ws_l, step.dev_status)
         P.turnopd_vocab_stats_merge(parts, step.loss_mask, merged)
         for r in range(n_shards):
             P.turnopd_vocab_shard_loss_grad(zs[:, cuts[r]:cuts[r + 1]], zt[:, cuts[r]:cuts[r + 1]],

@@ -317,7 +317,9 @@ turnopd_status turnopd_topk_loss_fwd_bwd(const void *z_student, const void *z_te
  *      row statistics stats_out[i, 0..5] = (m_s, S_s, A, d, m_t, S_t):
  *      m = max logit, S = sum exp(z - m), d = (z_s - z_t) at the student's
  *      largest logit, A = sum exp(z_s - m_s) ((z_s - z_t) - d)  (float32,
- *      turnopd_vocab_stats_bytes(num_tokens) bytes; masked rows untouched);
+ *      turnopd_vocab_stats_bytes(num_tokens) bytes; masked rows untouched;
+ *      workspace as for turnopd_loss_fwd_bwd, turnopd_loss_workspace_bytes
+ *      (num_tokens) bytes, 256-byte aligned, else TURNOPD_ERR_WORKSPACE);
  *   2. the caller gathers every shard's stats into parts[n_shards, num_tokens, 6]
  *      in shard order (e.g. an all-gather);
  *   3. turnopd_vocab_stats_merge: the whole vocabulary's row statistics, merged
@@ -335,8 +337,8 @@ size_t turnopd_vocab_stats_bytes(int64_t num_tokens);
 turnopd_status turnopd_vocab_shard_stats(const void *z_student, const void *z_teacher, int32_t in_dtype,
                                          int64_t ld, int64_t shard_vocab, int64_t num_rows,
                                          const int32_t *row_of_token, const uint8_t *loss_mask,
-                                         int64_t num_tokens, float *stats_out, int32_t *dev_status,
-                                         turnopd_stream_t stream);
+                                         int64_t num_tokens, float *stats_out, void *workspace,
+                                         size_t workspace_bytes, int32_t *dev_status, turnopd_stream_t stream);
 turnopd_status turnopd_vocab_stats_merge(const float *parts, int32_t n_shards, const uint8_t *loss_mask,
                                          int64_t num_tokens, float *merged_out, turnopd_stream_t stream);
 turnopd_status turnopd_vocab_shard_loss_grad(const void *z_student, const void *z_teacher, int32_t in_dtype,

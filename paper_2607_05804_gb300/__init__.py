@@ -100,7 +100,7 @@ def load():
         "turnopd_depth_efficiency": [P, P, P, i32, D, P, P, P, P],
         "turnopd_depth_coverage": [P, P, i32, D, i32, i32, i32, P],
         "turnopd_turn_diagnostics": [P, P, P, i32, i32, P, P, P],
-        "turnopd_vocab_shard_stats": [P, P, i32, i64, i64, i64, P, P, i64, P, P, P],
+        "turnopd_vocab_shard_stats": [P, P, i32, i64, i64, i64, P, P, i64, P, P, ctypes.c_size_t, P, P],
         "turnopd_vocab_stats_merge": [P, i32, P, i64, P, P],
         "turnopd_selftest_wait_timeout": [u32, P, P],
         "turnopd_vocab_shard_loss_grad": [P, P, i32, i64, i64, i64, P, P, P, i64, P, P, i32, u32, P, P, P,
@@ -359,10 +359,10 @@ def turnopd_vocab_stats_bytes(num_tokens: int) -> int:
     return int(load().turnopd_vocab_stats_bytes(int(num_tokens)))
 
 
-def turnopd_vocab_shard_stats(z_student, z_teacher, row_of_token, loss_mask, stats_out, dev_status,
+def turnopd_vocab_shard_stats(z_student, z_teacher, row_of_token, loss_mask, stats_out, workspace, dev_status,
                               stream=None):
     """z_student, z_teacher: this rank's [num_rows, shard_vocab] column shard (row stride ld);
-    stats_out float32 [T, 6]."""
+    stats_out float32 [T, 6]; workspace of turnopd_loss_workspace_bytes(T) bytes."""
     import torch
 
     ld, Vr = _shard_logits(z_student, z_teacher)
@@ -370,10 +370,12 @@ def turnopd_vocab_shard_stats(z_student, z_teacher, row_of_token, loss_mask, sta
     _need(row_of_token, "row_of_token", torch.int32, T)
     _need(loss_mask, "loss_mask", torch.uint8)
     _need(stats_out, "stats_out", torch.float32, T * 6)
+    _need(workspace, "workspace")
     _need(dev_status, "dev_status", torch.int32, 1)
     _check(load().turnopd_vocab_shard_stats(
         _ptr(z_student), _ptr(z_teacher), _dtype_code(z_student, "z_student"), ld, Vr, z_student.shape[0],
-        _ptr(row_of_token), _ptr(loss_mask), T, _ptr(stats_out), _ptr(dev_status), _stream(stream)),
+        _ptr(row_of_token), _ptr(loss_mask), T, _ptr(stats_out), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _ptr(dev_status), _stream(stream)),
         "turnopd_vocab_shard_stats")
 
 

@@ -298,7 +298,8 @@ static turnopd_status vocab_common_checks(const void *z_student, const void *z_t
 turnopd_status turnopd_vocab_shard_stats(const void *z_student, const void *z_teacher, int32_t in_dtype, int64_t ld,
                                          int64_t shard_vocab, int64_t num_rows, const int32_t *row_of_token,
                                          const uint8_t *loss_mask, int64_t num_tokens, float *stats_out,
-                                         int32_t *dev_status, turnopd_stream_t stream)
+                                         void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                                         turnopd_stream_t stream)
 {
     NvtxRange nvtx("turnopd_vocab_shard_stats");
     turnopd_status st = vocab_common_checks(z_student, z_teacher, in_dtype, ld, shard_vocab, num_rows, row_of_token,
@@ -309,10 +310,12 @@ turnopd_status turnopd_vocab_shard_stats(const void *z_student, const void *z_te
         return TURNOPD_ERR_NULL;
     if (misaligned(stats_out, 4))
         return TURNOPD_ERR_SHAPE;
+    if (!workspace || misaligned(workspace, 256) || workspace_bytes < loss_workspace_bytes(num_tokens))
+        return TURNOPD_ERR_WORKSPACE;
     if (num_tokens == 0)
         return TURNOPD_OK;
     VocabShardCall c{z_student, z_teacher, in_dtype, ld, shard_vocab, num_rows, row_of_token, loss_mask, nullptr,
-                     num_tokens, nullptr, TURNOPD_F32, 0u, nullptr, nullptr, nullptr, dev_status};
+                     num_tokens, nullptr, TURNOPD_F32, 0u, nullptr, nullptr, workspace, dev_status};
     return cuda_status(launch_vocab_shard_stats(c, stats_out, (cudaStream_t)stream));
 }
 

@@ -152,31 +152,18 @@ __device__ __forceinline__ void block_merge(Student &s, Teacher &t, Student *red
     }
 }
 
-__device__ __forceinline__ bool token_row(const ShardIn &p, int64_t i, int64_t *r)
-{
-    if (!p.mask[i])
-        return false;
-    const int64_t row = p.row_of_token ? (int64_t)p.row_of_token[i] : i;
-    if (row < 0 || row >= p.num_rows) {
-        if (threadIdx.x == 0)
-            set_status(p.status, TURNOPD_ERR_TOKEN_RANGE);
-        return false;
-    }
-    *r = row;
-    return true;
-}
-
 template <typename TIn, bool VEC>
-__global__ void __launch_bounds__(kVpThreads) k_shard_stats(ShardIn p, float *__restrict__ stats)
+__global__ void __launch_bounds__(kVpThreads) k_shard_stats(ShardIn p, const int4 *__restrict__ rows,
+                                                             const int32_t *__restrict__ nvalid, float *__restrict__ stats)
 {
     __shared__ Student red_s[kVpThreads / 32];
     __shared__ Teacher red_t[kVpThreads / 32];
     const TIn *zs = static_cast<const TIn *>(p.zs);
     const TIn *zt = static_cast<const TIn *>(p.zt);
-    for (int64_t i = blockIdx.x; i < p.T; i += gridDim.x) {
-        int64_t r;
-        if (!token_row(p, i, &r))
-            continue;
+    const int n = *nvalid;
+    for (int j = blockIdx.x; j < n; j += gridDim.x) {
+        const int4 m = rows[j];  // (token, row, -, -)
+        const int64_t i = m.x, r = m.y;
         Student s = student_empty();
         Teacher t = teacher_empty();
         if constexpr (VEC && std::is_same<TIn, __nv_bfloat16>::value) {
@@ -219,37 +206,31 @@ __global__ void k_stats_merge(const float *__restrict__ parts, int n_shards, con
 
 template <typename TIn, typename TOut, bool VEC>
 __global__ void __launch_bounds__(kVpThreads)
-k_shard_grad(ShardIn p, const float *__restrict__ merged, const float *__restrict__ w, TOut *grad, float *token_loss,
-             double *wl, int32_t *nvalid_slot)
+k_shard_grad(ShardIn p, const int4 *__restrict__ rows, const int32_t *__restrict__ nvalid,
+             const float *__restrict__ merged, TOut *grad, float *token_loss, double *wl)
 {
     __shared__ float bc[4];
     constexpr int N = Vec<TIn>::N;
-    if (blockIdx.x == 0 && threadIdx.x == 0)
-        *nvalid_slot = (int32_t)p.T;  // the loss sum runs over every token (0 for masked ones)
     const TIn *zs = static_cast<const TIn *>(p.zs);
     const TIn *zt = static_cast<const TIn *>(p.zt);
     const int64_t V = p.vocab;
     const int64_t nvec = VEC ? V / N : 0;
-    for (int64_t i = blockIdx.x; i < p.T; i += gridDim.x) {
-        int64_t r;
-        if (!token_row(p, i, &r)) {
-            if (threadIdx.x == 0) {
-                token_loss[i] = 0.f;
-                wl[i] = 0.0;
-            }
-            continue;
-        }
+    const int n = *nvalid;
+    for (int j = blockIdx.x; j < n; j += gridDim.x) {
+        const int4 m = rows[j];  // (token, row, -, w bits)
+        const int64_t i = m.x, r = m.y;
         if (threadIdx.x == 0) {
+            const float wi = __int_as_float(m.w);
             const float *q = merged + i * kStatWords;
             const RowConst rc = row_const(Student{q[0], q[1], q[2], q[3]}, Teacher{q[4], q[5]});
             if (!isfinite(rc.lse_s) || !isfinite(rc.lse_t) || !isfinite(rc.kl))
                 set_status(p.status, TURNOPD_ERR_NONFINITE);
             token_loss[i] = rc.kl;
-            wl[i] = (double)w[i] * (double)rc.kl;
+            wl[j] = (double)wi * (double)rc.kl;
             bc[0] = rc.lse_s;
             bc[1] = rc.d;
             bc[2] = rc.cp;
-            bc[3] = w[i];
+            bc[3] = wi;
         }
         __syncthreads();
         if (grad) {
@@ -326,14 +307,40 @@ int resident_grid(K kern, int64_t rows)
 
 size_t vocab_stats_bytes(int64_t T) { return sizeof(float) * kStatWords * (size_t)std::max<int64_t>(T, 0); }
 
+// The supervised rows in token order as (token, row, -, w) records, and their count
+// (the loss path's compaction; it also zeroes token_loss of the other tokens), so
+// each CTA of a persistent grid takes an equal share of the rows.
+static cudaError_t compact_rows(const VocabShardCall &c, const float *w, float *token_loss, const LossWorkspace &ws,
+                                cudaStream_t stream)
+{
+    LossArgs la{};
+    la.mask = c.mask;
+    la.row_of_token = c.row_of_token;
+    la.w = w;
+    la.T = c.T;
+    la.num_rows = c.num_rows;
+    la.vocab = c.vocab;
+    la.mode = TURNOPD_FULL_VOCAB;
+    la.token_loss = token_loss;
+    la.status = c.status;
+    return launch_compaction(la, ws.rows, ws.blk_count, ws.nvalid, stream);
+}
+
 cudaError_t launch_vocab_shard_stats(const VocabShardCall &c, float *stats, cudaStream_t stream)
 {
+    LossWorkspace ws = loss_workspace_layout(c.workspace, c.T);
+    // The statistics pass needs neither the records' weights nor the zeroed token
+    // losses: both point into the row_wl scratch (T doubles), unused by this call.
+    float *scratch = reinterpret_cast<float *>(ws.row_wl);
+    cudaError_t e = compact_rows(c, scratch, scratch, ws, stream);
+    if (e != cudaSuccess)
+        return e;
     ShardIn p{c.zs, c.zt, c.ld, c.vocab, c.num_rows, c.row_of_token, c.mask, c.T, c.status};
     const size_t esz = c.in_dtype == TURNOPD_BF16 ? 2 : 4;
     const bool vec = aligned16(c.zs) && aligned16(c.zt) && (c.ld * esz) % 16 == 0;
     auto kern = c.in_dtype == TURNOPD_BF16 ? (vec ? k_shard_stats<__nv_bfloat16, true> : k_shard_stats<__nv_bfloat16, false>)
                                            : (vec ? k_shard_stats<float, true> : k_shard_stats<float, false>);
-    kern<<<resident_grid(kern, c.T), kVpThreads, 0, stream>>>(p, stats);
+    kern<<<resident_grid(kern, c.T), kVpThreads, 0, stream>>>(p, ws.rows, ws.nvalid, stats);
     return cudaGetLastError();
 }
 
@@ -346,11 +353,12 @@ cudaError_t launch_vocab_stats_merge(const float *parts, int n_shards, const uin
 }
 
 template <typename TIn, typename TOut>
-static void shard_grad_kernel(const ShardIn &p, bool vec, int64_t rows, const float *merged, const float *w,
-                              void *grad, float *tl, double *wl, int32_t *nv, cudaStream_t stream)
+static void shard_grad_kernel(const ShardIn &p, bool vec, const LossWorkspace &ws, const float *merged, void *grad,
+                              float *tl, cudaStream_t stream)
 {
     auto kern = vec ? k_shard_grad<TIn, TOut, true> : k_shard_grad<TIn, TOut, false>;
-    kern<<<resident_grid(kern, rows), kVpThreads, 0, stream>>>(p, merged, w, static_cast<TOut *>(grad), tl, wl, nv);
+    kern<<<resident_grid(kern, p.T), kVpThreads, 0, stream>>>(p, ws.rows, ws.nvalid, merged,
+                                                                  static_cast<TOut *>(grad), tl, ws.row_wl);
 }
 
 cudaError_t launch_vocab_shard_grad(const VocabShardCall &c, const float *merged, cudaStream_t stream)
@@ -361,22 +369,21 @@ cudaError_t launch_vocab_shard_grad(const VocabShardCall &c, const float *merged
     const size_t gesz = c.grad_dtype == TURNOPD_BF16 ? 2 : 4;
     const bool vec = aligned16(c.zs) && aligned16(c.zt) && (c.ld * esz) % 16 == 0 &&
                      (!c.grad || (aligned16(c.grad) && (c.ld * gesz) % 16 == 0));
+    cudaError_t e = compact_rows(c, c.w, c.token_loss, ws, stream);
+    if (e != cudaSuccess)
+        return e;
     if (c.grad && (c.flags & TURNOPD_ZERO_MASKED_GRAD))
         launch_zero_masked_grad(c.mask, c.row_of_token, c.T, c.num_rows, c.ld, c.vocab, c.grad, c.grad_dtype, stream);
-    const int64_t grid = c.T;  // rows to spread over the resident grid
     const bool bf_in = c.in_dtype == TURNOPD_BF16, bf_out = c.grad_dtype == TURNOPD_BF16;
     if (bf_in && bf_out)
-        shard_grad_kernel<__nv_bfloat16, __nv_bfloat16>(p, vec, grid, merged, c.w, c.grad, c.token_loss, ws.row_wl,
-                                                        ws.nvalid, stream);
+        shard_grad_kernel<__nv_bfloat16, __nv_bfloat16>(p, vec, ws, merged, c.grad, c.token_loss, stream);
     else if (bf_in)
-        shard_grad_kernel<__nv_bfloat16, float>(p, vec, grid, merged, c.w, c.grad, c.token_loss, ws.row_wl, ws.nvalid,
-                                                stream);
+        shard_grad_kernel<__nv_bfloat16, float>(p, vec, ws, merged, c.grad, c.token_loss, stream);
     else if (bf_out)
-        shard_grad_kernel<float, __nv_bfloat16>(p, vec, grid, merged, c.w, c.grad, c.token_loss, ws.row_wl, ws.nvalid,
-                                                stream);
+        shard_grad_kernel<float, __nv_bfloat16>(p, vec, ws, merged, c.grad, c.token_loss, stream);
     else
-        shard_grad_kernel<float, float>(p, vec, grid, merged, c.w, c.grad, c.token_loss, ws.row_wl, ws.nvalid, stream);
-    cudaError_t e = cudaGetLastError();
+        shard_grad_kernel<float, float>(p, vec, ws, merged, c.grad, c.token_loss, stream);
+    e = cudaGetLastError();
     if (e != cudaSuccess)
         return e;
     launch_loss_sum(ws.row_wl, ws.nvalid, c.loss, c.status, stream);

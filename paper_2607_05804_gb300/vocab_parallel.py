@@ -21,7 +21,8 @@ def vocab_parallel_loss(z_student, z_teacher, row_of_token, loss_mask, w, grad_s
     T = loss_mask.numel()
     st = dev_status if dev_status is not None else torch.zeros(1, dtype=torch.int32, device=dev)
     part = torch.empty((max(T, 1), 6), dtype=torch.float32, device=dev)
-    turnopd_vocab_shard_stats(z_student, z_teacher, row_of_token, loss_mask, part[:T], st)
+    ws = torch.empty(max(turnopd_loss_workspace_bytes(T), 256), dtype=torch.uint8, device=dev)
+    turnopd_vocab_shard_stats(z_student, z_teacher, row_of_token, loss_mask, part[:T], ws, st)
     world = dist.get_world_size(group) if dist.is_available() and dist.is_initialized() else 1
     if world > 1:
         parts = [torch.empty_like(part) for _ in range(world)]
@@ -33,7 +34,6 @@ def vocab_parallel_loss(z_student, z_teacher, row_of_token, loss_mask, w, grad_s
     turnopd_vocab_stats_merge(parts[:, :T].contiguous(), loss_mask, merged[:T])
     token_loss = torch.empty(max(T, 1), dtype=torch.float32, device=dev)
     loss = torch.zeros(1, dtype=torch.float64, device=dev)
-    ws = torch.empty(max(turnopd_loss_workspace_bytes(T), 256), dtype=torch.uint8, device=dev)
     turnopd_vocab_shard_loss_grad(z_student, z_teacher, row_of_token, loss_mask, w, merged[:T], grad_shard, flags,
                                   token_loss[:T], loss, ws, st)
     return token_loss[:T], loss

@@ -145,6 +145,27 @@ def test_topk_host_validation(lib):
     assert call(wsb=ws_need - 1) == 10
 
 
+def test_vocab_shard_host_validation(lib):
+    f = lib.turnopd_vocab_shard_stats
+    ws_need = lib.turnopd_loss_workspace_bytes(64)
+
+    def call(zs=FAKE, ld=1024, vocab=1024, rows=64, T=64, in_dtype=1, stats=FAKE, ws=FAKE, wsb=None,
+             status=FAKE):
+        return f(zs, FAKE, in_dtype, ld, vocab, rows, None, FAKE, T, stats, ws,
+                 ws_need if wsb is None else wsb, status, None)
+
+    assert call(zs=None) == 1
+    assert call(status=None) == 1
+    assert call(stats=None) == 1
+    assert call(in_dtype=5) == 6
+    assert call(ld=100, vocab=101) == 2
+    assert call(rows=63) == 2                        # no row map: a row per token
+    assert call(stats=ctypes.c_void_p(0x10002)) == 2  # misaligned float32 output
+    assert call(ws=None) == 10
+    assert call(wsb=ws_need - 1) == 10
+    assert call(ws=ctypes.c_void_p(0x10010)) == 10    # not 256-byte aligned
+
+
 def test_selftest_wait_timeout_host_validation(lib):
     f = lib.turnopd_selftest_wait_timeout
     assert f(100, None, None) == 1                # TURNOPD_ERR_NULL

@@ -27,12 +27,12 @@ def run_split(P, zs, zt, rot, mask, w, cuts, grad_dtype):
     T = mask.numel()
     st = torch.zeros(1, dtype=torch.int32, device="cuda")
     parts = torch.empty((len(cuts) - 1, T, 6), dtype=torch.float32, device="cuda")
+    ws = torch.empty(max(P.turnopd_loss_workspace_bytes(T), 256), dtype=torch.uint8, device="cuda")
     for r, (a, b) in enumerate(zip(cuts[:-1], cuts[1:])):
-        P.turnopd_vocab_shard_stats(zs[:, a:b], zt[:, a:b], rot, mask, parts[r], st)
+        P.turnopd_vocab_shard_stats(zs[:, a:b], zt[:, a:b], rot, mask, parts[r], ws, st)
     merged = torch.empty((T, 6), dtype=torch.float32, device="cuda")
     P.turnopd_vocab_stats_merge(parts, mask, merged)
     grad = torch.full(zs.shape, 7.0, dtype=grad_dtype, device="cuda")
-    ws = torch.empty(max(P.turnopd_loss_workspace_bytes(T), 256), dtype=torch.uint8, device="cuda")
     losses, tls = [], []
     for a, b in zip(cuts[:-1], cuts[1:]):
         tl = torch.empty(T, dtype=torch.float32, device="cuda")
