@@ -156,13 +156,18 @@ template <typename TIn, bool VEC>
 __global__ void __launch_bounds__(kVpThreads) k_shard_stats(ShardIn p, const int4 *__restrict__ rows,
                                                              const int32_t *__restrict__ nvalid, float *__restrict__ stats)
 {
-    __shared__ Student red_s[kVpThreads / 32];
-    __shared__ Teacher red_t[kVpThreads / 32];
+    // reduction scratch per row parity: the next row's warps write the other half while
+    // thread 0 still reads this one, so no barrier closes the row
+    __shared__ Student red_s[2][kVpThreads / 32];
+    __shared__ Teacher red_t[2][kVpThreads / 32];
     const TIn *zs = static_cast<const TIn *>(p.zs);
     const TIn *zt = static_cast<const TIn *>(p.zt);
     const int n = *nvalid;
-    for (int j = blockIdx.x; j < n; j += gridDim.x) {
-        const int4 m = rows[j];  // (token, row, -, -)
+    int4 m_next = (int)blockIdx.x < n ? rows[blockIdx.x] : make_int4(0, 0, 0, 0);
+    for (int j = blockIdx.x, par = 0; j < n; j += gridDim.x, par ^= 1) {
+        const int4 m = m_next;  // (token, row, -, -), loaded a row ahead
+        if (j + (int)gridDim.x < n)
+            m_next = rows[j + gridDim.x];
         const int64_t i = m.x, r = m.y;
         Student s = student_empty();
         Teacher t = teacher_empty();
@@ -177,12 +182,11 @@ __global__ void __launch_bounds__(kVpThreads) k_shard_stats(ShardIn p, const int
         } else {
             fold_row<TIn, VEC>(zs + r * p.ld, zt + r * p.ld, p.vocab, s, t);
         }
-        block_merge(s, t, red_s, red_t);
+        block_merge(s, t, red_s[par], red_t[par]);
         if (threadIdx.x == 0) {
             float *o = stats + i * kStatWords;
             o[0] = s.m, o[1] = s.s, o[2] = s.a, o[3] = s.d, o[4] = t.m, o[5] = t.s;
         }
-        __syncthreads();
     }
 }
 
@@ -209,16 +213,20 @@ __global__ void __launch_bounds__(kVpThreads)
 k_shard_grad(ShardIn p, const int4 *__restrict__ rows, const int32_t *__restrict__ nvalid,
              const float *__restrict__ merged, TOut *grad, float *token_loss, double *wl)
 {
-    __shared__ float bc[4];
+    __shared__ float bc2[2][4];  // per row parity (see k_shard_stats)
     constexpr int N = Vec<TIn>::N;
     const TIn *zs = static_cast<const TIn *>(p.zs);
     const TIn *zt = static_cast<const TIn *>(p.zt);
     const int64_t V = p.vocab;
     const int64_t nvec = VEC ? V / N : 0;
     const int n = *nvalid;
-    for (int j = blockIdx.x; j < n; j += gridDim.x) {
-        const int4 m = rows[j];  // (token, row, -, w bits)
+    int4 m_next = (int)blockIdx.x < n ? rows[blockIdx.x] : make_int4(0, 0, 0, 0);
+    for (int j = blockIdx.x, par = 0; j < n; j += gridDim.x, par ^= 1) {
+        const int4 m = m_next;  // (token, row, -, w bits), loaded a row ahead
+        if (j + (int)gridDim.x < n)
+            m_next = rows[j + gridDim.x];
         const int64_t i = m.x, r = m.y;
+        float *bc = bc2[par];
         if (threadIdx.x == 0) {
             const float wi = __int_as_float(m.w);
             const float *q = merged + i * kStatWords;
@@ -285,7 +293,6 @@ k_shard_grad(ShardIn p, const int4 *__restrict__ rows, const int32_t *__restrict
                 gr[v] = from_float<TOut>(wi * ex2(fmaf(a, kLog2e, nl)) * (((a - b) - d) - cp));
             }
         }
-        __syncthreads();
     }
 }
 
