@@ -599,10 +599,11 @@ def main():
                             else committed_traffic(args.workload, R, "topk") if args.mode == "topk"
                             else committed_traffic(args.workload)),
             },
-            # vocabulary shards: counts(2) + weights(1) + per shard stats, gradient and loss sum + merge + stats(2)
+            # vocabulary shards: counts(2) + weights(1) + per shard the statistics call (compaction(2),
+            # statistics) and the gradient call (compaction(2), gradient, loss sum) + merge + stats(2)
             "gpu_launches": ((KERNELS_PER_STEP + (1 if args.zero_masked else 0) + (0 if args.mode == "topk" else 1))
                              if not args.vocab_shards
-                             else 6 + 3 * args.vocab_shards) * args.steps,
+                             else 6 + 7 * args.vocab_shards) * args.steps,
             "clocks": clocks,
             "e2e": e2e,
             "cpu_baseline": cpu,
