@@ -338,9 +338,9 @@ __host__ __device__ __forceinline__ size_t topk_bucket_bytes(int64_t V)
 
 size_t topk_smem_bytes(int64_t V, int K) { return topk_fixed_bytes(K) + 2 * topk_bucket_bytes(V); }
 
-// One CTA holds two rows at a time: its streaming warps run pass A of row
-// i + 1 (into bucket buffer (i + 1) % 2) while its two selector warps run
-// bound, collect, select and the KL of row i from buffer i % 2, so the SM's
+// One CTA holds two rows at a time: its streaming warps run pass A and the
+// bound of row i + 1 (into bucket buffer (i + 1) % 2) while its two selector
+// warps run collect, select and the KL of row i from buffer i % 2, so the SM's
 // teacher stream does not pause for the latency-bound phases.
 template <bool BF16>
 __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs a)
@@ -377,8 +377,8 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
     constexpr int VPG = BF16 ? 2 : 4;  // 16-byte vectors per group
     // lower bound of the K-th largest logit: for K <= 64 every streaming warp contributes
     // the 8 largest of its lanes' maxima, and the K-th largest of these distinct elements
-    // cannot exceed the row's K-th largest; above, the selectors take the K-th largest
-    // group bucket.
+    // cannot exceed the row's K-th largest; above, the streaming warps take the K-th
+    // largest group bucket.
     const bool lane_bound = K <= kTkLaneBoundMaxK;
 
     if (warp < kTkStreamWarps) {
@@ -576,8 +576,6 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
                 }
             }
         };
-        // elements >= tau live in groups whose bucket reaches tau's: the groups the
-        // streaming warps listed, or (list overflow, raised tau) a scan of the buckets
         // visit(g, ok) for the whole groups (g < ngv) whose bucket reaches tb, one per lane
         // and call, the lanes converged.  Each warp walks its share of the buckets in step,
         // queues the groups that pass (ballot) in its ring in shared memory, and visits 32 at a
@@ -589,10 +587,10 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
             for (int g0 = swarp * 32; g0 < ngv; g0 += kTkSelThreads) {
                 const int g = g0 + lane;
                 const bool pass = g < ngv && s_bucket[g] >= tb;
-                const unsigned m = __ballot_sync(0xffffffffu, pass);
+                const unsigned hit = __ballot_sync(0xffffffffu, pass);
                 if (pass)
-                    q[(tail + __popc(m & ((1u << lane) - 1u))) & (kTkQueue - 1)] = (uint16_t)g;
-                tail += __popc(m);
+                    q[(tail + __popc(hit & ((1u << lane) - 1u))) & (kTkQueue - 1)] = (uint16_t)g;
+                tail += __popc(hit);
                 __syncwarp();
                 if (tail - head >= 32) {
                     const int gq = q[(head + lane) & (kTkQueue - 1)];
@@ -620,6 +618,8 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
             }
             scan_group(vt, vs, g);
         };
+        // elements >= tau live in groups whose bucket reaches tau's: the groups the
+        // streaming warps listed, or (list overflow, raised tau) a walk over the buckets
         auto collect = [&](bool listed) {
             const uint32_t tb = bucket<BF16>((uint32_t)(tau >> 32));
             if (listed) {
