@@ -363,7 +363,8 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
     __shared__ int s_ng[2];                           // per buffer: candidate groups found
     __shared__ uint16_t s_glist[2][kTkGroupCap];      // per buffer: their indices
     __shared__ uint16_t s_wq[2][kTkQueue];            // per selector warp: groups found, not yet read
-    __shared__ int s_scnt[kTkStreamWarps];            // per streaming warp: a count of buckets
+    __shared__ int s_scnt[2][kTkStreamWarps];         // per streaming warp: a count of buckets
+    __shared__ uint32_t s_smax[kTkStreamWarps];       // per streaming warp: its largest bucket
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int n_rows = *a.nvalid;
@@ -485,9 +486,23 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
                 // bound, tau = 0, when the row has fewer than K groups)
                 const uint4 *b4 = reinterpret_cast<const uint4 *>(s_bucket);
                 const int n4 = (int)ng / 8;
-                uint32_t lo = 0, hi = 0xFFFFu;  // count(>= lo) >= K or lo = 0; the answer is in [lo, hi]
-                while (lo < hi) {
-                    const uint32_t mid = (lo + hi + 1) >> 1;
+                // The answer is at most the row's largest bucket; the first pass probes 255 below
+                // it (where the K-th largest bucket of a row with a few hundred large logits lies),
+                // and only when fewer than K buckets reach that does the search span the rest.
+                const uint32_t wmax = __reduce_max_sync(0xffffffffu, bucket<BF16>(tmax));
+                if (lane == 0)
+                    s_smax[warp] = wmax;
+                named_sync(kBarStream, kTkStreamThreads);
+                uint32_t hi = 0;
+#pragma unroll
+                for (int w = 0; w < kTkStreamWarps; ++w)
+                    hi = max(hi, s_smax[w]);
+                uint32_t lo = 0;  // count(>= lo) >= K or lo = 0; the answer is in [lo, hi]
+                const uint32_t probe = hi > 255u ? hi - 255u : 0u;
+                // the warps' counts alternate between two rows of s_scnt, so one barrier a pass
+                // suffices: a pass's reads finish before any thread passes the next barrier
+                for (int par = 0, first = 1; lo < hi; par ^= 1, first = 0) {
+                    const uint32_t mid = first && probe > lo ? probe : (lo + hi + 1) >> 1;
                     int c = 0;
                     for (int i = tid; i < n4; i += kTkStreamThreads) {
                         const uint4 q = b4[i];
@@ -497,13 +512,12 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
                         c += (uint32_t)s_bucket[g] >= mid;
                     c = __reduce_add_sync(0xffffffffu, c);
                     if (lane == 0)
-                        s_scnt[warp] = c;
+                        s_scnt[par][warp] = c;
                     named_sync(kBarStream, kTkStreamThreads);
                     int tot = 0;
 #pragma unroll
                     for (int w = 0; w < kTkStreamWarps; ++w)
-                        tot += s_scnt[w];
-                    named_sync(kBarStream, kTkStreamThreads);
+                        tot += s_scnt[par][w];
                     if (tot >= K)
                         lo = mid;
                     else
