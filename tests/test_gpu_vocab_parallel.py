@@ -105,3 +105,49 @@ def test_fp32_unaligned_split_and_helper(P, oracle):
     torch.cuda.synchronize()
     assert_token_loss(tl.cpu().numpy(), tl_ref, b.loss_mask)
     assert_loss(loss.item(), loss_ref)
+
+
+def test_bad_row_index_sets_status_and_skips_the_token(P, oracle):
+    """A supervised token whose row index is out of range: both calls record
+    TURNOPD_ERR_TOKEN_RANGE, the token gets loss 0 and no gradient row, and every
+    other token matches the oracle with that token masked out."""
+    b = W.tiny(seed=3)
+    V, T = 1024, b.num_tokens
+    zs, zt = W.make_logits(T, V, "tiny", torch.bfloat16, seed=42, device="cuda")
+    sup = np.nonzero(b.loss_mask)[0]
+    bad = int(sup[len(sup) // 2])
+    rot_np = np.arange(T, dtype=np.int32)
+    rot_np[bad] = T + 5
+    rot = torch.from_numpy(rot_np).cuda()
+    mask = torch.from_numpy(b.loss_mask).cuda()
+    w = torch.rand(T, generator=torch.Generator().manual_seed(6)).cuda()
+    cuts = [0, 512, V]
+    st = torch.zeros(1, dtype=torch.int32, device="cuda")
+    ws = torch.empty(max(P.turnopd_loss_workspace_bytes(T), 256), dtype=torch.uint8, device="cuda")
+    parts = torch.empty((2, T, 6), dtype=torch.float32, device="cuda")
+    for r, (a, e) in enumerate(zip(cuts[:-1], cuts[1:])):
+        P.turnopd_vocab_shard_stats(zs[:, a:e], zt[:, a:e], rot, mask, parts[r], ws, st)
+    torch.cuda.synchronize()
+    assert st.item() == 5  # TURNOPD_ERR_TOKEN_RANGE
+    merged = torch.empty((T, 6), dtype=torch.float32, device="cuda")
+    P.turnopd_vocab_stats_merge(parts, mask, merged)
+    grad = torch.full(zs.shape, 7.0, dtype=torch.float32, device="cuda")
+    tl = torch.full((T,), 3.0, dtype=torch.float32, device="cuda")
+    loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+    for a, e in zip(cuts[:-1], cuts[1:]):
+        st.zero_()
+        P.turnopd_vocab_shard_loss_grad(zs[:, a:e], zt[:, a:e], rot, mask, w, merged, grad[:, a:e], 0, tl, loss,
+                                        ws, st)
+        torch.cuda.synchronize()
+        assert st.item() == 5
+    m2 = b.loss_mask.copy()
+    m2[bad] = 0
+    g_ref, tl_ref, loss_ref = oracle.loss_fwd_bwd(W.bf16_bits(zs), W.bf16_bits(zt), V, m2, w.cpu().numpy())
+    tl_h = tl.cpu().numpy()
+    assert tl_h[bad] == 0.0
+    assert_token_loss(tl_h, tl_ref, m2)
+    assert_loss(loss.item(), loss_ref)
+    g = grad.cpu().numpy()
+    assert (g[bad] == 7.0).all()  # no token maps to this row
+    ok = m2 == 1
+    assert_grad_rows(g[ok], g_ref[ok], bf16=False)
