@@ -358,7 +358,7 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
     __shared__ int4 s_meta[2];      // per buffer: the row (token, row, -, weight bits)
 
     __shared__ int s_n, s_over;
-    __shared__ uint32_t s_wtop[2][kTkLaneBoundMaxK];  // per buffer: the 8 largest lane maxima of each warp
+    __shared__ __align__(16) uint32_t s_wtop[2][kTkLaneBoundMaxK];  // per buffer: each warp's 8 largest lane maxima
     __shared__ uint32_t s_tau[2];                     // per buffer: the bound (ordered logit)
     __shared__ int s_ng[2];                           // per buffer: candidate groups found
     __shared__ uint16_t s_glist[2][kTkGroupCap];      // per buffer: their indices
@@ -453,29 +453,33 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
             if (it + 1 < n_it)
                 load_batch(row_vectors(m_next), tid);  // in flight while the row is settled below
             if (lane_bound) {
-                bool taken = false;
+                // the warp's 8 largest lane maxima: a bitonic sort of the 32 in registers,
+                // descending, leaves them in lanes 0..7
+                uint32_t x = tmax;
 #pragma unroll
-                for (int i = 0; i < kTkLaneTop; ++i) {
-                    const uint32_t mx = __reduce_max_sync(0xffffffffu, taken ? 0u : tmax);
-                    const unsigned who = __ballot_sync(0xffffffffu, !taken && tmax == mx);
-                    if (who != 0u && lane == __ffs(who) - 1)
-                        taken = true;
-                    if (lane == 0)
-                        s_wtop[b][warp * kTkLaneTop + i] = mx;
-                }
+                for (int k = 2; k <= 32; k <<= 1)
+#pragma unroll
+                    for (int j = k >> 1; j > 0; j >>= 1) {
+                        const uint32_t y = __shfl_xor_sync(0xffffffffu, x, j);
+                        x = (((lane & j) == 0) == ((lane & k) == 0)) ? max(x, y) : min(x, y);
+                    }
+                if (lane < kTkLaneTop)
+                    s_wtop[b][warp * kTkLaneTop + lane] = x;
             }
             if (tid == 0)
                 s_ng[b] = 0;
             named_sync(kBarStream, kTkStreamThreads);
             if (lane_bound) {
                 constexpr int nw = kTkStreamWarps * kTkLaneTop;
+                const uint4 *w4 = reinterpret_cast<const uint4 *>(s_wtop[b]);
                 for (int u0 = tid; u0 < nw; u0 += kTkStreamThreads) {
                     const uint32_t v = s_wtop[b][u0];
                     int gt = 0, ge = 0;
-                    for (int u = 0; u < nw; ++u) {
-                        const uint32_t x = s_wtop[b][u];
-                        gt += x > v;
-                        ge += x >= v;
+#pragma unroll
+                    for (int q = 0; q < nw / 4; ++q) {
+                        const uint4 x = w4[q];
+                        gt += (x.x > v) + (x.y > v) + (x.z > v) + (x.w > v);
+                        ge += (x.x >= v) + (x.y >= v) + (x.z >= v) + (x.w >= v);
                     }
                     if (v != 0 && gt < K && ge >= K)
                         s_tau[b] = v;  // every such thread writes the same value
@@ -528,13 +532,26 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
             }
             named_sync(kBarStream, kTkStreamThreads);
             // the whole groups that can hold an element >= tau: their bucket reaches tau's
+            // (eight buckets a load; the list's order does not matter)
             const uint32_t tb = bucket<BF16>(s_tau[b]);
-            for (int g = tid; g < ngv; g += kTkStreamThreads)
-                if (s_bucket[g] >= tb) {
-                    const int p = atomicAdd(&s_ng[b], 1);
-                    if (p < kTkGroupCap)
-                        s_glist[b][p] = (uint16_t)g;
-                }
+            auto list = [&](int g) {
+                const int p = atomicAdd(&s_ng[b], 1);
+                if (p < kTkGroupCap)
+                    s_glist[b][p] = (uint16_t)g;
+            };
+            const uint4 *b8 = reinterpret_cast<const uint4 *>(s_bucket);
+            const int n8 = ngv / 8;
+            for (int i = tid; i < n8; i += kTkStreamThreads) {
+                const uint4 q = b8[i];
+                const uint32_t w4[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+                for (int e = 0; e < 8; ++e)
+                    if (((w4[e >> 1] >> (16 * (e & 1))) & 0xFFFFu) >= tb)
+                        list(i * 8 + e);
+            }
+            for (int g = n8 * 8 + tid; g < ngv; g += kTkStreamThreads)
+                if (s_bucket[g] >= tb)
+                    list(g);
             named_arrive(kBarFull + b, kTkThreads);  // row it is in buffer b
         }
         return;
