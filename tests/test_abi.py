@@ -171,3 +171,28 @@ def test_selftest_wait_timeout_host_validation(lib):
     assert f(100, None, None) == 1                # TURNOPD_ERR_NULL
     assert f(0, FAKE, None) == 2                  # TURNOPD_ERR_SHAPE: no polls
     assert f((1 << 24) + 1, FAKE, None) == 2      # TURNOPD_ERR_SHAPE: beyond the cap
+
+
+def declared_parameter_counts():
+    """name -> number of parameters, from every prototype in the header."""
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    src = re.sub(r"//[^\n]*", "", src)
+    out = {}
+    for m in re.finditer(r"^[A-Za-z_][\w \*]*?\b(turnopd_\w+)\s*\(([^;{]*?)\)\s*;", src, flags=re.M | re.S):
+        params = m.group(2).strip()
+        out[m.group(1)] = 0 if params in ("", "void") else params.count(",") + 1
+    return out
+
+
+def test_binding_argument_counts_match_header(lib):
+    counts = declared_parameter_counts()
+    assert "turnopd_vocab_shard_stats" in counts and "turnopd_loss_fwd_bwd" in counts
+    checked = 0
+    for name, n in counts.items():
+        argtypes = getattr(lib, name).argtypes
+        if argtypes is None:
+            continue
+        assert len(argtypes) == n, (name, len(argtypes), n)
+        checked += 1
+    assert checked >= 20
