@@ -104,7 +104,11 @@ __global__ void k_counts_reduce(const int32_t *__restrict__ n_bt, int32_t B, int
 // ---------------------------------------------------------------- weights
 
 // One CTA per trajectory: its token weights from n_bt[b][:] and the
-// (possibly rank-summed) count vector.  Arithmetic in fp64.
+// (possibly rank-summed) count vector.  Arithmetic in fp64, once per turn: a
+// token's weight depends only on its trajectory and turn, so the CTA fills a
+// per-turn table and each token reads its entry (fp64 runs at a small fraction
+// of the fp32 rate, and a division per token on one SM per trajectory cost
+// more than the rest of the kernel).
 __global__ void k_weights(const int32_t *__restrict__ turn_id, const uint8_t *__restrict__ mask,
                           const int64_t *__restrict__ off, int32_t B, int64_t T, int32_t Tmax,
                           double alpha, int32_t scope, int32_t n_min,
@@ -113,6 +117,7 @@ __global__ void k_weights(const int32_t *__restrict__ turn_id, const uint8_t *__
 {
     __shared__ int64_t red[4][32];
     __shared__ double coef[3];  // token weight 1/N_b (or 1/N), reliable-turn numerator, R
+    __shared__ float s_wt[TURNOPD_MAX_TURNS];  // this trajectory's token weight per turn
     const int b = blockIdx.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nw = blockDim.x >> 5;
@@ -158,18 +163,22 @@ __global__ void k_weights(const int32_t *__restrict__ turn_id, const uint8_t *__
     __syncthreads();
     const double w_traj = coef[0], share = coef[1], R = coef[2];
     const double norm = scope == TURNOPD_SCOPE_TRAJ ? (Bp > 0 ? 1.0 / (double)Bp : 0.0) : 1.0;
+    for (int t = threadIdx.x; t < Tmax; t += blockDim.x) {
+        float wt = 0.f;
+        if (w_traj > 0.0) {
+            const bool reliable = n_min <= 0 || S[t] >= n_min;
+            const double w_turn = (!reliable || R == 0.0) ? w_traj : share / (R * (double)nb[t]);
+            wt = (float)(((1.0 - alpha) * w_traj + alpha * w_turn) * norm);
+        }
+        s_wt[t] = wt;  // turns without tokens here are never read
+    }
+    __syncthreads();
 
     int64_t lo, hi;
     traj_range(off, B, T, b, lo, hi, status);
     for (int64_t i = lo + threadIdx.x; i < hi; i += blockDim.x) {
-        float wi = 0.f;
-        int32_t t = mask[i] ? turn_id[i] : -1;
-        if (t >= 0 && t < Tmax && w_traj > 0.0) {
-            const bool reliable = n_min <= 0 || S[t] >= n_min;
-            double w_turn = (!reliable || R == 0.0) ? w_traj : share / (R * (double)nb[t]);
-            wi = (float)(((1.0 - alpha) * w_traj + alpha * w_turn) * norm);
-        }
-        w_out[i] = wi;
+        const int32_t t = mask[i] ? turn_id[i] : -1;
+        w_out[i] = t >= 0 && t < Tmax ? s_wt[t] : 0.f;
     }
     // tokens outside every trajectory range (only with bad offsets) stay untouched
 }
