@@ -184,3 +184,68 @@ def test_fused_errors(P):
         P.turnopd_fused_lmhead_fwd_bwd(z(T, d_s), z(V, d_s), z(T, d_t), z(V, d_t), msk, w, 0, None, tl,
                                        loss, ws[:1024], st)
     assert e.value.code == 10
+
+
+# Pair tiles are 256 supervised rows; units of the forward and recompute grids are
+# enumerated in blocks of at most 16 row tiles; dL/dh_s has (rows/256) x (d_s/256)
+# tiles, of which the first floor(tiles/P)*P (P = co-resident pairs, at most 76 on
+# 152 SMs) are whole tiles and the rest are split over all pairs.
+PAIR_ROWS, UNIT_BLOCK, MAX_PAIRS = 256, 16, 76
+
+
+def test_fused_mid_size_all_rows_and_weight_gradient(P, oracle):
+    """Every supervised row of a 5,255-row batch (21 pair row tiles: the units run
+    as two blocks, 11 + 10 row tiles) with d_s = 1024 (84 dh tiles: whole tiles for
+    the first 76, split k-ranges and the pair-ordered fixup for the rest), d_t = 256,
+    V = 8192 (32 vocabulary tiles: three groups of 10 and a group of 2).  Loss,
+    per-token loss, dL/dh_s and dL/dW_s (128 tiles over the pairs, so pairs take two
+    tiles through the double accumulator) are compared element by element."""
+    b = W.packed(seed=21, num_traj=3, traj_len=2920)
+    d_s, d_t, V = 1024, 256, 8192
+    m_tiles = -(-b.num_valid // PAIR_ROWS)
+    assert m_tiles == 21 and m_tiles > UNIT_BLOCK and m_tiles * (d_s // 256) > MAX_PAIRS
+    heads, w, dh, tl, loss, dW = run_fused(P, b, d_s, d_t, V, seed=22, dw=True)
+    bits = [W.bf16_bits(x) for x in heads]
+    dh_ref, tl_ref, loss_ref, dw_ref = oracle.fused_lmhead(*bits, b.loss_mask, w, dW=True)
+    assert_token_loss(tl, tl_ref, b.loss_mask)
+    assert_loss(loss, loss_ref)
+    g = dh.cpu().numpy()
+    m = b.loss_mask == 1
+    assert (g[~m] == 0).all()
+    assert_dh(g[m], dh_ref[m])
+    assert_dh(dW.cpu().numpy(), dw_ref)
+
+
+def test_fused_full_size_sampled_rows(P, oracle):
+    """The benchmark's fused configuration at full size: 8 x 2048 tokens (9,840
+    supervised: 39 pair row tiles, so three unit blocks of 13), d_s = 4096,
+    d_t = 5120, V = 151,936, alpha = 1.  The oracle recomputes rows drawn from each
+    unit block, from whole dh tiles and from the last row tile, whose 16 dh tiles
+    are the split ones; every row is checked by the size-free properties."""
+    b = W.fused(0)
+    d_s, d_t, V = 4096, 5120, W.V_QWEN
+    R = b.num_valid
+    m_tiles = -(-R // PAIR_ROWS)
+    nb = -(-m_tiles // UNIT_BLOCK)
+    mb = -(-m_tiles // nb)
+    assert nb == 3 and (m_tiles * (d_s // 256)) % MAX_PAIRS != 0
+    heads, w, dh, tl, loss = run_fused(P, b, d_s, d_t, V, seed=30)
+    rng = np.random.default_rng(31)
+    picks = [0, R - 1]
+    for blk in range(nb):                        # rows of every unit block
+        lo, hi = blk * mb * PAIR_ROWS, min(R, (blk + 1) * mb * PAIR_ROWS)
+        picks += list(rng.integers(lo, hi, 4))
+    last = (m_tiles - 1) * PAIR_ROWS            # rows of the split dh tiles
+    picks += list(rng.integers(last, R, 4)) + [last]
+    rows = np.unique(np.asarray(picks))
+    toks = np.nonzero(b.loss_mask)[0][rows]
+    bits = [W.bf16_bits(x) for x in heads]
+    dh_ref, tl_ref, _ = oracle.fused_lmhead(*bits, b.loss_mask, w, subset=toks)
+    assert_token_loss(tl[toks], tl_ref[toks])
+    g = dh.cpu().numpy()
+    assert_dh(g[toks], dh_ref[toks])
+    assert (g[b.loss_mask == 0] == 0).all()
+    assert (tl[b.loss_mask == 0] == 0).all()
+    assert (tl[b.loss_mask == 1] >= -1e-4).all()
+    wl = float(np.dot(w.astype(np.float64), tl.astype(np.float64)))
+    assert abs(loss - wl) <= 1e-9 * abs(wl)
