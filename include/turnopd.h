@@ -201,8 +201,10 @@ size_t turnopd_loss_workspace_bytes(int64_t num_tokens);
  * Limits: num_tokens > TURNOPD_STATIC_MAX_TOKENS returns TURNOPD_ERR_WORKSPACE
  * before anything is launched.
  * Set-up: the first call on a device looks up the array's device address
- * (cudaGetSymbolAddress, with that device current).  Make that first call
- * before any stream capture.
+ * (cudaGetSymbolAddress, with that device current) and keeps it for the
+ * CUDA context it was taken in; a call made in another context of that device
+ * (after cudaDeviceReset, say) looks it up again.  Make the first call in each
+ * context before any stream capture.
  * Sharing: all calls use the one array.  Calls that can overlap on the GPU
  * (different streams, or several host threads) race on it and may return
  * wrong results: issue them on one stream.  The array keeps whatever the last

@@ -2,7 +2,9 @@
 // a file-scope device array, for callers that cannot allocate device memory.
 // It forwards to turnopd_loss_fwd_bwd with that array as the workspace.
 
-#include <atomic>
+#include <mutex>
+
+#include <cuda.h>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -21,10 +23,53 @@ static_assert(kBytes == TURNOPD_STATIC_SCRATCH_BYTES, "header constant out of da
 static __device__ __align__(256) unsigned char g_loss_scratch[kBytes];
 
 constexpr int kMaxDevices = 64;
-std::atomic<void *> g_scratch_addr[kMaxDevices];
 
-// Device address of g_loss_scratch on the current device (looked up once per
-// device; the host-side symbol itself is not a device address).
+// The array's device address belongs to one CUDA context: after a
+// cudaDeviceReset (or any teardown of the primary context) the module is
+// loaded again and the array may sit elsewhere.  So the cached address is
+// keyed on the context's process-unique id (cuCtxGetId), and looked up again
+// whenever the current context is not the one it was taken in.
+struct ScratchSlot {
+    std::mutex mu;
+    unsigned long long ctx_id = 0;
+    void *addr = nullptr;
+};
+ScratchSlot g_slot[kMaxDevices];
+
+typedef CUresult (*PFN_ctxGetCurrent)(CUcontext *);
+typedef CUresult (*PFN_ctxGetId)(CUcontext, unsigned long long *);
+
+template <class F>
+F driver_fn(const char *name, int version)
+{
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion(name, &p, version, cudaEnableDefault, &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+        return nullptr;
+    return reinterpret_cast<F>(p);
+}
+
+// Id of the context current on this thread (0 if none is current yet).
+turnopd_status current_ctx_id(unsigned long long *id)
+{
+    static PFN_ctxGetCurrent get_current = driver_fn<PFN_ctxGetCurrent>("cuCtxGetCurrent", 4000);
+    static PFN_ctxGetId get_id = driver_fn<PFN_ctxGetId>("cuCtxGetId", 12000);
+    if (!get_current || !get_id)
+        return TURNOPD_ERR_CUDA;
+    CUcontext ctx = nullptr;
+    if (get_current(&ctx) != CUDA_SUCCESS)
+        return TURNOPD_ERR_CUDA;
+    *id = 0;
+    if (ctx && get_id(ctx, id) != CUDA_SUCCESS)
+        return TURNOPD_ERR_CUDA;
+    return TURNOPD_OK;
+}
+
+// Device address of g_loss_scratch in the current context of the current
+// device.  The lookup (cudaGetSymbolAddress, which also makes the runtime's
+// primary context current if none is) runs on the first call in a context;
+// later calls in the same context take the cached address.
 turnopd_status scratch_address(void **out)
 {
     int dev = 0;
@@ -32,13 +77,22 @@ turnopd_status scratch_address(void **out)
         return TURNOPD_ERR_CUDA;
     if (dev < 0 || dev >= kMaxDevices)
         return TURNOPD_ERR_UNSUPPORTED;
-    void *p = g_scratch_addr[dev].load(std::memory_order_acquire);
-    if (!p) {
+    unsigned long long id = 0;
+    turnopd_status st = current_ctx_id(&id);
+    if (st != TURNOPD_OK)
+        return st;
+    ScratchSlot &slot = g_slot[dev];
+    std::lock_guard<std::mutex> lock(slot.mu);
+    if (id == 0 || id != slot.ctx_id || !slot.addr) {
+        void *p = nullptr;
         if (cudaGetSymbolAddress(&p, g_loss_scratch) != cudaSuccess || !p)
             return TURNOPD_ERR_CUDA;
-        g_scratch_addr[dev].store(p, std::memory_order_release);
+        if ((st = current_ctx_id(&id)) != TURNOPD_OK || id == 0)
+            return st != TURNOPD_OK ? st : TURNOPD_ERR_CUDA;
+        slot.ctx_id = id;
+        slot.addr = p;
     }
-    *out = p;
+    *out = slot.addr;
     return TURNOPD_OK;
 }
 

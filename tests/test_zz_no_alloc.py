@@ -4,16 +4,17 @@ workspace entry point (turnopd_loss_fwd_bwd).
 turnopd_loss_fwd_bwd_static exists for callers that cannot allocate device
 memory (their memory belongs to an allocator or arena that forbids raw
 cudaMalloc/cudaFree, or they have no allocator to hand out a workspace); it keeps
-its scratch in a static device array inside the library.  Two calls in a row,
+its scratch in a static device array inside the library.  Three calls in a row,
 with different inputs and sizes, must each match the workspace entry point on
-the same inputs within the parity tolerances, so nothing left in the shared
-array by one call leaks into the next.  This file is collected last on purpose.
+the same inputs bit for bit (the library's outputs are bitwise reproducible),
+so nothing left in the shared array by one call leaks into the next; and they
+must leave the device's free memory unchanged.  This file is collected last on
+purpose.
 """
 import numpy as np
 import pytest
 
 import workloads as W
-from parity import assert_grad_rows, assert_loss, assert_token_loss
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -50,27 +51,47 @@ def _outputs(zs, T):
 
 
 def test_static_entry_matches_workspace_entry_twice(P):
+    """Three static calls in a row (a large batch, a smaller one with another vocabulary
+    and mode, then the large one again, so a leftover of either call in the shared
+    array would show), each against the workspace entry point on the same inputs.
+    After one warm-up call of each case, the static calls change neither the device's
+    free memory nor torch's allocated bytes."""
     cases = [(W.packed(seed=21, num_traj=2, traj_len=4096), W.V_QWEN, 21, 0),
              (W.household(seed=22, num_traj=2, traj_len=2048), 50000, 22, 1)]
-    for b, V, seed, mode in cases:  # two calls in a row, second one smaller and different
+    prepared = []
+    for b, V, seed, mode in cases:
         assert b.num_tokens <= P.TURNOPD_STATIC_MAX_TOKENS
         zs, zt, msk, rot, w, y = _inputs(b, V, seed, mode)
         T = b.num_tokens
         ws = torch.empty(P.turnopd_loss_workspace_bytes(T), dtype=torch.uint8, device="cuda")
-        g_ref, tl_ref, l_ref, st_ref = _outputs(zs, T)
+        ref = _outputs(zs, T)
+        g_ref, tl_ref, l_ref, st_ref = ref
         P.turnopd_loss_fwd_bwd(zs, zt, V, rot, y, msk, w, mode, g_ref, 0, tl_ref, l_ref, ws, st_ref)
-        g, tl, l, st = _outputs(zs, T)
+        prepared.append((b, V, mode, (zs, zt, msk, rot, w, y), ref))
+    order = [0, 1, 0]
+    outs = [_outputs(prepared[c][3][0], prepared[c][0].num_tokens) for c in order]
+
+    def call(case, out):
+        b, V, mode, (zs, zt, msk, rot, w, y), _ = prepared[case]
+        g, tl, l, st = out
         P.turnopd_loss_fwd_bwd_static(zs, zt, V, rot, y, msk, w, mode, g, 0, tl, l, st)
-        torch.cuda.synchronize()
+
+    for c in range(len(cases)):   # warm-up: kernels of both cases loaded on the device
+        call(c, _outputs(prepared[c][3][0], prepared[c][0].num_tokens))
+    torch.cuda.synchronize()
+    free0, alloc0 = torch.cuda.mem_get_info()[0], torch.cuda.memory_allocated()
+    for c, out in zip(order, outs):
+        call(c, out)
+    torch.cuda.synchronize()
+    assert torch.cuda.mem_get_info()[0] == free0
+    assert torch.cuda.memory_allocated() == alloc0
+
+    for c, (g, tl, l, st) in zip(order, outs):
+        b, V, mode, (zs, zt, msk, rot, w, y), (g_ref, tl_ref, l_ref, st_ref) = prepared[c]
         assert st_ref.item() == 0 and st.item() == 0
-        tl_ref_np = tl_ref.cpu().numpy().astype(np.float64)
-        assert_token_loss(tl.cpu().numpy(), tl_ref_np, b.loss_mask)
-        assert_loss(l.item(), l_ref.item())
-        rows = np.arange(0, b.num_valid, max(1, b.num_valid // 64))
-        toks = np.nonzero(b.loss_mask)[0][rows]
-        extra = dict(ell=tl_ref_np[toks], w=w.cpu().numpy()[toks]) if mode == 1 else {}
-        assert_grad_rows(g[rows].float().cpu().numpy(), g_ref[rows].float().cpu().numpy(),
-                         bf16=True, **extra)
+        # the same kernels on the same inputs: the library's results are bitwise
+        # reproducible, so only the scratch's home differs
+        assert torch.equal(tl, tl_ref) and torch.equal(l, l_ref) and torch.equal(g, g_ref)
 
 
 def test_static_entry_rejects_oversized_batches(P):
