@@ -4,14 +4,15 @@ against the fp64 oracle.
 The selected ids are compared bit for bit (the selection is a decision on the
 bf16/fp32 teacher logits, taken exactly on both sides).  Per-token loss and
 total loss use the loss path's bounds; the gradient at the selected ids is
-within 1e-4 of the row's largest |g| (fp32 output) and the dense bf16 rows
-within 2 bf16 ulps or that bound.
+within 1e-4 of the row's largest |g| (fp32 output), and a dense gradient row
+holds exactly those fp32 values (rounded to nearest even when it is bf16) at
+the selected ids and zeros elsewhere.
 """
 import numpy as np
 import pytest
 
 import workloads as W
-from parity import assert_loss, assert_token_loss, bf16_ulp
+from parity import assert_loss, assert_token_loss
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -154,15 +155,13 @@ def test_dense_gradient_misaligned_stride_and_zero_flag(P, oracle, dtype):
     assert (ids[m] == -1).all() and (gk[m] == 0).all()
     dn = dense.float().cpu().numpy()
     assert (dn[:, V:] == 3.0).all()  # padding columns untouched
-    for t in np.nonzero(b.loss_mask)[0][:64]:
-        r = rot_np[t]
-        want = np.zeros(V)
-        want[rids[t]] = rg[t]
-        got = dn[r, :V]
-        tol = 1e-4 * np.abs(rg[t]).max()
-        if dtype == torch.bfloat16:
-            tol = np.maximum(tol, 2 * bf16_ulp(want))
-        assert (np.abs(got - want) <= tol + 1e-30).all()
+    # the dense row holds the sparse fp32 values (checked against the oracle above),
+    # rounded to nearest even in bf16, at the support ids and zeros elsewhere
+    gk_dense = torch.from_numpy(gk).to(dtype).float().numpy()
+    for t in np.nonzero(b.loss_mask)[0]:
+        want = np.zeros(V, np.float32)
+        want[ids[t]] = gk_dense[t]
+        assert np.array_equal(dn[rot_np[t], :V], want)
 
 
 def test_full_vocab_packed_sampled_rows_and_properties(P, oracle):

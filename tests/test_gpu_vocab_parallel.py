@@ -81,7 +81,8 @@ def test_virtual_ranks_match_single_call_and_oracle(P, oracle, cuts):
                                            subset=pick)
     assert_token_loss(tls[0][pick], tl_ref[pick])
     rows = rot_np[pick]
-    assert_grad_rows(grad.float().cpu().numpy()[rows], g_ref[rows], bf16=True)
+    assert_grad_rows(grad.float().cpu().numpy()[rows], g_ref[rows], bf16=True,
+                     zs=zs[torch.from_numpy(rows).cuda()], w=w.cpu().numpy()[pick], ell=tl_ref[pick])
 
 
 def test_fp32_unaligned_split_and_helper(P, oracle):
