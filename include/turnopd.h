@@ -456,6 +456,19 @@ turnopd_status turnopd_turn_stats(const float *token_loss, const int32_t *turn_i
 double turnopd_alpha_schedule(int64_t k, int64_t K, double s, double e);
 
 /*
+ * turnopd_turn_floor -- the turn-reliability floor of the internal blend,
+ * n_min = max(min_floor, ceil(min_frac * n_traj)) (hyper-parameter table,
+ * internal-blend group: min_floor = 8, min_frac = 0.15), to pass as n_min to
+ * turnopd_weights.  n_traj is the number of trajectories of the step's batch
+ * (all data-parallel ranks together, empty trajectories included), the
+ * population over which the survivor counts S_t are taken.  Host function.
+ * The ceiling is exact for decimal fractions: 0.07 * 100 gives 7, not 8.
+ * Returns -1 if n_traj < 0, min_floor < 0, min_frac is outside [0, 1] (or
+ * NaN), or the result exceeds INT32_MAX.
+ */
+int32_t turnopd_turn_floor(int64_t n_traj, int32_t min_floor, double min_frac);
+
+/*
  * turnopd_selftest_wait_timeout -- diagnostic of the device-side timeout path.
  * Every wait of the library's kernels on an mbarrier or a flag is a bounded poll
  * loop: when the limit runs out the kernel records TURNOPD_ERR_TIMEOUT in

@@ -21,7 +21,7 @@ __all__ = [
     "TURNOPD_FORCE_PORTABLE", "TURNOPD_MAX_TURNS",
     "turnopd_turn_counts", "turnopd_weights", "turnopd_weights_workspace_bytes",
     "turnopd_loss_fwd_bwd", "turnopd_loss_workspace_bytes", "turnopd_turn_stats",
-    "turnopd_alpha_schedule", "turnopd_status_string", "turnopd_loss_fwd_bwd_static",
+    "turnopd_alpha_schedule", "turnopd_turn_floor", "turnopd_status_string", "turnopd_loss_fwd_bwd_static",
     "turnopd_selftest_wait_timeout",
     "TURNOPD_STATIC_MAX_TOKENS", "turnopd_fused_lmhead_fwd_bwd", "turnopd_fused_workspace_bytes",
     "turnopd_topk_loss_fwd_bwd", "TURNOPD_TOPK_MAX", "TURNOPD_TOPK_MAX_VOCAB",
@@ -118,6 +118,8 @@ def load():
     lib.turnopd_fused_workspace_bytes.restype = sz
     lib.turnopd_alpha_schedule.argtypes = [i64, i64, f64, f64]
     lib.turnopd_alpha_schedule.restype = f64
+    lib.turnopd_turn_floor.argtypes = [i64, i32, f64]
+    lib.turnopd_turn_floor.restype = i32
     lib.turnopd_depth_default_params.restype = None
     lib.turnopd_vocab_stats_bytes.argtypes = [i64]
     lib.turnopd_vocab_stats_bytes.restype = sz
@@ -189,6 +191,16 @@ def turnopd_selftest_wait_timeout(poll_limit: int, dev_status, stream=None):
 
 def turnopd_alpha_schedule(k: int, K: int, s: float = 0.0, e: float = 1.0) -> float:
     return float(load().turnopd_alpha_schedule(int(k), int(K), float(s), float(e)))
+
+
+def turnopd_turn_floor(n_traj: int, min_floor: int = 8, min_frac: float = 0.15) -> int:
+    """n_min = max(min_floor, ceil(min_frac * n_traj)) for turnopd_weights; defaults
+    are the paper's internal-blend settings.  n_traj counts the step's trajectories
+    over all ranks."""
+    n = int(load().turnopd_turn_floor(int(n_traj), int(min_floor), float(min_frac)))
+    if n < 0:
+        raise ValueError("turnopd_turn_floor: n_traj and min_floor must be >= 0, min_frac in [0, 1]")
+    return n
 
 
 def turnopd_weights_workspace_bytes(num_traj: int, max_turns: int) -> int:

@@ -95,6 +95,19 @@ double turnopd_alpha_schedule(int64_t k, int64_t K, double s, double e)
     return a < 0.0 ? 0.0 : (a > 1.0 ? 1.0 : a);
 }
 
+int32_t turnopd_turn_floor(int64_t n_traj, int32_t min_floor, double min_frac)
+{
+    if (n_traj < 0 || min_floor < 0 || !(min_frac >= 0.0) || !(min_frac <= 1.0))
+        return -1;
+    // min_frac is usually a short decimal (0.15, 0.07) whose binary value lies a hair
+    // off it, so an exact integer product can land one ulp above the integer;
+    // the relative guard of 2^-40 keeps ceil() from stepping past it.
+    const double x = min_frac * (double)n_traj;
+    const double c = ceil(x - x * 0x1p-40);
+    const double n = c > (double)min_floor ? c : (double)min_floor;
+    return n > 2147483647.0 ? -1 : (int32_t)n;
+}
+
 turnopd_status turnopd_selftest_wait_timeout(uint32_t poll_limit, int32_t *dev_status, turnopd_stream_t stream)
 {
     if (!dev_status)

@@ -119,6 +119,27 @@ def test_alpha_schedule_and_status_strings(lib, oracle):
     assert P.turnopd_status_string(0) == "ok"
 
 
+def test_turn_floor_is_the_paper_rule_with_an_exact_ceiling(lib):
+    """n_min = max(floor, ceil(frac * n_traj)) (hyper-parameter table: floor 8,
+    frac 0.15), checked against exact rational arithmetic on the decimal frac."""
+    from fractions import Fraction
+
+    import paper_2607_05804_gb300 as P
+
+    for frac in ("0.15", "0.1", "0.3", "0.25", "0.07", "1", "0"):
+        for floor in (0, 8):
+            for n in list(range(0, 201)) + [1000, 4096, 65536, 10 ** 7]:
+                want = max(floor, math.ceil(Fraction(frac) * n))
+                assert P.turnopd_turn_floor(n, floor, float(frac)) == want, (frac, floor, n)
+    assert P.turnopd_turn_floor(64) == 10          # the paper's batch of 64 trajectories
+    assert P.turnopd_turn_floor(16) == 8           # household: the floor binds
+    assert 0.07 * 100 > 7 and P.turnopd_turn_floor(100, 0, 0.07) == 7
+    for bad in ((-1, 8, 0.15), (10, -1, 0.15), (10, 8, -0.1), (10, 8, 1.5), (10, 8, float("nan"))):
+        assert lib.turnopd_turn_floor(*bad) == -1
+    with pytest.raises(ValueError):
+        P.turnopd_turn_floor(-1)
+
+
 def test_topk_host_validation(lib):
     f = lib.turnopd_topk_loss_fwd_bwd
     ws_need = lib.turnopd_loss_workspace_bytes(64)
