@@ -3,7 +3,7 @@
 Each rank owns half of the trajectories of one batch, computes its count vector
 and weights with the fp64 oracle, sums the count vectors through
 paper_2607_05804_gb300.dp.global_counts, and reduces loss and turn statistics
-through dp.reduce_step.  The merged results must equal the single-process oracle
+through dp.reduce_step, which packs them into one all-reduce.  The merged results must equal the single-process oracle
 on the whole batch: weights and counts exactly, sums within fp64 rounding."""
 import os
 import socket
@@ -54,7 +54,15 @@ def _rank_main(rank, world, port, result_path):
         ts = torch.from_numpy(st["turn_sum"].copy())
         tc = torch.from_numpy(st["turn_cnt"].copy())
         sv = torch.from_numpy(st["turn_surv"].copy())
-        dp.reduce_step(L, ts, tc, sv)
+        calls = []
+        real = dist.all_reduce
+        dist.all_reduce = lambda *a, **k: (calls.append(1), real(*a, **k))[1]
+        try:
+            dp.reduce_step(L, ts, tc, sv)
+        finally:
+            dist.all_reduce = real
+        assert len(calls) == 1  # one packed collective after the step
+        assert tc.dtype == torch.int64 and sv.dtype == torch.int32
         parts = [None] * world
         dist.all_gather_object(parts, w)
         out[(scope, n_min)] = (np.concatenate(parts), L.item(), ts.numpy(), tc.numpy(), sv.numpy())
