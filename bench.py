@@ -659,7 +659,9 @@ def e2e_leg(args, step, zs, zt, grad, world, dist, device, R):
         dist.all_reduce(t, op=dist.ReduceOp.MAX)
         ms = float(t.item())
     return {"value": R * world * steps / (ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": 8, "steps": steps}
+            "d2h_bytes_per_step": 8, "steps": steps,
+            "d2h": "the loss only: the student-logit gradient stays on the device, where the "
+                   "backward pass through the student consumes it"}
 
 
 if __name__ == "__main__":
