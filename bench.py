@@ -36,7 +36,7 @@ sys.path.insert(0, ROOT)
 METRIC = "loss fwd+bwd tokens/s at V=151936 bf16 on 1 GB300; achieved HBM GB/s vs peak"
 UNIT = "tokens/s"
 # counts(2) + weights(1) + compaction(2) + row kernel + loss sum + stats(2); the full and
-# sampled modes add the helper grid that runs beside the cluster grid
+# sampled modes on bf16 logits add the helper grid that runs beside the cluster grid
 KERNELS_PER_STEP = 9
 ROW_KERNEL_SOURCES = ["paper_2607_05804_gb300/csrc/rowkl_cluster.cu",
                       "paper_2607_05804_gb300/csrc/loss_kernels.cu",
@@ -61,6 +61,8 @@ def parse():
     p.add_argument("--zero-masked", action="store_true",
                    help="dense layout with TURNOPD_ZERO_MASKED_GRAD: masked tokens' gradient rows written as zeros")
     p.add_argument("--fp32-grad", action="store_true", help="full/sampled modes: an fp32 gradient instead of bf16")
+    p.add_argument("--fp32-logits", action="store_true",
+                   help="full/sampled modes: fp32 logits instead of bf16 (the split-row kernel)")
     p.add_argument("--alpha", type=float, default=0.5)
     p.add_argument("--no-e2e", action="store_true")
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -184,7 +186,8 @@ def build_inputs(args, rank, device):
     V = W.V_QWEN
     dense = dense_layout(args)
     rows = b.num_tokens if dense else b.num_valid
-    zs, zt = W.make_logits(rows, V, "agent", torch.bfloat16, seed=1000 + rank, device=device)
+    zs, zt = W.make_logits(rows, V, "agent", torch.float32 if args.fp32_logits else torch.bfloat16,
+                           seed=1000 + rank, device=device)
     mode = TURNOPD_SAMPLED_TOKEN if args.mode == "sampled" else TURNOPD_FULL_VOCAB
     y = None
     if mode == TURNOPD_SAMPLED_TOKEN:
@@ -272,11 +275,12 @@ def cpu_baseline(b, zs, zt, V, alpha, mode, rows_override=0, budget_s=15.0, k_to
     done, spent, chunk = 0, 0.0, 512
     while done < limit and (rows_override or spent < budget_s):
         n = min(chunk, limit - done)
+        host = W.bf16_bits if zs.dtype == torch.bfloat16 else (lambda t: t.cpu().numpy())
         if dense:  # the supervised tokens' own rows
             sel = torch.from_numpy(valid[done:done + n]).to(zs.device)
-            zsn, ztn = W.bf16_bits(zs.index_select(0, sel)), W.bf16_bits(zt.index_select(0, sel))
+            zsn, ztn = host(zs.index_select(0, sel)), host(zt.index_select(0, sel))
         else:
-            zsn, ztn = W.bf16_bits(zs[done:done + n]), W.bf16_bits(zt[done:done + n])
+            zsn, ztn = host(zs[done:done + n]), host(zt[done:done + n])
         t0 = time.perf_counter()
         if k_top:
             oracle.topk_loss(zsn, ztn, V, np.ones(n, np.uint8), w[valid[done:done + n]], k_top)
@@ -495,6 +499,8 @@ def main():
     P.load()
     b, V, zs, zt, grad, step = build_inputs(args, rank, device)
     R = b.num_valid
+    if args.fp32_logits and (args.mode == "topk" or args.vocab_shards):
+        raise SystemExit("--fp32-logits times the full-vocabulary and sampled modes")
     if args.vocab_shards:
         if args.mode != "full" or dense_layout(args):
             raise SystemExit("--vocab-shards times the full-vocabulary mode on compact rows")
@@ -546,8 +552,8 @@ def main():
         # statistics pass (two logit rows read), gradient pass (read again, gradient written)
         bytes_per_row = 5 * V * 2
     else:
-        # two bf16 logit rows read + one gradient row written (bf16, or fp32)
-        bytes_per_row = 2 * V * 2 + V * (4 if args.fp32_grad else 2)
+        # two logit rows read (bf16, or fp32) + one gradient row written (bf16, or fp32)
+        bytes_per_row = 2 * V * (4 if args.fp32_logits else 2) + V * (4 if args.fp32_grad else 2)
     alg_bytes = R * bytes_per_row
     masked_rows = b.num_tokens - R
     if args.zero_masked:
@@ -569,7 +575,8 @@ def main():
         out = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32" if args.fp32_logits else "bf16",
+            "data": "synthetic",
             "config": {
                 "workload": f"{b.name}_V{V}", "tokens": b.num_tokens, "supervised_tokens": R,
                 "tokens_counted": "supervised (assistant) tokens", "vocab": V,
@@ -578,6 +585,7 @@ def main():
                 **({"zero_masked_grad": True, "masked_rows": masked_rows} if args.zero_masked else {}),
                 "grad_dtype": ("fp32 sparse (ids, values)" if args.mode == "topk"
                                else "fp32" if args.fp32_grad else "bf16"),
+                "logits_dtype": "fp32" if args.fp32_logits else "bf16",
                 "mode": args.mode, "alpha": args.alpha, "scope": "traj",
                 **({"k_top": args.k_top} if args.mode == "topk" else {}),
                 **({"vocab_shards": args.vocab_shards} if args.vocab_shards else {}),
@@ -591,17 +599,20 @@ def main():
                            if args.mode == "topk" else
                            f"vocabulary-parallel path, {args.vocab_shards} shards of one GPU "
                            "(shard stats + merge + shard gradients)" if args.vocab_shards else
+                           "turnopd_loss_fwd_bwd launch sequence (split-row kernel on clusters of 4 "
+                           "+ compaction + loss sum)" if args.fp32_logits else
                            "turnopd_loss_fwd_bwd launch sequence (cluster row kernel beside the helper grid "
                            "+ compaction + loss sum)"),
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "launch_ms": loss_avg_ms,
-                "traffic": (None if (args.vocab_shards or dense_layout(args))
+                "traffic": (None if (args.vocab_shards or dense_layout(args) or args.fp32_logits)
                             else committed_traffic(args.workload, R, "topk") if args.mode == "topk"
                             else committed_traffic(args.workload)),
             },
             # vocabulary shards: counts(2) + weights(1) + per shard the statistics call (compaction(2),
             # statistics) and the gradient call (compaction(2), gradient, loss sum) + merge + stats(2)
-            "gpu_launches": ((KERNELS_PER_STEP + (1 if args.zero_masked else 0) + (0 if args.mode == "topk" else 1))
+            "gpu_launches": ((KERNELS_PER_STEP + (1 if args.zero_masked else 0)
+                              + (0 if args.mode == "topk" or args.fp32_logits else 1))
                              if not args.vocab_shards
                              else 6 + 7 * args.vocab_shards) * args.steps,
             "clocks": clocks,

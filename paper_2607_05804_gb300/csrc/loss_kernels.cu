@@ -1,7 +1,8 @@
 // Per-token OPD loss and student-logit gradient: compaction of supervised
 // tokens, the portable one-CTA-per-row kernel, masked-row zero fill and the
 // fixed-order loss sum (sm_103a).  The cluster-resident row kernel used for
-// aligned bf16 rows lives in rowkl_cluster.cu.
+// aligned bf16 rows lives in rowkl_cluster.cu, the split-row kernel for
+// aligned fp32 rows in rowkl_split.cu.
 //
 // Per supervised token (Eq. opd-rkl), from one read of each logit row:
 //   m, S = sum exp(z - m) for both models by an online (rescaling) pass,
@@ -384,8 +385,9 @@ cudaError_t launch_loss(const LossArgs &a, const LossWorkspace &ws, cudaStream_t
     RowIn p{a.zs, a.zt, a.ld, a.vocab, a.row_of_token, a.sampled_ids, a.w, a.mode, a.grad,
             a.token_loss, ws.row_wl, ws.rows, ws.nvalid, a.status, 0, 0};
     bool done = false;
-    if (a.in_dtype == TURNOPD_BF16 && !(a.flags & TURNOPD_FORCE_PORTABLE)) {
-        e = launch_row_cluster(p, a.grad_dtype == TURNOPD_F32, stream, &done);
+    if (!(a.flags & TURNOPD_FORCE_PORTABLE)) {
+        e = a.in_dtype == TURNOPD_BF16 ? launch_row_cluster(p, a.grad_dtype == TURNOPD_F32, stream, &done)
+                                        : launch_row_split(p, a.grad_dtype == TURNOPD_F32, stream, &done);
         if (e != cudaSuccess)
             return e;
     }

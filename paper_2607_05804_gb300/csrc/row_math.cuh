@@ -1,7 +1,8 @@
-// Row-streaming helpers shared by the portable row kernel and the
-// vocabulary-parallel kernels: 16-byte vector loads widened to fp32, vector
-// stores of the gradient, and the online fold of logits into the student /
-// teacher accumulators (max, sum exp, sum exp ((z_s - z_t) - d)).
+// Row-streaming helpers shared by the row kernels and the vocabulary-parallel
+// kernels: 16-byte vector loads widened to fp32, vector stores of the
+// gradient, the online fold of logits into the student / teacher accumulators
+// (max, sum exp, sum exp ((z_s - z_t) - d)), and the fixed-order merge of
+// per-lane partials across a warp.
 #pragma once
 
 #include "common.cuh"
@@ -52,6 +53,43 @@ template <> __device__ __forceinline__ void store_vec<float, 8>(float *p, const 
 template <> __device__ __forceinline__ void store_vec<float, 4>(float *p, const float *g)
 {
     *reinterpret_cast<float4 *>(p) = make_float4(g[0], g[1], g[2], g[3]);
+}
+
+// Merge per-lane partial statistics across the first `width` lanes of a warp
+// (lanes beyond hold empty partials): exact max by butterfly, one rescale
+// exponential per lane, then butterfly sums.  Lane 0's result is used; its
+// association order is fixed, so every warp and CTA gets the same bits.
+template <int WIDTH, bool USE_D = true>
+__device__ __forceinline__ void lane_merge(Student &S, Teacher &T)
+{
+    float m = S.m, mt = T.m;
+#pragma unroll
+    for (int o = 1; o < WIDTH; o <<= 1) {
+        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
+        mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
+    }
+    // reference difference of the lowest lane holding the max
+    float d = 0.f;
+    if (USE_D) {
+        const unsigned own = __ballot_sync(0xffffffffu, S.m == m && m != -INFINITY);
+        const int src = own ? __ffs(own) - 1 : 0;
+        d = __shfl_sync(0xffffffffu, S.d, src);
+    }
+    const float f = m == -INFINITY ? 0.f : ex2((S.m - m) * kLog2e);
+    const float ft = mt == -INFINITY ? 0.f : ex2((T.m - mt) * kLog2e);
+    float s = S.s * f, a = (USE_D ? fmaf(S.s, S.d - d, S.a) : S.a) * f, t = T.s * ft;
+    if (S.m == -INFINITY)
+        s = 0.f, a = 0.f;
+    if (T.m == -INFINITY)
+        t = 0.f;
+#pragma unroll
+    for (int o = 1; o < WIDTH; o <<= 1) {
+        s += __shfl_xor_sync(0xffffffffu, s, o);
+        a += __shfl_xor_sync(0xffffffffu, a, o);
+        t += __shfl_xor_sync(0xffffffffu, t, o);
+    }
+    S = Student{m, s, a, d};
+    T = Teacher{mt, t};
 }
 
 // Fold n student/teacher values into the online accumulators.

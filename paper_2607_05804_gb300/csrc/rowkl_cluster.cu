@@ -36,6 +36,7 @@
 #include "kernels.h"
 #include "packed.cuh"
 #include "ptx.cuh"
+#include "row_math.cuh"
 
 namespace turnopd {
 namespace {
@@ -43,43 +44,6 @@ namespace {
 constexpr int kStages = 3;
 constexpr uint32_t kCopyChunk = 65536;       // bytes per bulk copy instruction
 constexpr uint32_t kWaitLimit = 1u << 22;    // mbarrier polls before giving up
-
-// Merge per-lane partial statistics across the first `width` lanes of a warp
-// (lanes beyond hold empty partials): exact max by butterfly, one rescale
-// exponential per lane, then butterfly sums.  Lane 0's result is used; its
-// association order is fixed, so every warp and CTA gets the same bits.
-template <int WIDTH, bool USE_D = true>
-__device__ __forceinline__ void lane_merge(Student &S, Teacher &T)
-{
-    float m = S.m, mt = T.m;
-#pragma unroll
-    for (int o = 1; o < WIDTH; o <<= 1) {
-        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-        mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
-    }
-    // reference difference of the lowest lane holding the max
-    float d = 0.f;
-    if (USE_D) {
-        const unsigned own = __ballot_sync(0xffffffffu, S.m == m && m != -INFINITY);
-        const int src = own ? __ffs(own) - 1 : 0;
-        d = __shfl_sync(0xffffffffu, S.d, src);
-    }
-    const float f = m == -INFINITY ? 0.f : ex2((S.m - m) * kLog2e);
-    const float ft = mt == -INFINITY ? 0.f : ex2((T.m - mt) * kLog2e);
-    float s = S.s * f, a = (USE_D ? fmaf(S.s, S.d - d, S.a) : S.a) * f, t = T.s * ft;
-    if (S.m == -INFINITY)
-        s = 0.f, a = 0.f;
-    if (T.m == -INFINITY)
-        t = 0.f;
-#pragma unroll
-    for (int o = 1; o < WIDTH; o <<= 1) {
-        s += __shfl_xor_sync(0xffffffffu, s, o);
-        a += __shfl_xor_sync(0xffffffffu, a, o);
-        t += __shfl_xor_sync(0xffffffffu, t, o);
-    }
-    S = Student{m, s, a, d};
-    T = Teacher{mt, t};
-}
 
 // Per-row constants the gradient pass needs (computed once per row).
 struct GradConst {

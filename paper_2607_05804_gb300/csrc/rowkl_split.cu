@@ -1,0 +1,516 @@
+// Split-row kernel for fp32 logit rows (sm_103a).
+//
+// One fp32 logit row of V = 151,936 values is 607,744 bytes per model, so the
+// two rows of a token (1.2 MB) fit no SM, and one row in flight per SM would
+// ask 185 MB of the 126 MB L2 for the gradient pass's second read.  A cluster
+// of kCS CTAs therefore shares every row: CTA c owns the c-th quarter of the
+// columns (its slice), and the 36 co-resident clusters keep 36 rows in flight.
+// (Even so, most second reads miss L2 under the full stream: about 1.5 times
+// the algorithmic bytes reach DRAM, which bounds this kernel near 0.7 of HBM.)
+//
+// Per CTA (persistent, one per SM, rows cid, cid + nclusters, ...):
+//   * a producer warp streams the slice, both models, through a ring of
+//     kSStages chunks with bulk asynchronous copies (completion on a "full"
+//     mbarrier; a chunk is refilled once every consumer warp has arrived on
+//     its "empty" mbarrier).  It does not stop at row boundaries, so HBM stays
+//     busy while rows are merged;
+//   * 15 consumer warps fold each chunk into per-thread online accumulators
+//     (max, S = sum exp(z - m) for both models, A = sum exp(z_s - m_s)
+//     ((z_s - z_t) - d) with d at the running student argmax), merge them
+//     across the CTA in a fixed lane order and push the CTA's 32-byte record
+//     to every CTA of the cluster (st.async into a record ring, completion on
+//     the receiver's mbarrier: no cluster barrier per row);
+//   * every CTA merges the kCS records in the same fixed order, so all use
+//     bit-identical LSE and KL (deterministic), then writes the gradient of its
+//     slice, g = w p_s ((z_s - z_t) - LSE_s + LSE_t - KL) (full vocabulary) or
+//     g = w l (e_y - p_s) (sampled token), from the slice read again -- from L2,
+//     where the stream left it moments before -- by the producer into a second
+//     ring, while the producer keeps streaming the next row's fresh chunks.
+// HBM traffic per row: each logit row read once, the gradient row written once.
+// Every wait is bounded: on timeout the kernel records TURNOPD_ERR_TIMEOUT,
+// stops waiting, lets its own copies land and returns.
+
+#include <algorithm>
+
+#include "common.cuh"
+#include "kernels.h"
+#include "packed.cuh"
+#include "ptx.cuh"
+#include "row_math.cuh"
+
+namespace turnopd {
+namespace {
+
+constexpr int kCS = 4;                          // CTAs per row
+constexpr int kNT = 480;                        // consumer threads (15 warps: with the producer,
+                                                // 16 warps, so up to 128 registers a thread)
+constexpr int kNW = kNT / 32;                   // consumer warps
+constexpr int kThreads = kNT + 32;              // + the producer warp
+constexpr int kChunkVec = 960;                  // float4 vectors per model per chunk (15 KB)
+constexpr int kVPT = kChunkVec / kNT;           // vectors of each model per thread and chunk: 2
+#ifndef TURNOPD_SPLIT_SSTAGES
+#define TURNOPD_SPLIT_SSTAGES 3
+#endif
+#ifndef TURNOPD_SPLIT_KEEP
+#define TURNOPD_SPLIT_KEEP 1
+#endif
+// Seven 30 KB stages in all.  Measured on the packed 8 x 4096 fp32 batch: 3 fresh
+// + 4 read-again stages 7.48 ms, 4 + 3 7.88 ms, 5 + 2 9.19 ms (most second reads
+// reach DRAM, so they want the deeper ring).
+constexpr int kSStages = TURNOPD_SPLIT_SSTAGES;  // fresh chunks in flight (from HBM)
+constexpr int kGStages = 7 - kSStages;          // chunks read again for the gradient
+// The fresh chunks are marked L2 evict-last, so that the gradient's second read
+// a few microseconds later finds more of them there; after that read the lines go
+// back to normal priority.  Forward-only calls (no second read) leave the
+// default priority.
+constexpr bool kKeep = TURNOPD_SPLIT_KEEP != 0;
+constexpr int kSlots = 4;                       // record ring
+constexpr uint32_t kWaitLimit = 1u << 22;       // mbarrier polls before giving up
+constexpr uint32_t kStageBytes = 2u * kChunkVec * 16u;
+constexpr int kBar = 1;                         // named barrier of the consumer warps
+static_assert(kVPT == 2, "the chunk loop holds two vectors of each model per thread");
+
+constexpr size_t kSmemBytes = (size_t)(kSStages + kGStages) * kStageBytes  // the two rings
+                              + kSlots * kCS * 8 * sizeof(float)             // records
+                              + (2 * kSStages + 2 * kGStages + kSlots) * sizeof(uint64_t)
+                              + kNW * 8 * sizeof(float)                      // per-warp partials
+                              + 2 * 8 * sizeof(float)                        // row constants, by row parity
+                              + 2 * 2 * sizeof(float);                       // sampled-token logits, by parity
+
+__device__ __forceinline__ float lane4(const float4 &v, int i)
+{
+    return i == 0 ? v.x : (i == 1 ? v.y : (i == 2 ? v.z : v.w));
+}
+
+// Gradient of one vector (4 columns) from the row constants c (set in
+// `constants` below): g = w p ((z_s - z_t) - d - cp), or w l (e_y - p) with the
+// w l term at column yi (-1: none).
+template <bool G32>
+__device__ __forceinline__ float4 grad4(const float4 &a, const float4 &b, const float *c, bool sampled, int yi)
+{
+    const float2 L2 = splat(kLog2e), NLW = splat(c[0]);
+    const float2 a01 = make_float2(a.x, a.y), a23 = make_float2(a.z, a.w);
+    const float2 p01 = ex2x2(ffma2(a01, L2, NLW)), p23 = ex2x2(ffma2(a23, L2, NLW));
+    float2 g01, g23;
+    if (!sampled) {
+        const float2 SG = splat(c[1]);
+        const float2 x01 = fsub2(a01, make_float2(b.x, b.y)), x23 = fsub2(a23, make_float2(b.z, b.w));
+        if (G32) {
+            const float2 ND = splat(c[2]), NCP = splat(c[3]);
+            g01 = fmul2(p01, fadd2(ffma2(x01, SG, ND), NCP));
+            g23 = fmul2(p23, fadd2(ffma2(x23, SG, ND), NCP));
+        } else {
+            const float2 NC = splat(c[4]);
+            g01 = fmul2(p01, ffma2(x01, SG, NC));
+            g23 = fmul2(p23, ffma2(x23, SG, NC));
+        }
+    } else {
+        const float2 SGL = splat(c[5]);
+        g01 = fmul2(p01, SGL);
+        g23 = fmul2(p23, SGL);
+        const float wl = c[6];
+        if (yi == 0) g01.x += wl;
+        if (yi == 1) g01.y += wl;
+        if (yi == 2) g23.x += wl;
+        if (yi == 3) g23.y += wl;
+    }
+    return make_float4(g01.x, g01.y, g23.x, g23.y);
+}
+
+template <bool G32>
+__global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_vec, int nvec)
+{
+    extern __shared__ __align__(128) unsigned char smem[];
+    __shared__ int s_dead;
+    float4 *sring = reinterpret_cast<float4 *>(smem);                       // [kSStages][2][kChunkVec]
+    float4 *gring = sring + (size_t)kSStages * 2 * kChunkVec;              // [kGStages][2][kChunkVec]
+    float *rec = reinterpret_cast<float *>(gring + (size_t)kGStages * 2 * kChunkVec);  // [kSlots][kCS][8]
+    uint64_t *sfull = reinterpret_cast<uint64_t *>(rec + kSlots * kCS * 8);  // [kSStages]
+    uint64_t *sempty = sfull + kSStages;                                     // [kSStages]
+    uint64_t *gfull = sempty + kSStages;                                     // [kGStages]
+    uint64_t *gempty = gfull + kGStages;                                     // [kGStages]
+    uint64_t *recv = gempty + kGStages;                                      // [kSlots]
+    float *red = reinterpret_cast<float *>(recv + kSlots);                   // [kNW][8]
+    float *bcs = red + kNW * 8;                                              // [2][8]
+    float *ysvs = bcs + 2 * 8;                                               // [2][2]
+
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const uint32_t rank = cluster_ctarank();
+    const int cid = (int)cluster_id(), ncl = (int)cluster_count();
+    const int v0 = (int)rank * slice_vec;  // first vector (4 floats) of my slice
+    const int my_vec = max(0, min(slice_vec, nvec - v0));
+    const int nchunk = (my_vec + kChunkVec - 1) / kChunkVec;
+    const bool do_grad = p.grad != nullptr;
+
+    if (tid == 0) {
+        s_dead = 0;
+        for (int s = 0; s < kSStages; ++s) {
+            mbar_init(&sfull[s], 1);
+            mbar_init(&sempty[s], kNW);
+        }
+        for (int s = 0; s < kGStages; ++s) {
+            mbar_init(&gfull[s], 1);
+            mbar_init(&gempty[s], kNW);
+        }
+        for (int s = 0; s < kSlots; ++s)
+            mbar_init(&recv[s], 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        for (int s = 0; s < kSlots; ++s)
+            mbar_arrive_expect_tx(&recv[s], kCS * 32u);  // first record of each slot
+    }
+    __syncthreads();
+    cluster_sync();  // peers' barriers are initialised before any record is sent
+
+    const int nv = *p.nvalid;
+    const int n = nv > cid ? (nv - cid + ncl - 1) / ncl : 0;  // same for the whole cluster
+    if (n == 0)
+        return;
+
+    const float *zs = static_cast<const float *>(p.zs);
+    const float *zt = static_cast<const float *>(p.zt);
+
+    auto dead = [&]() { return *(volatile int *)&s_dead != 0; };
+    auto wait_bar = [&](uint64_t *bar, uint32_t parity, bool cluster_scope) {
+        if (dead())
+            return;
+        for (uint32_t it = 0; it < kWaitLimit; ++it)
+            if (cluster_scope ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity))
+                return;
+        s_dead = 1;
+        set_status(p.status, TURNOPD_ERR_TIMEOUT);
+    };
+
+    if (warp == kNW) {
+        // ---------------------------------------------------------------- producer
+        // Chunk c of row k from HBM into the fresh ring, then chunk c of row k - 1
+        // again (from L2, where it has been since row k - 1 streamed it) into the
+        // gradient ring; a sampled-token row's gradient needs the student chunk only.
+        if (lane == 0) {
+            const uint64_t keep = evict_last_policy();
+            auto issue = [&](float4 *ring, uint64_t *fullb, int stages, uint32_t t, bool fresh) {
+                const int k = (int)(t / (uint32_t)nchunk), c = (int)(t % (uint32_t)nchunk);
+                const int4 m = p.rows[cid + k * ncl];
+                const int s = (int)(t % stages);
+                const size_t base = (size_t)m.y * (size_t)p.ld + (size_t)v0 * 4 + (size_t)c * kChunkVec * 4;
+                const uint32_t bytes = (uint32_t)min(kChunkVec, my_vec - c * kChunkVec) * 16u;
+                const bool teacher = fresh || m.z < 0;  // a sampled-token gradient needs the student only
+                float4 *dst = ring + (size_t)s * 2 * kChunkVec;
+                mbar_arrive_expect_tx(&fullb[s], (teacher ? 2u : 1u) * bytes);
+                if (kKeep && do_grad && fresh) {
+                    bulk_g2s(dst, zs + base, bytes, &fullb[s], keep);
+                    bulk_g2s(dst + kChunkVec, zt + base, bytes, &fullb[s], keep);
+                } else {
+                    bulk_g2s_keep(dst, zs + base, bytes, &fullb[s]);
+                    if (teacher)
+                        bulk_g2s_keep(dst + kChunkVec, zt + base, bytes, &fullb[s]);
+                }
+            };
+            // fresh chunks in row order; row k's chunks again once all of row k's
+            // fresh chunks are issued.  Neither stream waits for the other's ring.
+            const uint32_t total = (uint32_t)n * (uint32_t)nchunk;
+            const uint32_t total_g = do_grad ? total : 0u;
+            uint32_t ts = 0, tg = 0, idle = 0;
+            while ((ts < total || tg < total_g) && !dead()) {
+                bool moved = false;
+                if (ts < total) {
+                    const int s = (int)(ts % kSStages);
+                    if (ts < (uint32_t)kSStages || mbar_test_wait(&sempty[s], ((ts / kSStages) - 1) & 1)) {
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                        issue(sring, sfull, kSStages, ts++, true);
+                        moved = true;
+                    }
+                }
+                if (tg < total_g && ts >= (tg / (uint32_t)nchunk + 1u) * (uint32_t)nchunk) {
+                    const int s = (int)(tg % kGStages);
+                    if (tg < (uint32_t)kGStages || mbar_test_wait(&gempty[s], ((tg / kGStages) - 1) & 1)) {
+                        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                        issue(gring, gfull, kGStages, tg++, false);
+                        moved = true;
+                    }
+                }
+                if (moved) {
+                    idle = 0;
+                } else if (++idle >= 16 * kWaitLimit) {  // test_wait never suspends: more polls
+                    s_dead = 1;
+                    set_status(p.status, TURNOPD_ERR_TIMEOUT);
+                }
+            }
+            // after a timeout, let this CTA's own copies land before it exits
+            if (dead()) {
+                for (uint32_t u = ts > (uint32_t)kSStages ? ts - kSStages : 0; u < ts; ++u)
+                    for (uint32_t it = 0; it < kWaitLimit; ++it)
+                        if (mbar_try_wait(&sfull[u % kSStages], (u / kSStages) & 1))
+                            break;
+                for (uint32_t u = tg > (uint32_t)kGStages ? tg - kGStages : 0; u < tg; ++u)
+                    for (uint32_t it = 0; it < kWaitLimit; ++it)
+                        if (mbar_try_wait(&gfull[u % kGStages], (u / kGStages) & 1))
+                            break;
+            }
+        }
+        cluster_sync();
+        return;
+    }
+
+    // -------------------------------------------------------------------- consumers
+    // Per row: the statistics from the fresh chunks, the cluster merge, then the
+    // gradient from the chunks read again; meanwhile the producer streams the
+    // next row's fresh chunks.
+    auto bar_sync = [&]() { asm volatile("bar.sync %0, %1;" ::"r"(kBar), "r"(kNT) : "memory"); };
+    uint32_t ts = 0, tg = 0;
+    int4 m = p.rows[cid];
+
+    // row constants of row j from its cluster records (warp 0; identical in every CTA)
+    auto constants = [&](int j, const int4 &mj) {
+        const int slot = j % kSlots;
+        float *bc = bcs + (j & 1) * 8;
+        if (warp == 0) {
+            wait_bar(&recv[slot], (uint32_t)((j / kSlots) & 1), true);
+            const float *r = rec + slot * kCS * 8;
+            Student A = student_empty();
+            Teacher B = teacher_empty();
+            if (lane < kCS) {
+                const float4 x = *reinterpret_cast<const float4 *>(r + lane * 8);
+                const float4 z = *reinterpret_cast<const float4 *>(r + lane * 8 + 4);
+                A = Student{x.x, x.y, x.z, x.w};
+                B = Teacher{z.x, z.y};
+            }
+            lane_merge<kCS, true>(A, B);
+            if (lane == 0) {
+                const RowConst rc = row_const(A, B);
+                const int y = mj.z;
+                float e = rc.kl;
+                if (y >= 0) {
+                    const int owner = (y >> 2) / slice_vec;
+                    e = (r[owner * 8 + 6] - r[owner * 8 + 7]) - rc.dl;
+                }
+                // p |w| = 2^(z_s log2e - LSE_s log2e + log2 |w|); the sign of w enters
+                // through an fma by sg
+                const float wi = __int_as_float(mj.w), wl = wi * e;
+                const float sg = wi < 0.f ? -1.f : 1.f;
+                bc[0] = -rc.lse_s * kLog2e + log2f(fabsf(y < 0 ? wi : wl));  // nlw
+                bc[1] = sg;
+                bc[2] = -sg * rc.d;             // fp32 output: d and cp added separately
+                bc[3] = -sg * rc.cp;
+                bc[4] = -sg * (rc.d + rc.cp);   // bf16 output: one rounding of d + cp
+                bc[5] = wl > 0.f ? -1.f : 1.f;  // sampled: sign of -w l
+                bc[6] = wl;
+                if (rank == 0) {
+                    if (!isfinite(rc.lse_s) || !isfinite(rc.lse_t) || !isfinite(e))
+                        set_status(p.status, TURNOPD_ERR_NONFINITE);
+                    p.token_loss[mj.x] = e;
+                    p.row_wl[cid + j * ncl] = (double)wi * (double)e;
+                }
+                mbar_arrive_expect_tx(&recv[slot], kCS * 32u);  // re-arm for row j + kSlots
+            }
+        }
+        bar_sync();
+    };
+
+    // gradient of chunk c of row j, from the gradient ring's next stage
+    auto grad_chunk = [&](int j, const int4 &mj, int c) {
+        const int s = (int)(tg % kGStages);
+        wait_bar(&gfull[s], (tg / kGStages) & 1, false);
+        ++tg;
+        if (!dead()) {
+            const float *bc = bcs + (j & 1) * 8;
+            const float4 *ga = gring + (size_t)s * 2 * kChunkVec, *gb = ga + kChunkVec;
+            const size_t off = (size_t)mj.y * (size_t)p.ld + (size_t)v0 * 4;
+            const int cv = min(kChunkVec, my_vec - c * kChunkVec);
+            const int y = mj.z, yq = y >= 0 ? (y >> 2) - v0 : -1;
+#pragma unroll
+            for (int u = 0; u < kVPT; ++u) {
+                const int ql = tid + u * kNT;
+                if (ql < cv) {
+                    const int q = c * kChunkVec + ql;
+                    const float4 a = ga[ql], b = y < 0 ? gb[ql] : a;
+                    if (kKeep && (ql & 7) == 0) {  // one thread per 128-byte line of each model
+                        l2_evict_normal(zs + off + (size_t)q * 4);
+                        l2_evict_normal(zt + off + (size_t)q * 4);
+                    }
+                    const float4 g4 = grad4<G32>(a, b, bc, y >= 0, q == yq ? (y & 3) : -1);
+                    if (G32) {
+                        __stcs(reinterpret_cast<float4 *>(static_cast<float *>(p.grad) + off) + q, g4);
+                    } else {
+                        uint2 o;
+                        o.x = pack_bf16x2(g4.x, g4.y);
+                        o.y = pack_bf16x2(g4.z, g4.w);
+                        __stcs(reinterpret_cast<uint2 *>(static_cast<__nv_bfloat16 *>(p.grad) + off) + q, o);
+                    }
+                }
+            }
+        }
+        __syncwarp();
+        if (lane == 0)
+            mbar_arrive(&gempty[s]);
+    };
+
+    for (int k = 0; k < n; ++k) {
+        const int4 m_next = k + 1 < n ? p.rows[cid + (k + 1) * ncl] : m;  // a row ahead
+        float *ysv = ysvs + (k & 1) * 2;
+        const int y = m.z, yq = y >= 0 ? (y >> 2) - v0 : -1;
+
+        // statistics of row k's slice, in packed pairs: per chunk a max pass, one
+        // rescale if the maximum moved, then the sums
+        float ms = -INFINITY, mt = -INFINITY, dd = 0.f;
+        float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
+        for (int c = 0; c < nchunk; ++c) {
+            const int s = (int)(ts % kSStages);
+            wait_bar(&sfull[s], (ts / kSStages) & 1, false);
+            ++ts;
+            const float4 *cs = sring + (size_t)s * 2 * kChunkVec;
+            const float4 *ct = cs + kChunkVec;
+            const int cv = min(kChunkVec, my_vec - c * kChunkVec);
+            const bool v0ok = tid < cv, v1ok = tid + kNT < cv;
+            if (!dead() && v0ok) {
+                const float4 x0 = cs[tid], z0 = ct[tid];
+                const float4 x1 = v1ok ? cs[tid + kNT] : x0, z1 = v1ok ? ct[tid + kNT] : z0;
+                if (c * kChunkVec + tid == yq) {
+                    ysv[0] = lane4(x0, y & 3);
+                    ysv[1] = lane4(z0, y & 3);
+                }
+                if (v1ok && c * kChunkVec + tid + kNT == yq) {
+                    ysv[0] = lane4(x1, y & 3);
+                    ysv[1] = lane4(z1, y & 3);
+                }
+                // (x1, z1 repeat x0, z0 when the second vector is past the chunk: the
+                // maxima are unchanged and its sums are skipped)
+                const float cm = fmaxf(fmaxf(fmaxf(x0.x, x0.y), fmaxf(x0.z, x0.w)),
+                                       fmaxf(fmaxf(x1.x, x1.y), fmaxf(x1.z, x1.w)));
+                const float cmt = fmaxf(fmaxf(fmaxf(z0.x, z0.y), fmaxf(z0.z, z0.w)),
+                                        fmaxf(fmaxf(z1.x, z1.y), fmaxf(z1.z, z1.w)));
+                if (cm > ms) {
+                    // reference difference at the first element equal to the new maximum
+                    float xd = x0.x - z0.x;
+                    if (x0.x != cm) {
+                        xd = x0.y == cm ? x0.y - z0.y : x0.z == cm ? x0.z - z0.z : x0.w == cm ? x0.w - z0.w
+                           : x1.x == cm ? x1.x - z1.x : x1.y == cm ? x1.y - z1.y
+                           : x1.z == cm ? x1.z - z1.z : x1.w - z1.w;
+                    }
+                    const float2 f = splat(ex2((ms - cm) * kLog2e));
+                    A2 = fmul2(ffma2(S2, splat(dd - xd), A2), f);
+                    S2 = fmul2(S2, f);
+                    dd = xd;
+                    ms = cm;
+                }
+                if (cmt > mt) {
+                    T2 = fmul2(T2, splat(ex2((mt - cmt) * kLog2e)));
+                    mt = cmt;
+                }
+                const float2 L2 = splat(kLog2e), NS = splat(-ms * kLog2e), NTT = splat(-mt * kLog2e);
+                const float2 D = splat(dd);
+                const float4 xs[2] = {x0, x1}, zz[2] = {z0, z1};
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    if (u == 1 && !v1ok)
+                        break;
+                    const float2 a01 = make_float2(xs[u].x, xs[u].y), a23 = make_float2(xs[u].z, xs[u].w);
+                    const float2 b01 = make_float2(zz[u].x, zz[u].y), b23 = make_float2(zz[u].z, zz[u].w);
+                    const float2 e01 = ex2x2(ffma2(a01, L2, NS)), e23 = ex2x2(ffma2(a23, L2, NS));
+                    S2 = fadd2(S2, fadd2(e01, e23));
+                    A2 = ffma2(e01, fsub2(fsub2(a01, b01), D), A2);
+                    A2 = ffma2(e23, fsub2(fsub2(a23, b23), D), A2);
+                    T2 = fadd2(T2, fadd2(ex2x2(ffma2(b01, L2, NTT)), ex2x2(ffma2(b23, L2, NTT))));
+                }
+            }
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&sempty[s]);
+        }
+
+        // row k's partial -> record to every CTA of the cluster
+        Student S = ms == -INFINITY ? student_empty() : Student{ms, S2.x + S2.y, A2.x + A2.y, dd};
+        Teacher U = mt == -INFINITY ? teacher_empty() : Teacher{mt, T2.x + T2.y};
+        lane_merge<32, true>(S, U);
+        if (lane == 0) {
+            float *rw = red + warp * 8;
+            rw[0] = S.m, rw[1] = S.s, rw[2] = S.a, rw[3] = S.d, rw[4] = U.m, rw[5] = U.s;
+        }
+        bar_sync();
+        if (warp == 0) {
+            Student A = student_empty();
+            Teacher B = teacher_empty();
+            if (lane < kNW) {
+                const float *r = red + lane * 8;
+                A = Student{r[0], r[1], r[2], r[3]};
+                B = Teacher{r[4], r[5]};
+            }
+            lane_merge<kNW, true>(A, B);
+            A.m = __shfl_sync(0xffffffffu, A.m, 0);
+            A.s = __shfl_sync(0xffffffffu, A.s, 0);
+            A.a = __shfl_sync(0xffffffffu, A.a, 0);
+            A.d = __shfl_sync(0xffffffffu, A.d, 0);
+            B.m = __shfl_sync(0xffffffffu, B.m, 0);
+            B.s = __shfl_sync(0xffffffffu, B.s, 0);
+            if (lane < kCS) {
+                const bool mine = yq >= 0 && yq < my_vec;
+                const float ys = mine ? ysv[0] : 0.f, yt = mine ? ysv[1] : 0.f;
+                const int slot = k % kSlots;
+                const uint32_t ra = mapa(smem_u32(rec + (slot * kCS + (int)rank) * 8), (uint32_t)lane);
+                const uint32_t rbar = mapa(smem_u32(&recv[slot]), (uint32_t)lane);
+                st_async16(ra, rbar, make_float4(A.m, A.s, A.a, A.d));
+                st_async16(ra + 16, rbar, make_float4(B.m, B.s, ys, yt));
+            }
+        }
+        constants(k, m);
+        if (do_grad)
+            for (int c = 0; c < nchunk; ++c)
+                grad_chunk(k, m, c);
+        m = m_next;
+    }
+    cluster_sync();  // no CTA leaves while a peer may still address its shared memory
+}
+
+}  // namespace
+
+// fp32 logits, 16-byte aligned rows (V and ld multiples of 4): the split-row
+// kernel on as many clusters as are co-resident.  *used = false leaves the row
+// to the portable kernel.
+cudaError_t launch_row_split(const RowIn &p, bool fp32_grad, cudaStream_t stream, bool *used)
+{
+    *used = false;
+    auto al16 = [](const void *q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
+    if (p.vocab % 4 != 0 || p.ld % 4 != 0 || !al16(p.zs) || !al16(p.zt) || (p.grad && !al16(p.grad)))
+        return cudaSuccess;
+    if (p.vocab / 4 > (int64_t)0x7fffffff)
+        return cudaSuccess;
+    const int nvec = (int)(p.vocab / 4);
+    const int slice_vec = (nvec + kCS - 1) / kCS;
+    auto kern = fp32_grad ? k_row_split<true> : k_row_split<false>;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess)
+        return e;
+    if (dev >= 64)
+        return cudaErrorInvalidDevice;
+    static int grid_cache[64][2];
+    const int gi = fp32_grad ? 1 : 0;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = kCS;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.stream = stream;
+    if (grid_cache[dev][gi] == 0) {
+        if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
+            cudaSuccess)
+            return e;
+        cfg.gridDim = dim3(kCS);
+        int ncl = 0;
+        if ((e = cudaOccupancyMaxActiveClusters(&ncl, kern, &cfg)) != cudaSuccess)
+            return e;
+        if (ncl < 1)
+            return cudaErrorInvalidConfiguration;
+        grid_cache[dev][gi] = ncl;
+    }
+    cfg.gridDim = dim3(grid_cache[dev][gi] * kCS);
+    *used = true;
+    return cudaLaunchKernelEx(&cfg, kern, p, slice_vec, nvec);
+}
+
+}  // namespace turnopd

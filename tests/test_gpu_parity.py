@@ -105,9 +105,11 @@ def test_tiny_exhaustive(P, oracle, alpha, mode, flags):
 @pytest.mark.parametrize("V,ld", [(4099, 4104), (4099, 4099), (16384, 16384)])
 @pytest.mark.parametrize("gdt", ["bf16", "f32"])
 @pytest.mark.parametrize("flags", [0, FORCE_PORTABLE], ids=["default", "portable"])
-def test_packed_reduced_vocab(P, oracle, V, ld, gdt, flags):
+@pytest.mark.parametrize("idt", ["bf16", "f32"])
+def test_packed_reduced_vocab(P, oracle, V, ld, gdt, flags, idt):
     b = W.packed(seed=2, num_traj=4, traj_len=1024)
-    zs, zt = W.make_logits(b.num_tokens, V, "agent", torch.bfloat16, seed=3, device="cuda", ld=ld)
+    zs, zt = W.make_logits(b.num_tokens, V, "agent", torch.bfloat16 if idt == "bf16" else torch.float32,
+                           seed=3, device="cuda", ld=ld)
     run_chain(P, oracle, b, V, zs, zt, mode=0, alpha=0.5, flags=flags,
               grad_dtype=torch.bfloat16 if gdt == "bf16" else torch.float32)
 
@@ -167,6 +169,39 @@ def test_cluster_kernel_all_rows(P, oracle, V, mode, gdt):
     zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=12, device="cuda")
     run_chain(P, oracle, b, V, zs, zt, mode=mode, alpha=0.5, compact=True,
               grad_dtype=torch.bfloat16 if gdt == "bf16" else torch.float32)
+
+
+@pytest.mark.parametrize("V,ld", [(4100, 4100), (4100, 4104), (W.V_QWEN, W.V_QWEN), (262144, 262144)])
+@pytest.mark.parametrize("mode", [0, 1], ids=["full", "sampled"])
+@pytest.mark.parametrize("gdt", ["bf16", "f32"])
+def test_split_kernel_fp32_all_rows(P, oracle, V, ld, mode, gdt):
+    """fp32 logits through the split-row kernel on every row: clusters of 4 CTAs
+    share each row (ragged last slice at V = 4100, a ragged last chunk at
+    V = 151,936, whole chunks at 262,144), about 8 rows per cluster so the chunk
+    ring wraps across rows, and padding columns beyond V never read."""
+    b = W.packed(seed=11, num_traj=2, traj_len=256)
+    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.float32, seed=12, device="cuda", ld=ld)
+    _, grad = run_chain(P, oracle, b, V, zs, zt, mode=mode, alpha=0.5, compact=True,
+                        grad_dtype=torch.bfloat16 if gdt == "bf16" else torch.float32)
+    if ld > V:
+        assert (grad[:, V:].float() == 7.0).all()
+
+
+@pytest.mark.parametrize("n_sup", [1, 5])
+def test_split_kernel_fewer_rows_than_clusters(P, oracle, n_sup):
+    """fp32 rows at the full vocabulary with fewer rows than clusters: most clusters
+    have no row and leave at once."""
+    T = 40
+    turn_id = np.full(T, -1, np.int32)
+    mask = np.zeros(T, np.uint8)
+    idx = np.linspace(3, T - 2, n_sup).astype(int)
+    mask[idx] = 1
+    turn_id[idx] = np.arange(n_sup) % 3
+    b = W.Batch("few", turn_id, mask, np.array([0, T], np.int64), 3)
+    zs, zt = W.make_logits(b.num_valid, FULL_V, "agent", torch.float32, seed=60 + n_sup, device="cuda")
+    for mode in (0, 1):
+        run_chain(P, oracle, b, FULL_V, zs, zt, mode=mode, alpha=0.5, compact=True,
+                  grad_dtype=torch.float32)
 
 
 @pytest.mark.parametrize("V", [50000, W.V_QWEN])
