@@ -40,7 +40,9 @@ UNIT = "tokens/s"
 KERNELS_PER_STEP = 9
 ROW_KERNEL_SOURCES = ["paper_2607_05804_gb300/csrc/rowkl_cluster.cu",
                       "paper_2607_05804_gb300/csrc/loss_kernels.cu",
-                      "paper_2607_05804_gb300/csrc/common.cuh"]
+                      "paper_2607_05804_gb300/csrc/common.cuh",
+                      "paper_2607_05804_gb300/csrc/row_math.cuh",
+                      "paper_2607_05804_gb300/csrc/packed.cuh"]
 
 
 def parse():

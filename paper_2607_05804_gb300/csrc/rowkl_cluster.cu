@@ -656,9 +656,22 @@ constexpr int kSmallRowVec = 7168;  // up to this many vectors per row: 256-thre
 // clusters of 16), about 0.9 for 1563 (V = 100,000 / 200,000); linear between.
 double helper_rate(int slice_vec)
 {
+#ifdef TURNOPD_HELPER_RATE
+    (void)slice_vec;
+    return TURNOPD_HELPER_RATE;
+#else
     const double r = 0.61 + (2048 - slice_vec) * 0.0006;
     return r < 0.61 ? 0.61 : (r > 1.0 ? 1.0 : r);
+#endif
 }
+// The helper grid beside the clusters: CTAs of kSideThreads threads, kSideBlocks per free SM.
+#ifndef TURNOPD_HELPER_THREADS
+#define TURNOPD_HELPER_THREADS 512
+#endif
+#ifndef TURNOPD_HELPER_BLOCKS
+#define TURNOPD_HELPER_BLOCKS 1
+#endif
+constexpr int kSideThreads = TURNOPD_HELPER_THREADS, kSideBlocks = TURNOPD_HELPER_BLOCKS;
 
 size_t cluster_smem_bytes(int slice_vec, int cs)
 {
@@ -733,10 +746,10 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
     ha[0].val.programmaticStreamSerializationAllowed = 1;
     hc.attrs = ha;
     hc.numAttrs = 1;
-    hc.gridDim = dim3(free_sm);
-    hc.blockDim = dim3(kHelpThreads);
+    hc.gridDim = dim3(free_sm * kSideBlocks);
+    hc.blockDim = dim3(kSideThreads);
     hc.stream = stream;
-    return cudaLaunchKernelEx(&hc, k_row_helper<G32>, pl);
+    return cudaLaunchKernelEx(&hc, k_row_helper<G32, kSideThreads, kSideBlocks>, pl);
 }
 
 }  // namespace
