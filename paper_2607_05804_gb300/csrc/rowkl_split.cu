@@ -5,8 +5,10 @@
 // ask 185 MB of the 126 MB L2 for the gradient pass's second read.  A cluster
 // of kCS CTAs therefore shares every row: CTA c owns the c-th quarter of the
 // columns (its slice), and the 36 co-resident clusters keep 36 rows in flight.
-// (Even so, most second reads miss L2 under the full stream: about 1.5 times
-// the algorithmic bytes reach DRAM, which bounds this kernel near 0.7 of HBM.)
+// The gradient's second read of a chunk follows its first within one row's
+// statistics, so it mostly hits L2 (DRAM traffic is about 1.04 times the
+// algorithmic bytes); the kernel is bound by each row's sequence of
+// statistics, cluster exchange and gradient.
 //
 // Per CTA (persistent, one per SM, rows cid, cid + nclusters, ...):
 //   * a producer warp streams the slice, both models, through a ring of
@@ -25,7 +27,9 @@
 //     slice, g = w p_s ((z_s - z_t) - LSE_s + LSE_t - KL) (full vocabulary) or
 //     g = w l (e_y - p_s) (sampled token), from the slice read again -- from L2,
 //     where the stream left it moments before -- by the producer into a second
-//     ring, while the producer keeps streaming the next row's fresh chunks.
+//     ring, while the producer keeps streaming the next row's fresh chunks.  A
+//     row's gradient waits until the next row's first fresh chunk is folded, so
+//     the cluster exchange completes meanwhile.
 // HBM traffic per row: each logit row read once, the gradient row written once.
 // Every wait is bounded: on timeout the kernel records TURNOPD_ERR_TIMEOUT,
 // stops waiting, lets its own copies land and returns.
@@ -41,7 +45,10 @@
 namespace turnopd {
 namespace {
 
-constexpr int kCS = 4;                          // CTAs per row
+#ifndef TURNOPD_SPLIT_CS
+#define TURNOPD_SPLIT_CS 4
+#endif
+constexpr int kCS = TURNOPD_SPLIT_CS;           // CTAs per row
 constexpr int kNT = 480;                        // consumer threads (15 warps: with the producer,
                                                 // 16 warps, so up to 128 registers a thread)
 constexpr int kNW = kNT / 32;                   // consumer warps
@@ -55,8 +62,7 @@ constexpr int kVPT = kChunkVec / kNT;           // vectors of each model per thr
 #define TURNOPD_SPLIT_KEEP 1
 #endif
 // Seven 30 KB stages in all.  Measured on the packed 8 x 4096 fp32 batch: 3 fresh
-// + 4 read-again stages 7.48 ms, 4 + 3 7.88 ms, 5 + 2 9.19 ms (most second reads
-// reach DRAM, so they want the deeper ring).
+// + 4 read-again stages 7.48 ms, 4 + 3 8.12 ms.
 constexpr int kSStages = TURNOPD_SPLIT_SSTAGES;  // fresh chunks in flight (from HBM)
 constexpr int kGStages = 7 - kSStages;          // chunks read again for the gradient
 // The fresh chunks are marked L2 evict-last, so that the gradient's second read
@@ -64,6 +70,12 @@ constexpr int kGStages = 7 - kSStages;          // chunks read again for the gra
 // back to normal priority.  Forward-only calls (no second read) leave the
 // default priority.
 constexpr bool kKeep = TURNOPD_SPLIT_KEEP != 0;
+// Row k - 1's constants and gradient wait until this many fresh chunks of row k are
+// folded, so its cluster records arrive meanwhile (0: right after its own merge).
+#ifndef TURNOPD_SPLIT_LAG
+#define TURNOPD_SPLIT_LAG 1
+#endif
+constexpr int kLag = TURNOPD_SPLIT_LAG;
 constexpr int kSlots = 4;                       // record ring
 constexpr uint32_t kWaitLimit = 1u << 22;       // mbarrier polls before giving up
 constexpr uint32_t kStageBytes = 2u * kChunkVec * 16u;
@@ -345,16 +357,30 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
             mbar_arrive(&gempty[s]);
     };
 
-    for (int k = 0; k < n; ++k) {
+    int4 m_prev = m;
+    for (int k = 0; k <= n; ++k) {
+        const bool have = k < n, prev = k > 0;
         const int4 m_next = k + 1 < n ? p.rows[cid + (k + 1) * ncl] : m;  // a row ahead
         float *ysv = ysvs + (k & 1) * 2;
         const int y = m.z, yq = y >= 0 ? (y >> 2) - v0 : -1;
+        // row k - 1's constants and gradient, once kLag fresh chunks of row k have been
+        // folded: its cluster records are in flight meanwhile
+        bool prev_done = !prev;
+        auto finish_prev = [&]() {
+            constants(k - 1, m_prev);
+            if (do_grad)
+                for (int c = 0; c < nchunk; ++c)
+                    grad_chunk(k - 1, m_prev, c);
+            prev_done = true;
+        };
 
         // statistics of row k's slice, in packed pairs: per chunk a max pass, one
         // rescale if the maximum moved, then the sums
         float ms = -INFINITY, mt = -INFINITY, dd = 0.f;
         float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
-        for (int c = 0; c < nchunk; ++c) {
+        for (int c = 0; c < (have ? nchunk : 0); ++c) {
+            if (!prev_done && c == kLag)
+                finish_prev();
             const int s = (int)(ts % kSStages);
             wait_bar(&sfull[s], (ts / kSStages) & 1, false);
             ++ts;
@@ -417,6 +443,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
             if (lane == 0)
                 mbar_arrive(&sempty[s]);
         }
+        if (!prev_done)
+            finish_prev();
+        if (!have)
+            break;
 
         // row k's partial -> record to every CTA of the cluster
         Student S = ms == -INFINITY ? student_empty() : Student{ms, S2.x + S2.y, A2.x + A2.y, dd};
@@ -452,10 +482,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
                 st_async16(ra + 16, rbar, make_float4(B.m, B.s, ys, yt));
             }
         }
-        constants(k, m);
-        if (do_grad)
-            for (int c = 0; c < nchunk; ++c)
-                grad_chunk(k, m, c);
+        m_prev = m;
         m = m_next;
     }
     cluster_sync();  // no CTA leaves while a peer may still address its shared memory
@@ -499,6 +526,8 @@ cudaError_t launch_row_split(const RowIn &p, bool fp32_grad, cudaStream_t stream
     if (grid_cache[dev][gi] == 0) {
         if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
             cudaSuccess)
+            return e;
+        if (kCS > 8 && (e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) != cudaSuccess)
             return e;
         cfg.gridDim = dim3(kCS);
         int ncl = 0;

@@ -187,6 +187,22 @@ def test_split_kernel_fp32_all_rows(P, oracle, V, ld, mode, gdt):
         assert (grad[:, V:].float() == 7.0).all()
 
 
+@pytest.mark.parametrize("ld", [151937, 151944])
+@pytest.mark.parametrize("idt", ["bf16", "f32"])
+def test_odd_vocabulary_full_size(P, oracle, ld, idt):
+    """V = 151,937 (not a multiple of 8 or 4) at the full size, with a row stride that
+    breaks 16-byte alignment and one padded to a multiple of 8: every row through the
+    kernel these shapes take, the padding columns of the gradient never written."""
+    b = W.packed(seed=31, num_traj=1, traj_len=256)
+    V = 151937
+    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16 if idt == "bf16" else torch.float32,
+                           seed=32, device="cuda", ld=ld)
+    for mode in (0, 1):
+        _, grad = run_chain(P, oracle, b, V, zs, zt, mode=mode, alpha=0.5, compact=True)
+        if ld > V:
+            assert (grad[:, V:].float() == 7.0).all()
+
+
 @pytest.mark.parametrize("n_sup", [1, 5])
 def test_split_kernel_fewer_rows_than_clusters(P, oracle, n_sup):
     """fp32 rows at the full vocabulary with fewer rows than clusters: most clusters
