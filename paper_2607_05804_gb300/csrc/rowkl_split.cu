@@ -6,7 +6,7 @@
 // of kCS CTAs therefore shares every row: CTA c owns the c-th quarter of the
 // columns (its slice), and the 36 co-resident clusters keep 36 rows in flight.
 // The gradient's second read of a chunk follows its first within one row's
-// statistics, so it mostly hits L2 (DRAM traffic is about 1.04 times the
+// statistics, so it mostly hits L2 (DRAM traffic is about 1.05 times the
 // algorithmic bytes); the kernel is bound by each row's sequence of
 // statistics, cluster exchange and gradient.
 //
