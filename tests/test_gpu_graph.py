@@ -1,6 +1,7 @@
 """One loss step captured in a CUDA graph and replayed gives the same bits as the
-stream-ordered call (weights, both row grids with the helper's programmatic launch,
-the loss sum and the turn statistics)."""
+stream-ordered call (weights, both row grids with the helper's programmatic launch
+-- or, for fp32 logits, the split-row kernel's clusters -- the loss sum and the
+turn statistics)."""
 import pytest
 
 import workloads as W
@@ -9,8 +10,9 @@ torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
 
 
+@pytest.mark.parametrize("dtype", ["bf16", "f32"])
 @pytest.mark.parametrize("mode", [0, 1], ids=["full", "sampled"])
-def test_step_in_a_cuda_graph_matches_eager(mode):
+def test_step_in_a_cuda_graph_matches_eager(mode, dtype):
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     import paper_2607_05804_gb300 as P
@@ -19,7 +21,8 @@ def test_step_in_a_cuda_graph_matches_eager(mode):
     P.load()
     b = W.packed(seed=5, num_traj=2, traj_len=1024)
     V = W.V_QWEN
-    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=5, device="cuda")
+    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16 if dtype == "bf16" else torch.float32,
+                           seed=5, device="cuda")
     tid, msk, off, rot = to_device(b, "cuda", compact=True)
     y = None
     if mode == 1:
