@@ -114,7 +114,8 @@ turnopd_status turnopd_turn_counts(const int32_t *turn_id, const uint8_t *loss_m
  * scope = TURNOPD_SCOPE_BATCH (one token mean over the batch):
  *     w_i = (1 - alpha) / N + alpha / (S n_bt),  N = sum C_t, S = sum S_t.
  * n_min > 0 enables the turn-reliability floor (hyper-parameter table:
- * n_min = max(floor, ceil(frac * n_traj)), computed by the caller): turn index
+ * n_min = max(floor, ceil(frac * n_traj)), computed by the caller, e.g. with
+ * turnopd_turn_floor): turn index
  * t is reliable iff S_t >= n_min; tokens of unreliable turns keep the token
  * weight (1/N_b, resp. 1/N), the reliable non-empty turns share the remaining
  * mass equally; with no reliable turn w_turn = w_traj.  n_min <= 0: no floor.
@@ -169,6 +170,14 @@ size_t turnopd_weights_workspace_bytes(int32_t num_traj, int32_t max_turns);
  * Device errors: TURNOPD_ERR_TOKEN_RANGE (row or sampled id; token skipped,
  *   l_i = 0), TURNOPD_ERR_NONFINITE (non-finite LSE or l_i).
  * Precision: fp32 arithmetic on exact fp32/bf16 inputs, fp64 loss sum.
+ * Kernels (the results agree within the tolerances above whichever runs):
+ *   bf16 logits, vocab and ld multiples of 8, 16-byte aligned arrays: row
+ *     clusters of 8 CTAs beside a helper grid on the remaining SMs;
+ *   fp32 logits, vocab and ld multiples of 4, 16-byte aligned arrays: the
+ *     split-row kernel (clusters of 4 CTAs per row), which marks its first
+ *     read of each logit chunk L2 evict-last and returns the lines to normal
+ *     priority after the gradient's second read;
+ *   any other shape: one CTA per row.
  */
 turnopd_status turnopd_loss_fwd_bwd(const void *z_student, const void *z_teacher,
                                     int32_t in_dtype, int64_t ld, int64_t vocab,
