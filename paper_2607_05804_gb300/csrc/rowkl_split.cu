@@ -5,10 +5,8 @@
 // ask 185 MB of the 126 MB L2 for the gradient pass's second read.  A cluster
 // of kCS CTAs therefore shares every row: CTA c owns the c-th quarter of the
 // columns (its slice), and the 36 co-resident clusters keep 36 rows in flight.
-// The gradient's second read of a chunk follows its first within one row's
-// statistics, so it mostly hits L2 (DRAM traffic is about 1.05 times the
-// algorithmic bytes); the kernel is bound by each row's sequence of
-// statistics, cluster exchange and gradient.
+// The gradient's second read of a chunk follows its first within about one
+// row's statistics, so it mostly hits L2.
 //
 // Per CTA (persistent, one per SM, rows cid, cid + nclusters, ...):
 //   * a producer warp streams the slice, both models, through a ring of
@@ -16,7 +14,8 @@
 //     mbarrier; a chunk is refilled once every consumer warp has arrived on
 //     its "empty" mbarrier).  It does not stop at row boundaries, so HBM stays
 //     busy while rows are merged;
-//   * 15 consumer warps fold each chunk into per-thread online accumulators
+//   * two groups of 8 consumer warps take the cluster's rows in turn; each
+//     folds its row's chunks into per-thread online accumulators
 //     (max, S = sum exp(z - m) for both models, A = sum exp(z_s - m_s)
 //     ((z_s - z_t) - d) with d at the running student argmax), merge them
 //     across the CTA in a fixed lane order and push the CTA's 32-byte record
@@ -27,9 +26,8 @@
 //     slice, g = w p_s ((z_s - z_t) - LSE_s + LSE_t - KL) (full vocabulary) or
 //     g = w l (e_y - p_s) (sampled token), from the slice read again -- from L2,
 //     where the stream left it moments before -- by the producer into a second
-//     ring, while the producer keeps streaming the next row's fresh chunks.  A
-//     row's gradient waits until the next row's first fresh chunk is folded, so
-//     the cluster exchange completes meanwhile.
+//     ring.  While one group exchanges records and writes its gradient, the
+//     other folds the next row's fresh chunks, so the HBM stream does not pause.
 // HBM traffic per row: each logit row read once, the gradient row written once.
 // Every wait is bounded: on timeout the kernel records TURNOPD_ERR_TIMEOUT,
 // stops waiting, lets its own copies land and returns.
@@ -49,20 +47,20 @@ namespace {
 #define TURNOPD_SPLIT_CS 4
 #endif
 constexpr int kCS = TURNOPD_SPLIT_CS;           // CTAs per row
-constexpr int kNT = 480;                        // consumer threads (15 warps: with the producer,
-                                                // 16 warps, so up to 128 registers a thread)
-constexpr int kNW = kNT / 32;                   // consumer warps
-constexpr int kThreads = kNT + 32;              // + the producer warp
-constexpr int kChunkVec = 960;                  // float4 vectors per model per chunk (15 KB)
-constexpr int kVPT = kChunkVec / kNT;           // vectors of each model per thread and chunk: 2
+constexpr int kG = 2;                           // row groups per CTA (alternate rows)
+constexpr int kNT = 256;                        // threads per group
+constexpr int kNWG = kNT / 32;                  // warps per group
+constexpr int kThreads = kG * kNT + 32;         // + the producer warp (17 warps: up to 96 registers)
+constexpr int kChunkVec = 4 * kNT;              // float4 vectors per model per chunk (16 KB)
 #ifndef TURNOPD_SPLIT_SSTAGES
 #define TURNOPD_SPLIT_SSTAGES 3
 #endif
 #ifndef TURNOPD_SPLIT_KEEP
 #define TURNOPD_SPLIT_KEEP 1
 #endif
-// Seven 30 KB stages in all.  Measured on the packed 8 x 4096 fp32 batch: 3 fresh
-// + 4 read-again stages 7.48 ms, 4 + 3 8.12 ms.
+// Seven 32 KB stages in all, split between the fresh chunks and the chunks read
+// again.  Measured on the packed 8 x 4096 fp32 batch: 3 fresh + 4 read-again
+// stages 7.01 ms, 2 + 5 7.62 ms, 4 + 3 7.88 ms.
 constexpr int kSStages = TURNOPD_SPLIT_SSTAGES;  // fresh chunks in flight (from HBM)
 constexpr int kGStages = 7 - kSStages;          // chunks read again for the gradient
 // The fresh chunks are marked L2 evict-last, so that the gradient's second read
@@ -70,24 +68,17 @@ constexpr int kGStages = 7 - kSStages;          // chunks read again for the gra
 // back to normal priority.  Forward-only calls (no second read) leave the
 // default priority.
 constexpr bool kKeep = TURNOPD_SPLIT_KEEP != 0;
-// Row k - 1's constants and gradient wait until this many fresh chunks of row k are
-// folded, so its cluster records arrive meanwhile (0: right after its own merge).
-#ifndef TURNOPD_SPLIT_LAG
-#define TURNOPD_SPLIT_LAG 1
-#endif
-constexpr int kLag = TURNOPD_SPLIT_LAG;
-constexpr int kSlots = 4;                       // record ring
+constexpr int kSlots = 2 * kG;                  // record ring
 constexpr uint32_t kWaitLimit = 1u << 22;       // mbarrier polls before giving up
 constexpr uint32_t kStageBytes = 2u * kChunkVec * 16u;
-constexpr int kBar = 1;                         // named barrier of the consumer warps
-static_assert(kVPT == 2, "the chunk loop holds two vectors of each model per thread");
 
 constexpr size_t kSmemBytes = (size_t)(kSStages + kGStages) * kStageBytes  // the two rings
                               + kSlots * kCS * 8 * sizeof(float)             // records
                               + (2 * kSStages + 2 * kGStages + kSlots) * sizeof(uint64_t)
-                              + kNW * 8 * sizeof(float)                      // per-warp partials
-                              + 2 * 8 * sizeof(float)                        // row constants, by row parity
-                              + 2 * 2 * sizeof(float);                       // sampled-token logits, by parity
+                              + (kSStages + kGStages) * sizeof(uint32_t)     // chunk held by each stage
+                              + kG * kNWG * 8 * sizeof(float)                // per-warp partials
+                              + kG * 8 * sizeof(float)                       // row constants
+                              + kG * 2 * sizeof(float);                      // sampled-token logits
 
 __device__ __forceinline__ float lane4(const float4 &v, int i)
 {
@@ -142,9 +133,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
     uint64_t *gfull = sempty + kSStages;                                     // [kGStages]
     uint64_t *gempty = gfull + kGStages;                                     // [kGStages]
     uint64_t *recv = gempty + kGStages;                                      // [kSlots]
-    float *red = reinterpret_cast<float *>(recv + kSlots);                   // [kNW][8]
-    float *bcs = red + kNW * 8;                                              // [2][8]
-    float *ysvs = bcs + 2 * 8;                                               // [2][2]
+    uint32_t *stag = reinterpret_cast<uint32_t *>(recv + kSlots);            // [kSStages]
+    uint32_t *gtag = stag + kSStages;                                        // [kGStages]
+    float *reds = reinterpret_cast<float *>(gtag + kGStages);                // [kG][kNWG][8]
+    float *bcs = reds + kG * kNWG * 8;                                       // [kG][8]
+    float *ysvs = bcs + kG * 8;                                              // [kG][2]
 
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const uint32_t rank = cluster_ctarank();
@@ -158,11 +151,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
         s_dead = 0;
         for (int s = 0; s < kSStages; ++s) {
             mbar_init(&sfull[s], 1);
-            mbar_init(&sempty[s], kNW);
+            mbar_init(&sempty[s], kNWG);
+            stag[s] = 0xffffffffu;
         }
         for (int s = 0; s < kGStages; ++s) {
             mbar_init(&gfull[s], 1);
-            mbar_init(&gempty[s], kNW);
+            mbar_init(&gempty[s], kNWG);
+            gtag[s] = 0xffffffffu;
         }
         for (int s = 0; s < kSlots; ++s)
             mbar_init(&recv[s], 1);
@@ -183,24 +178,24 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
     const float *zt = static_cast<const float *>(p.zt);
 
     auto dead = [&]() { return *(volatile int *)&s_dead != 0; };
+    auto give_up = [&]() {
+        s_dead = 1;
+        set_status(p.status, TURNOPD_ERR_TIMEOUT);
+    };
     auto wait_bar = [&](uint64_t *bar, uint32_t parity, bool cluster_scope) {
         if (dead())
             return;
         for (uint32_t it = 0; it < kWaitLimit; ++it)
             if (cluster_scope ? mbar_try_wait_cluster(bar, parity) : mbar_try_wait(bar, parity))
                 return;
-        s_dead = 1;
-        set_status(p.status, TURNOPD_ERR_TIMEOUT);
+        give_up();
     };
 
-    if (warp == kNW) {
+    if (warp == kG * kNWG) {
         // ---------------------------------------------------------------- producer
-        // Chunk c of row k from HBM into the fresh ring, then chunk c of row k - 1
-        // again (from L2, where it has been since row k - 1 streamed it) into the
-        // gradient ring; a sampled-token row's gradient needs the student chunk only.
         if (lane == 0) {
             const uint64_t keep = evict_last_policy();
-            auto issue = [&](float4 *ring, uint64_t *fullb, int stages, uint32_t t, bool fresh) {
+            auto issue = [&](float4 *ring, uint64_t *fullb, uint32_t *tag, int stages, uint32_t t, bool fresh) {
                 const int k = (int)(t / (uint32_t)nchunk), c = (int)(t % (uint32_t)nchunk);
                 const int4 m = p.rows[cid + k * ncl];
                 const int s = (int)(t % stages);
@@ -208,6 +203,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
                 const uint32_t bytes = (uint32_t)min(kChunkVec, my_vec - c * kChunkVec) * 16u;
                 const bool teacher = fresh || m.z < 0;  // a sampled-token gradient needs the student only
                 float4 *dst = ring + (size_t)s * 2 * kChunkVec;
+                *(volatile uint32_t *)&tag[s] = t;     // the stage now belongs to chunk t
                 mbar_arrive_expect_tx(&fullb[s], (teacher ? 2u : 1u) * bytes);
                 if (kKeep && do_grad && fresh) {
                     bulk_g2s(dst, zs + base, bytes, &fullb[s], keep);
@@ -229,7 +225,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
                     const int s = (int)(ts % kSStages);
                     if (ts < (uint32_t)kSStages || mbar_test_wait(&sempty[s], ((ts / kSStages) - 1) & 1)) {
                         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                        issue(sring, sfull, kSStages, ts++, true);
+                        issue(sring, sfull, stag, kSStages, ts++, true);
                         moved = true;
                     }
                 }
@@ -237,16 +233,14 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
                     const int s = (int)(tg % kGStages);
                     if (tg < (uint32_t)kGStages || mbar_test_wait(&gempty[s], ((tg / kGStages) - 1) & 1)) {
                         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                        issue(gring, gfull, kGStages, tg++, false);
+                        issue(gring, gfull, gtag, kGStages, tg++, false);
                         moved = true;
                     }
                 }
-                if (moved) {
+                if (moved)
                     idle = 0;
-                } else if (++idle >= 16 * kWaitLimit) {  // test_wait never suspends: more polls
-                    s_dead = 1;
-                    set_status(p.status, TURNOPD_ERR_TIMEOUT);
-                }
+                else if (++idle >= 16 * kWaitLimit)  // test_wait never suspends: more polls
+                    give_up();
             }
             // after a timeout, let this CTA's own copies land before it exits
             if (dead()) {
@@ -264,23 +258,151 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
         return;
     }
 
-    // -------------------------------------------------------------------- consumers
-    // Per row: the statistics from the fresh chunks, the cluster merge, then the
-    // gradient from the chunks read again; meanwhile the producer streams the
-    // next row's fresh chunks.
-    auto bar_sync = [&]() { asm volatile("bar.sync %0, %1;" ::"r"(kBar), "r"(kNT) : "memory"); };
-    uint32_t ts = 0, tg = 0;
-    int4 m = p.rows[cid];
+    // -------------------------------------------------------------------- row groups
+    // Group g takes rows g, g + 2, ... of the cluster's list: the statistics from the
+    // fresh chunks, the cluster merge, then the gradient from the chunks read again.
+    // While one group exchanges records and writes its gradient, the other folds the
+    // next row's fresh chunks, so the HBM stream does not pause for either.
+    const int group = warp / kNWG, gwarp = warp % kNWG, gtid = tid % kNT;
+    float *red = reds + group * kNWG * 8;
+    float *bc = bcs + group * 8;
+    float *ysv = ysvs + group * 2;
+    auto group_sync = [&]() { asm volatile("bar.sync %0, %1;" ::"r"(1 + group), "r"(kNT) : "memory"); };
+    // chunk t of a ring: the stage must first be armed for chunk t (the other group
+    // may still hold the stage's previous chunk), then its phase must complete
+    auto wait_chunk = [&](uint64_t *fullb, const uint32_t *tag, int stages, uint32_t t) {
+        const int s = (int)(t % stages);
+        if (dead())
+            return;
+        uint32_t it = 0;
+        while (*(volatile const uint32_t *)&tag[s] != t && ++it < kWaitLimit) {
+        }
+        if (it >= kWaitLimit) {
+            give_up();
+            return;
+        }
+        wait_bar(&fullb[s], (t / stages) & 1, false);
+    };
 
-    // row constants of row j from its cluster records (warp 0; identical in every CTA)
-    auto constants = [&](int j, const int4 &mj) {
-        const int slot = j % kSlots;
-        float *bc = bcs + (j & 1) * 8;
-        if (warp == 0) {
-            wait_bar(&recv[slot], (uint32_t)((j / kSlots) & 1), true);
-            const float *r = rec + slot * kCS * 8;
+    int4 m = make_int4(0, 0, -1, 0);
+    if (group < n)
+        m = p.rows[cid + group * ncl];
+    for (int k = group; k < n; k += kG) {
+        const int4 m_next = k + kG < n ? p.rows[cid + (k + kG) * ncl] : m;  // a row ahead
+        const int y = m.z, yq = y >= 0 ? (y >> 2) - v0 : -1;
+
+        // statistics of row k's slice, in packed pairs: per pair of vectors a max
+        // pass, one rescale if the maximum moved, then the sums
+        float ms = -INFINITY, mt = -INFINITY, dd = 0.f;
+        float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
+        for (int c = 0; c < nchunk; ++c) {
+            const uint32_t t = (uint32_t)k * (uint32_t)nchunk + (uint32_t)c;
+            const int s = (int)(t % kSStages);
+            wait_chunk(sfull, stag, kSStages, t);
+            const float4 *cs = sring + (size_t)s * 2 * kChunkVec;
+            const float4 *ct = cs + kChunkVec;
+            const int cv = min(kChunkVec, my_vec - c * kChunkVec);
+            if (!dead()) {
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int q0 = gtid + 2 * h * kNT, q1 = q0 + kNT;
+                    if (q0 >= cv)
+                        break;
+                    const bool v1ok = q1 < cv;
+                    const float4 x0 = cs[q0], z0 = ct[q0];
+                    const float4 x1 = v1ok ? cs[q1] : x0, z1 = v1ok ? ct[q1] : z0;
+                    if (c * kChunkVec + q0 == yq) {
+                        ysv[0] = lane4(x0, y & 3);
+                        ysv[1] = lane4(z0, y & 3);
+                    }
+                    if (v1ok && c * kChunkVec + q1 == yq) {
+                        ysv[0] = lane4(x1, y & 3);
+                        ysv[1] = lane4(z1, y & 3);
+                    }
+                    // (x1, z1 repeat x0, z0 when the second vector is past the chunk: the
+                    // maxima are unchanged and its sums are skipped)
+                    const float cm = fmaxf(fmaxf(fmaxf(x0.x, x0.y), fmaxf(x0.z, x0.w)),
+                                           fmaxf(fmaxf(x1.x, x1.y), fmaxf(x1.z, x1.w)));
+                    const float cmt = fmaxf(fmaxf(fmaxf(z0.x, z0.y), fmaxf(z0.z, z0.w)),
+                                            fmaxf(fmaxf(z1.x, z1.y), fmaxf(z1.z, z1.w)));
+                    if (cm > ms) {
+                        // reference difference at the first element equal to the new maximum
+                        float xd = x0.x - z0.x;
+                        if (x0.x != cm) {
+                            xd = x0.y == cm ? x0.y - z0.y : x0.z == cm ? x0.z - z0.z : x0.w == cm ? x0.w - z0.w
+                               : x1.x == cm ? x1.x - z1.x : x1.y == cm ? x1.y - z1.y
+                               : x1.z == cm ? x1.z - z1.z : x1.w - z1.w;
+                        }
+                        const float2 f = splat(ex2((ms - cm) * kLog2e));
+                        A2 = fmul2(ffma2(S2, splat(dd - xd), A2), f);
+                        S2 = fmul2(S2, f);
+                        dd = xd;
+                        ms = cm;
+                    }
+                    if (cmt > mt) {
+                        T2 = fmul2(T2, splat(ex2((mt - cmt) * kLog2e)));
+                        mt = cmt;
+                    }
+                    const float2 L2 = splat(kLog2e), NS = splat(-ms * kLog2e), NTT = splat(-mt * kLog2e);
+                    const float2 D = splat(dd);
+                    const float4 xs[2] = {x0, x1}, zz[2] = {z0, z1};
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        if (u == 1 && !v1ok)
+                            break;
+                        const float2 a01 = make_float2(xs[u].x, xs[u].y), a23 = make_float2(xs[u].z, xs[u].w);
+                        const float2 b01 = make_float2(zz[u].x, zz[u].y), b23 = make_float2(zz[u].z, zz[u].w);
+                        const float2 e01 = ex2x2(ffma2(a01, L2, NS)), e23 = ex2x2(ffma2(a23, L2, NS));
+                        S2 = fadd2(S2, fadd2(e01, e23));
+                        A2 = ffma2(e01, fsub2(fsub2(a01, b01), D), A2);
+                        A2 = ffma2(e23, fsub2(fsub2(a23, b23), D), A2);
+                        T2 = fadd2(T2, fadd2(ex2x2(ffma2(b01, L2, NTT)), ex2x2(ffma2(b23, L2, NTT))));
+                    }
+                }
+            }
+            __syncwarp();
+            if (lane == 0)
+                mbar_arrive(&sempty[s]);
+        }
+
+        // row k's partial -> record to every CTA of the cluster
+        Student S = ms == -INFINITY ? student_empty() : Student{ms, S2.x + S2.y, A2.x + A2.y, dd};
+        Teacher U = mt == -INFINITY ? teacher_empty() : Teacher{mt, T2.x + T2.y};
+        lane_merge<32, true>(S, U);
+        if (lane == 0) {
+            float *rw = red + gwarp * 8;
+            rw[0] = S.m, rw[1] = S.s, rw[2] = S.a, rw[3] = S.d, rw[4] = U.m, rw[5] = U.s;
+        }
+        group_sync();
+        const int slot = k % kSlots;
+        if (gwarp == 0) {
             Student A = student_empty();
             Teacher B = teacher_empty();
+            if (lane < kNWG) {
+                const float *r = red + lane * 8;
+                A = Student{r[0], r[1], r[2], r[3]};
+                B = Teacher{r[4], r[5]};
+            }
+            lane_merge<kNWG, true>(A, B);
+            A.m = __shfl_sync(0xffffffffu, A.m, 0);
+            A.s = __shfl_sync(0xffffffffu, A.s, 0);
+            A.a = __shfl_sync(0xffffffffu, A.a, 0);
+            A.d = __shfl_sync(0xffffffffu, A.d, 0);
+            B.m = __shfl_sync(0xffffffffu, B.m, 0);
+            B.s = __shfl_sync(0xffffffffu, B.s, 0);
+            if (lane < kCS) {
+                const bool mine = yq >= 0 && yq < my_vec;
+                const float ys = mine ? ysv[0] : 0.f, yt = mine ? ysv[1] : 0.f;
+                const uint32_t ra = mapa(smem_u32(rec + (slot * kCS + (int)rank) * 8), (uint32_t)lane);
+                const uint32_t rbar = mapa(smem_u32(&recv[slot]), (uint32_t)lane);
+                st_async16(ra, rbar, make_float4(A.m, A.s, A.a, A.d));
+                st_async16(ra + 16, rbar, make_float4(B.m, B.s, ys, yt));
+            }
+            // the row's constants from the kCS records, in the same order in every CTA
+            wait_bar(&recv[slot], (uint32_t)((k / kSlots) & 1), true);
+            const float *r = rec + slot * kCS * 8;
+            A = student_empty();
+            B = teacher_empty();
             if (lane < kCS) {
                 const float4 x = *reinterpret_cast<const float4 *>(r + lane * 8);
                 const float4 z = *reinterpret_cast<const float4 *>(r + lane * 8 + 4);
@@ -290,7 +412,6 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
             lane_merge<kCS, true>(A, B);
             if (lane == 0) {
                 const RowConst rc = row_const(A, B);
-                const int y = mj.z;
                 float e = rc.kl;
                 if (y >= 0) {
                     const int owner = (y >> 2) / slice_vec;
@@ -298,7 +419,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
                 }
                 // p |w| = 2^(z_s log2e - LSE_s log2e + log2 |w|); the sign of w enters
                 // through an fma by sg
-                const float wi = __int_as_float(mj.w), wl = wi * e;
+                const float wi = __int_as_float(m.w), wl = wi * e;
                 const float sg = wi < 0.f ? -1.f : 1.f;
                 bc[0] = -rc.lse_s * kLog2e + log2f(fabsf(y < 0 ? wi : wl));  // nlw
                 bc[1] = sg;
@@ -310,179 +431,51 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
                 if (rank == 0) {
                     if (!isfinite(rc.lse_s) || !isfinite(rc.lse_t) || !isfinite(e))
                         set_status(p.status, TURNOPD_ERR_NONFINITE);
-                    p.token_loss[mj.x] = e;
-                    p.row_wl[cid + j * ncl] = (double)wi * (double)e;
+                    p.token_loss[m.x] = e;
+                    p.row_wl[cid + k * ncl] = (double)wi * (double)e;
                 }
-                mbar_arrive_expect_tx(&recv[slot], kCS * 32u);  // re-arm for row j + kSlots
+                mbar_arrive_expect_tx(&recv[slot], kCS * 32u);  // re-arm for row k + kSlots
             }
         }
-        bar_sync();
-    };
+        group_sync();
 
-    // gradient of chunk c of row j, from the gradient ring's next stage
-    auto grad_chunk = [&](int j, const int4 &mj, int c) {
-        const int s = (int)(tg % kGStages);
-        wait_bar(&gfull[s], (tg / kGStages) & 1, false);
-        ++tg;
-        if (!dead()) {
-            const float *bc = bcs + (j & 1) * 8;
-            const float4 *ga = gring + (size_t)s * 2 * kChunkVec, *gb = ga + kChunkVec;
-            const size_t off = (size_t)mj.y * (size_t)p.ld + (size_t)v0 * 4;
-            const int cv = min(kChunkVec, my_vec - c * kChunkVec);
-            const int y = mj.z, yq = y >= 0 ? (y >> 2) - v0 : -1;
+        // the gradient of my slice from the chunks read again
+        if (do_grad) {
+            const size_t off = (size_t)m.y * (size_t)p.ld + (size_t)v0 * 4;
+            for (int c = 0; c < nchunk; ++c) {
+                const uint32_t t = (uint32_t)k * (uint32_t)nchunk + (uint32_t)c;
+                const int s = (int)(t % kGStages);
+                wait_chunk(gfull, gtag, kGStages, t);
+                if (!dead()) {
+                    const float4 *ga = gring + (size_t)s * 2 * kChunkVec, *gb = ga + kChunkVec;
+                    const int cv = min(kChunkVec, my_vec - c * kChunkVec);
 #pragma unroll
-            for (int u = 0; u < kVPT; ++u) {
-                const int ql = tid + u * kNT;
-                if (ql < cv) {
-                    const int q = c * kChunkVec + ql;
-                    const float4 a = ga[ql], b = y < 0 ? gb[ql] : a;
-                    if (kKeep && (ql & 7) == 0) {  // one thread per 128-byte line of each model
-                        l2_evict_normal(zs + off + (size_t)q * 4);
-                        l2_evict_normal(zt + off + (size_t)q * 4);
+                    for (int u = 0; u < 4; ++u) {
+                        const int ql = gtid + u * kNT;
+                        if (ql < cv) {
+                            const int q = c * kChunkVec + ql;
+                            const float4 a = ga[ql], b = y < 0 ? gb[ql] : a;
+                            if (kKeep && (ql & 7) == 0) {  // one thread per 128-byte line of each model
+                                l2_evict_normal(zs + off + (size_t)q * 4);
+                                l2_evict_normal(zt + off + (size_t)q * 4);
+                            }
+                            const float4 g4 = grad4<G32>(a, b, bc, y >= 0, q == yq ? (y & 3) : -1);
+                            if (G32) {
+                                __stcs(reinterpret_cast<float4 *>(static_cast<float *>(p.grad) + off) + q, g4);
+                            } else {
+                                uint2 o;
+                                o.x = pack_bf16x2(g4.x, g4.y);
+                                o.y = pack_bf16x2(g4.z, g4.w);
+                                __stcs(reinterpret_cast<uint2 *>(static_cast<__nv_bfloat16 *>(p.grad) + off) + q, o);
+                            }
+                        }
                     }
-                    const float4 g4 = grad4<G32>(a, b, bc, y >= 0, q == yq ? (y & 3) : -1);
-                    if (G32) {
-                        __stcs(reinterpret_cast<float4 *>(static_cast<float *>(p.grad) + off) + q, g4);
-                    } else {
-                        uint2 o;
-                        o.x = pack_bf16x2(g4.x, g4.y);
-                        o.y = pack_bf16x2(g4.z, g4.w);
-                        __stcs(reinterpret_cast<uint2 *>(static_cast<__nv_bfloat16 *>(p.grad) + off) + q, o);
-                    }
                 }
+                __syncwarp();
+                if (lane == 0)
+                    mbar_arrive(&gempty[s]);
             }
         }
-        __syncwarp();
-        if (lane == 0)
-            mbar_arrive(&gempty[s]);
-    };
-
-    int4 m_prev = m;
-    for (int k = 0; k <= n; ++k) {
-        const bool have = k < n, prev = k > 0;
-        const int4 m_next = k + 1 < n ? p.rows[cid + (k + 1) * ncl] : m;  // a row ahead
-        float *ysv = ysvs + (k & 1) * 2;
-        const int y = m.z, yq = y >= 0 ? (y >> 2) - v0 : -1;
-        // row k - 1's constants and gradient, once kLag fresh chunks of row k have been
-        // folded: its cluster records are in flight meanwhile
-        bool prev_done = !prev;
-        auto finish_prev = [&]() {
-            constants(k - 1, m_prev);
-            if (do_grad)
-                for (int c = 0; c < nchunk; ++c)
-                    grad_chunk(k - 1, m_prev, c);
-            prev_done = true;
-        };
-
-        // statistics of row k's slice, in packed pairs: per chunk a max pass, one
-        // rescale if the maximum moved, then the sums
-        float ms = -INFINITY, mt = -INFINITY, dd = 0.f;
-        float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
-        for (int c = 0; c < (have ? nchunk : 0); ++c) {
-            if (!prev_done && c == kLag)
-                finish_prev();
-            const int s = (int)(ts % kSStages);
-            wait_bar(&sfull[s], (ts / kSStages) & 1, false);
-            ++ts;
-            const float4 *cs = sring + (size_t)s * 2 * kChunkVec;
-            const float4 *ct = cs + kChunkVec;
-            const int cv = min(kChunkVec, my_vec - c * kChunkVec);
-            const bool v0ok = tid < cv, v1ok = tid + kNT < cv;
-            if (!dead() && v0ok) {
-                const float4 x0 = cs[tid], z0 = ct[tid];
-                const float4 x1 = v1ok ? cs[tid + kNT] : x0, z1 = v1ok ? ct[tid + kNT] : z0;
-                if (c * kChunkVec + tid == yq) {
-                    ysv[0] = lane4(x0, y & 3);
-                    ysv[1] = lane4(z0, y & 3);
-                }
-                if (v1ok && c * kChunkVec + tid + kNT == yq) {
-                    ysv[0] = lane4(x1, y & 3);
-                    ysv[1] = lane4(z1, y & 3);
-                }
-                // (x1, z1 repeat x0, z0 when the second vector is past the chunk: the
-                // maxima are unchanged and its sums are skipped)
-                const float cm = fmaxf(fmaxf(fmaxf(x0.x, x0.y), fmaxf(x0.z, x0.w)),
-                                       fmaxf(fmaxf(x1.x, x1.y), fmaxf(x1.z, x1.w)));
-                const float cmt = fmaxf(fmaxf(fmaxf(z0.x, z0.y), fmaxf(z0.z, z0.w)),
-                                        fmaxf(fmaxf(z1.x, z1.y), fmaxf(z1.z, z1.w)));
-                if (cm > ms) {
-                    // reference difference at the first element equal to the new maximum
-                    float xd = x0.x - z0.x;
-                    if (x0.x != cm) {
-                        xd = x0.y == cm ? x0.y - z0.y : x0.z == cm ? x0.z - z0.z : x0.w == cm ? x0.w - z0.w
-                           : x1.x == cm ? x1.x - z1.x : x1.y == cm ? x1.y - z1.y
-                           : x1.z == cm ? x1.z - z1.z : x1.w - z1.w;
-                    }
-                    const float2 f = splat(ex2((ms - cm) * kLog2e));
-                    A2 = fmul2(ffma2(S2, splat(dd - xd), A2), f);
-                    S2 = fmul2(S2, f);
-                    dd = xd;
-                    ms = cm;
-                }
-                if (cmt > mt) {
-                    T2 = fmul2(T2, splat(ex2((mt - cmt) * kLog2e)));
-                    mt = cmt;
-                }
-                const float2 L2 = splat(kLog2e), NS = splat(-ms * kLog2e), NTT = splat(-mt * kLog2e);
-                const float2 D = splat(dd);
-                const float4 xs[2] = {x0, x1}, zz[2] = {z0, z1};
-#pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    if (u == 1 && !v1ok)
-                        break;
-                    const float2 a01 = make_float2(xs[u].x, xs[u].y), a23 = make_float2(xs[u].z, xs[u].w);
-                    const float2 b01 = make_float2(zz[u].x, zz[u].y), b23 = make_float2(zz[u].z, zz[u].w);
-                    const float2 e01 = ex2x2(ffma2(a01, L2, NS)), e23 = ex2x2(ffma2(a23, L2, NS));
-                    S2 = fadd2(S2, fadd2(e01, e23));
-                    A2 = ffma2(e01, fsub2(fsub2(a01, b01), D), A2);
-                    A2 = ffma2(e23, fsub2(fsub2(a23, b23), D), A2);
-                    T2 = fadd2(T2, fadd2(ex2x2(ffma2(b01, L2, NTT)), ex2x2(ffma2(b23, L2, NTT))));
-                }
-            }
-            __syncwarp();
-            if (lane == 0)
-                mbar_arrive(&sempty[s]);
-        }
-        if (!prev_done)
-            finish_prev();
-        if (!have)
-            break;
-
-        // row k's partial -> record to every CTA of the cluster
-        Student S = ms == -INFINITY ? student_empty() : Student{ms, S2.x + S2.y, A2.x + A2.y, dd};
-        Teacher U = mt == -INFINITY ? teacher_empty() : Teacher{mt, T2.x + T2.y};
-        lane_merge<32, true>(S, U);
-        if (lane == 0) {
-            float *rw = red + warp * 8;
-            rw[0] = S.m, rw[1] = S.s, rw[2] = S.a, rw[3] = S.d, rw[4] = U.m, rw[5] = U.s;
-        }
-        bar_sync();
-        if (warp == 0) {
-            Student A = student_empty();
-            Teacher B = teacher_empty();
-            if (lane < kNW) {
-                const float *r = red + lane * 8;
-                A = Student{r[0], r[1], r[2], r[3]};
-                B = Teacher{r[4], r[5]};
-            }
-            lane_merge<kNW, true>(A, B);
-            A.m = __shfl_sync(0xffffffffu, A.m, 0);
-            A.s = __shfl_sync(0xffffffffu, A.s, 0);
-            A.a = __shfl_sync(0xffffffffu, A.a, 0);
-            A.d = __shfl_sync(0xffffffffu, A.d, 0);
-            B.m = __shfl_sync(0xffffffffu, B.m, 0);
-            B.s = __shfl_sync(0xffffffffu, B.s, 0);
-            if (lane < kCS) {
-                const bool mine = yq >= 0 && yq < my_vec;
-                const float ys = mine ? ysv[0] : 0.f, yt = mine ? ysv[1] : 0.f;
-                const int slot = k % kSlots;
-                const uint32_t ra = mapa(smem_u32(rec + (slot * kCS + (int)rank) * 8), (uint32_t)lane);
-                const uint32_t rbar = mapa(smem_u32(&recv[slot]), (uint32_t)lane);
-                st_async16(ra, rbar, make_float4(A.m, A.s, A.a, A.d));
-                st_async16(ra + 16, rbar, make_float4(B.m, B.s, ys, yt));
-            }
-        }
-        m_prev = m;
         m = m_next;
     }
     cluster_sync();  // no CTA leaves while a peer may still address its shared memory
