@@ -284,7 +284,9 @@ int oracle_weights(const int32_t *turn_id, const uint8_t *mask,
  * full vocabulary:  l = KL(p_s || p_t) = sum_v p_v (ls_v - lt_v)
  *                   g_v = w p_v (ls_v - lt_v - l)          (= w dKL/dzs_v)
  * sampled token y:  l = ls_y - lt_y
- *                   g_v = w l (delta_{v,y} - p_v)          (score function)
+ *                   g_v = w l (delta_{v,y} - p_v)          (score function),
+ *                   with 1 - p_y taken as sum_{v != y} p_v (equal, as the p_v sum
+ *                   to 1, and free of the cancellation of 1 - p_y near p_y = 1)
  * out[0] = LSE_s, out[1] = LSE_t, out[2] = l, out[3] = full-vocab KL.
  * g (nullable) receives V doubles.
  */
@@ -322,6 +324,11 @@ static int row_core(const double *zs, const double *zt, int64_t V, int32_t mode,
     else
         ell = (zs[y] - lse_s) - (zt[y] - lse_t);
     if (g) {
+        kahan_t rest = {0, 0};  /* sampled token: 1 - p_y = sum_{v != y} p_v */
+        if (mode == OR_SAMPLED_TOKEN)
+            for (int64_t v = 0; v < V; ++v)
+                if (v != y)
+                    kadd(&rest, exp(zs[v] - lse_s));
         for (int64_t v = 0; v < V; ++v) {
             double ls = zs[v] - lse_s;
             double lt = zt[v] - lse_t;
@@ -329,7 +336,7 @@ static int row_core(const double *zs, const double *zt, int64_t V, int32_t mode,
             if (mode == OR_FULL_VOCAB)
                 g[v] = w * p * (ls - lt - KL);
             else
-                g[v] = w * ell * ((v == y ? 1.0 : 0.0) - p);
+                g[v] = v == y ? w * ell * kval(&rest) : -w * ell * p;
         }
     }
     out[0] = lse_s;

@@ -402,6 +402,28 @@ def test_sampled_mode_exact_expectation(oracle):
         np.testing.assert_allclose(eg, gfull, rtol=1e-9, atol=1e-14)
 
 
+def test_sampled_gradient_at_a_dominant_token(oracle):
+    """Sampled token y whose student logit c stands above V - 1 zeros: p_y = e^c / (e^c + V - 1),
+    so g_y = w l (V - 1) / (e^c + V - 1) and g_v = -w l / (e^c + V - 1) in closed form, with
+    1 - p_y down to ~6e-13 at c = 40 (where 1 - p_y formed by subtraction keeps only ~4
+    digits even in fp64, and none in fp32)."""
+    rng = np.random.default_rng(9)
+    V = 151936
+    for c in (10.0, 20.0, 30.0, 40.0):
+        y = int(rng.integers(0, V))
+        zs = np.zeros(V, np.float32)
+        zs[y] = c
+        zt = f32(rng.normal(0, 2, V))
+        lse_s, lse_t, l, _, g = oracle.row(zs, zt, mode=1, y=y, w=0.7)
+        den = math.exp(c) + (V - 1)
+        assert math.isclose(lse_s, math.log(den), rel_tol=1e-14)
+        lse_t_ref = float(np.logaddexp.reduce(zt.astype(np.float64)))
+        assert math.isclose(l, (c - float(zt[y])) - (math.log(den) - lse_t_ref), rel_tol=1e-12, abs_tol=1e-12)
+        assert math.isclose(g[y], 0.7 * l * (V - 1) / den, rel_tol=1e-10)
+        others = np.delete(g, y)
+        np.testing.assert_allclose(others, -0.7 * l / den, rtol=1e-12)
+
+
 def test_sampled_mode_monte_carlo(oracle):
     """V = 1024: the sample mean of l(y), y drawn from softmax(z_s), lies within 5 sigma of KL."""
     rng = np.random.default_rng(8)
