@@ -35,6 +35,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "loss fwd+bwd tokens/s at V=151936 bf16 on 1 GB300; achieved HBM GB/s vs peak"
 UNIT = "tokens/s"
+V_QWEN = 151_936  # the workloads' vocabulary (a --vocab run has no committed traffic record)
 # counts(2) + weights(1) + compaction(2) + row kernel + loss sum + stats(2); the full and
 # sampled modes on bf16 logits add the helper grid that runs beside the cluster grid
 KERNELS_PER_STEP = 9
@@ -63,6 +64,8 @@ def parse():
     p.add_argument("--zero-masked", action="store_true",
                    help="dense layout with TURNOPD_ZERO_MASKED_GRAD: masked tokens' gradient rows written as zeros")
     p.add_argument("--fp32-grad", action="store_true", help="full/sampled modes: an fp32 gradient instead of bf16")
+    p.add_argument("--vocab", type=int, default=0,
+                   help="full/sampled/top-K modes: vocabulary size (0 = the workload's 151,936)")
     p.add_argument("--fp32-logits", action="store_true",
                    help="full/sampled modes: fp32 logits instead of bf16 (the split-row kernel)")
     p.add_argument("--alpha", type=float, default=0.5)
@@ -185,7 +188,7 @@ def build_inputs(args, rank, device):
         b = W.CONFIGS[args.workload](seed=rank)
     from paper_2607_05804_gb300 import TURNOPD_ZERO_MASKED_GRAD
 
-    V = W.V_QWEN
+    V = args.vocab or W.V_QWEN
     dense = dense_layout(args)
     rows = b.num_tokens if dense else b.num_valid
     zs, zt = W.make_logits(rows, V, "agent", torch.float32 if args.fp32_logits else torch.bfloat16,
@@ -607,7 +610,8 @@ def main():
                            "+ compaction + loss sum)"),
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "launch_ms": loss_avg_ms,
-                "traffic": (None if (args.vocab_shards or dense_layout(args) or args.fp32_logits)
+                "traffic": (None if (args.vocab_shards or dense_layout(args) or args.fp32_logits
+                                     or V != V_QWEN)
                             else committed_traffic(args.workload, R, "topk") if args.mode == "topk"
                             else committed_traffic(args.workload)),
             },

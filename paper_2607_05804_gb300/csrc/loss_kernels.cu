@@ -8,9 +8,12 @@
 //   m, S = sum exp(z - m) for both models by an online (rescaling) pass,
 //   A = sum exp(z_s - m_s) (z_s - z_t)  ->  KL = A/S_s - (LSE_s - LSE_t),
 // then the gradient pass g_v = w p_v ((z_s - z_t)_v - (LSE_s - LSE_t) - KL)
-// (full vocabulary) or g_v = w l (delta_vy - p_v) (sampled token).
+// (full vocabulary) or g_v = w l (delta_vy - p_v) (sampled token; g_y = w l (1 - p_y)
+// from student statistics without y, merged back at the end, so that it keeps its
+// precision when p_y is near 1).
 
 #include <algorithm>
+#include <cfloat>
 
 #include "common.cuh"
 #include "row_math.cuh"
@@ -176,7 +179,7 @@ k_row_portable(RowIn p)
 {
     __shared__ Student red_s[kRowThreads / 32];
     __shared__ Teacher red_t[kRowThreads / 32];
-    __shared__ float bc[5];
+    __shared__ float bc[6];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int nvalid = *p.nvalid;
     const TIn *zs = static_cast<const TIn *>(p.zs);
@@ -194,17 +197,31 @@ k_row_portable(RowIn p)
         const TIn *rt = zt + r * p.ld;
         Student s = student_empty();
         Teacher t = teacher_empty();
+        // a sampled-token row leaves y out of the student statistics (add_sampled_term
+        // brings its term back at the merge): in a vector its logit reads as the lowest
+        // finite value (never the maximum beside the other N - 1, adds 0); read alone
+        // it folds into the teacher only
+        const int64_t ys = p.mode == TURNOPD_SAMPLED_TOKEN ? (int64_t)meta.z : -1;
         if (VEC) {
             for (int64_t q = threadIdx.x; q < nvec; q += kRowThreads) {
                 float a[N], b[N];
                 Vec<TIn>::load(rs + q * N, a);
                 Vec<TIn>::load(rt + q * N, b);
+                if (ys >= 0 && q == ys / N) {
+#pragma unroll
+                    for (int k = 0; k < N; ++k)
+                        if (k == (int)(ys % N))
+                            a[k] = -FLT_MAX;
+                }
                 accumulate<N>(s, t, a, b);
             }
         }
         for (int64_t v = nvec * N + threadIdx.x; v < V; v += kRowThreads) {
-            float a = to_float(rs[v]), b = to_float(rt[v]);
-            accumulate<1>(s, t, &a, &b);
+            const float a = to_float(rs[v]), b = to_float(rt[v]);
+            if (v == ys)
+                accumulate_teacher(t, b);
+            else
+                accumulate<1>(s, t, &a, &b);
         }
         s = warp_merge(s);
         t = warp_merge(t);
@@ -220,12 +237,13 @@ k_row_portable(RowIn p)
                 S = student_merge(S, red_s[k]);
                 U = teacher_merge(U, red_t[k]);
             }
+            float omp = 0.f;  // 1 - p_y (sampled)
+            if (ys >= 0)
+                omp = add_sampled_term(S, to_float(rs[ys]));
             const RowConst rc = row_const(S, U);
             float ell = rc.kl;
-            if (p.mode == TURNOPD_SAMPLED_TOKEN) {
-                const int32_t y = meta.z;
-                ell = (to_float(rs[y]) - to_float(rt[y])) - rc.dl;
-            }
+            if (ys >= 0)
+                ell = (to_float(rs[ys]) - to_float(rt[ys])) - rc.dl;
             const float wi = __int_as_float(meta.w);
             if (!isfinite(rc.lse_s) || !isfinite(rc.lse_t) || !isfinite(ell))
                 set_status(p.status, TURNOPD_ERR_NONFINITE);
@@ -236,10 +254,11 @@ k_row_portable(RowIn p)
             bc[2] = rc.cp;  // g = w p (((z_s - z_t) - d) - cp)
             bc[3] = wi;
             bc[4] = wi * ell;
+            bc[5] = wi * ell * omp;  // g_y = w l (1 - p_y)
         }
         __syncthreads();
         if (grad) {
-            const float nl = -bc[0] * kLog2e, d = bc[1], cp = bc[2], wi = bc[3], wl = bc[4];
+            const float nl = -bc[0] * kLog2e, d = bc[1], cp = bc[2], wi = bc[3], wl = bc[4], gy = bc[5];
             const bool sampled = p.mode == TURNOPD_SAMPLED_TOKEN;
             const int64_t y = sampled ? (int64_t)meta.z : -1;
             TOut *gr = grad + r * p.ld;
@@ -251,7 +270,7 @@ k_row_portable(RowIn p)
 #pragma unroll
                     for (int k = 0; k < N; ++k) {
                         const float pv = ex2(fmaf(a[k], kLog2e, nl));
-                        g[k] = sampled ? (((q * N + k) == y ? wl : 0.f) - wl * pv)
+                        g[k] = sampled ? ((q * N + k) == y ? gy : -wl * pv)
                                        : wi * pv * (((a[k] - b[k]) - d) - cp);
                     }
                     store_vec<TOut, N>(gr + q * N, g);
@@ -260,7 +279,7 @@ k_row_portable(RowIn p)
             for (int64_t v = nvec * N + threadIdx.x; v < V; v += kRowThreads) {
                 const float a = to_float(rs[v]), b = to_float(rt[v]);
                 const float pv = ex2(fmaf(a, kLog2e, nl));
-                const float g = sampled ? ((v == y ? wl : 0.f) - wl * pv) : wi * pv * (((a - b) - d) - cp);
+                const float g = sampled ? (v == y ? gy : -wl * pv) : wi * pv * (((a - b) - d) - cp);
                 gr[v] = from_float<TOut>(g);
             }
         }

@@ -126,4 +126,35 @@ __device__ __forceinline__ void accumulate(Student &s, Teacher &t, const float *
     }
 }
 
+// Fold one teacher value alone, in the steps of accumulate<1>: a sampled-token row's y
+// where it is not part of a vector (see add_sampled_term).
+__device__ __forceinline__ void accumulate_teacher(Teacher &t, float b)
+{
+    if (b > t.m) {
+        t.s *= ex2((t.m - b) * kLog2e);
+        t.m = b;
+    }
+    t.s += ex2(fmaf(b, kLog2e, -t.m * kLog2e));
+}
+
+// Sampled-token row (Eq. opd-rkl's one-token estimator): the student statistics leave y
+// out altogether -- within a vector of finite logits its logit is replaced by the
+// lowest finite value, which is then never the maximum and adds 0 to every sum; a y
+// read alone folds into the teacher only -- so s holds S' = sum_{v != y} exp(z_s - m')
+// at the maximum m' of the other logits.  This adds y's own term at M = max(m', z_y):
+// S = S' e^{m' - M} + e^{z_y - M}, and returns 1 - p_y = S' e^{m' - M} / S, which
+// keeps its relative precision when p_y is close to 1 (1 - p_y formed as 1 - e_y / S,
+// or as w l - w l p_y, loses it to cancellation).  A is rescaled with S; y's term of
+// A stays out (a sampled-token row does not use A).
+__device__ __forceinline__ float add_sampled_term(Student &s, float zy)
+{
+    const float M = fmaxf(s.m, zy);
+    const float f = s.m == -INFINITY ? 0.f : ex2((s.m - M) * kLog2e);
+    const float sx = s.s * f;
+    s.a *= f;
+    s.m = M;
+    s.s = sx + ex2((zy - M) * kLog2e);
+    return sx / s.s;
+}
+
 }  // namespace turnopd

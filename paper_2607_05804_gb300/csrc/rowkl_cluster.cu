@@ -53,14 +53,15 @@ struct GradConst {
     float nd, ncp;    // -sg d, -sg cp
     float nc;         // -sg (d + cp)
     float sgl;        // sign of -w l (sampled)
-    float wl;         // w l
+    float gy;         // sampled: g_y = w l (1 - p_y)
 };
 
 // G groups of NT threads per CTA take the rows of the cluster in turn (row k
 // to group k % G).  Record slots: 2G, so a slot is reused by the same group
 // two rows later, after that group has read it (a peer can run at most G rows
-// ahead of the slowest CTA in sending records).
-template <int CS, int NT, int VPT, int G, bool G32>
+// ahead of the slowest CTA in sending records).  SM: a sampled-token call, where
+// every listed row carries its y in [0, V); otherwise the full vocabulary (y = -1).
+template <int CS, int NT, int VPT, int G, bool G32, bool SM>
 __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_vec, int nvec)
 {
     constexpr int kSlots = 2 * G;
@@ -90,7 +91,8 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
     uint64_t *recv = empty + kStages;                                      // [kSlots]
     float *red = reinterpret_cast<float *>(recv + kSlots);                 // [G][NWG][8]
     int *srow = reinterpret_cast<int *>(red + G * NWG * 8);                // [kStages] row in stage
-    float *rcs = reinterpret_cast<float *>(srow + 4);                       // [G][16] row constants
+    int *yown = srow + 4;                                                  // [kStages] thread reading y, or -1
+    float *rcs = reinterpret_cast<float *>(srow + 8);                       // [G][16] row constants; [15]: z_s[y]
 
     if (tid == 0) {
         s_dead = 0;
@@ -156,6 +158,10 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
     auto issue = [&](int k, int4 m) {
         const int s = k % kStages;
         meta[s] = m;
+        if (SM) {  // the thread that will read y's vector (sampled-token rows; see stats)
+            const int q = m.z >= 0 ? (m.z >> 3) - v0 : -1;
+            yown[s] = q >= 0 && q < my_vec ? q % NT : -1;
+        }
         *(volatile int *)&srow[s] = k;
         const size_t off = (size_t)m.y * (size_t)p.ld + (size_t)v0 * 8;
         const char *gs = reinterpret_cast<const char *>(zs + off);
@@ -175,6 +181,22 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
         const int s = k % kStages;
         const uint4 *vs = reinterpret_cast<const uint4 *>(stage + s * stage_bytes);
         const uint4 *vt = reinterpret_cast<const uint4 *>(stage + s * stage_bytes + slice_bytes);
+        // A sampled-token row leaves y out of the student statistics (add_sampled_term
+        // brings its term back at the merge): the thread that reads y's vector in both
+        // passes below (named at issue) keeps z_s[y] for the record and puts the lowest
+        // finite bf16 in its place, which is never the maximum and adds 0.  (The gradient
+        // pass replaces g_y; the proxy fence orders the store before the stage's next
+        // bulk copy.)
+        if (SM && yown[s] == gtid) {
+            const uint32_t ay = smem_u32(stage + s * stage_bytes) + 2u * (uint32_t)(meta[s].z - v0 * 8);
+            uint32_t old;
+            asm volatile("ld.shared.u16 %0, [%1];\n\tst.shared.u16 [%1], %2;\n\t"
+                         "fence.proxy.async.shared::cta;"
+                         : "=r"(old)
+                         : "r"(ay), "r"(0xff7fu)
+                         : "memory");
+            rcs[group * 16 + 15] = __uint_as_float(old << 16);
+        }
         // max pass (packed bf16): running maxima, plus each vector's student
         // maximum kept packed so the argmax vector is found after the loop
         uint32_t smax = 0xff80ff80u, tmax = 0xff80ff80u;  // (-inf, -inf)
@@ -263,7 +285,7 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
                 const int y = meta[s].z;
                 if (y >= 0 && y / 8 >= v0 && y / 8 < v0 + my_vec) {
                     const int e = y - v0 * 8;
-                    ys = to_float(reinterpret_cast<const __nv_bfloat16 *>(vs)[e]);
+                    ys = SM ? rcs[group * 16 + 15] : to_float(reinterpret_cast<const __nv_bfloat16 *>(vs)[e]);
                     yt = to_float(reinterpret_cast<const __nv_bfloat16 *>(vt)[e]);
                 }
                 const int slot = k % kSlots;
@@ -294,25 +316,27 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
             }
             lane_merge<CS, kUseD>(A, B);
             if (lane == 0) {
+                const int y = meta[k % kStages].z;
+                const int owner = SM ? (y / 8) / slice_vec : 0;
+                float omp = 0.f;  // 1 - p_y (sampled)
+                if (SM)
+                    omp = add_sampled_term(A, r[owner * 8 + 6]);
                 const RowConst rc = row_const(A, B);
                 float e = rc.kl;
-                const int y = meta[k % kStages].z;
-                if (y >= 0) {
-                    const int owner = (y / 8) / slice_vec;
+                if (SM)
                     e = (r[owner * 8 + 6] - r[owner * 8 + 7]) - rc.dl;
-                }
                 // gradient constants of the row (see grad): p w = 2^(z_s log2e + nlw),
                 // sign sg of w applied through fma by (sg, sg)
                 const float wi = __int_as_float(meta[k % kStages].w), wl = wi * e;
                 const float sg = wi < 0.f ? -1.f : 1.f;
                 bc[0] = rc.lse_s, bc[1] = rc.lse_t, bc[2] = rc.kl, bc[3] = e;
-                bc[4] = -rc.lse_s * kLog2e + log2f(fabsf(y < 0 ? wi : wl));  // nlw
+                bc[4] = -rc.lse_s * kLog2e + log2f(fabsf(SM ? wl : wi));  // nlw
                 bc[5] = sg;
                 bc[6] = -sg * rc.d;
                 bc[7] = -sg * rc.cp;
                 bc[8] = -sg * (rc.d + rc.cp);     // bf16 output: one rounding of d + cp
                 bc[9] = wl > 0.f ? -1.f : 1.f;    // sampled: sign of -w l
-                bc[10] = wl;
+                bc[10] = wl * omp;                 // sampled: g_y = w l (1 - p_y)
                 mbar_arrive_expect_tx(&recv[slot], CS * 32u);  // re-arm for row k + kSlots
             }
         }
@@ -321,7 +345,7 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
         gc.lse_s = bc[0], gc.lse_t = bc[1], gc.kl = bc[2];
         ell = bc[3];
         gc.nlw = bc[4], gc.sg = bc[5], gc.nd = bc[6], gc.ncp = bc[7], gc.nc = bc[8], gc.sgl = bc[9];
-        gc.wl = bc[10];
+        gc.gy = bc[10];
         return gc;
     };
 
@@ -333,7 +357,7 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
         const uint4 *vs = reinterpret_cast<const uint4 *>(stage + s * stage_bytes);
         const uint4 *vt = reinterpret_cast<const uint4 *>(stage + s * stage_bytes + slice_bytes);
         const int y = m.z;
-        const float wl = gc.wl;
+        const float gy = gc.gy;
         const size_t row_off = (size_t)m.y * (size_t)p.ld + (size_t)v0 * 8;
         // p |w| = 2^(z_s log2e - LSE_s log2e + log2 |w|); the sign of w enters through an
         // fma by (sg, sg), which is exact on z_s - z_t
@@ -345,7 +369,7 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
             const int q = gtid + u * NT;
             if (q < my_vec) {
                 float2 g[4];
-                if (y < 0) {  // full vocabulary: g = w p ((z_s - z_t) - d - cp)
+                if (!SM) {  // full vocabulary: g = w p ((z_s - z_t) - d - cp)
                     const uint4 a = vs[q], b = vt[q];
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
@@ -355,21 +379,11 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
                         const float2 x = fsub2(a2, b2);
                         g[j] = G32 ? fmul2(pw, fadd2(ffma2(x, SG, ND), NCP)) : fmul2(pw, ffma2(x, SG, NC));
                     }
-                } else {  // sampled token: g = w l (e_y - p)
+                } else {  // sampled token: g = -w l p (g_y is written after the loop)
                     const uint4 a = vs[q];
 #pragma unroll
                     for (int j = 0; j < 4; ++j)
                         g[j] = fmul2(ex2x2(ffma2(unpack2(word(a, j)), L2, NLW)), SGL);
-                    if (v0 + q == (y >> 3)) {  // the vector holding y
-                        const int yi = y & 7;
-#pragma unroll
-                        for (int j = 0; j < 4; ++j) {
-                            if (yi == 2 * j)
-                                g[j].x += wl;
-                            if (yi == 2 * j + 1)
-                                g[j].y += wl;
-                        }
-                    }
                 }
                 if (G32) {
                     float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(p.grad) + row_off +
@@ -387,6 +401,15 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
                            o);
                 }
             }
+        }
+        // sampled token: g_y = w l (1 - p_y), over the value the vector store wrote
+        // (same thread, so the later store wins)
+        if (SM && yown[s] == gtid) {
+            const size_t yo = (size_t)m.y * (size_t)p.ld + (size_t)y;
+            if (G32)
+                static_cast<float *>(p.grad)[yo] = gy;
+            else
+                static_cast<__nv_bfloat16 *>(p.grad)[yo] = __float2bfloat16_rn(gy);
         }
     };
 
@@ -432,6 +455,19 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
     cluster_sync();  // no CTA leaves while a peer may still address its shared memory
 }
 
+// v with its bf16 lane i (0..7) replaced by the lowest finite bf16
+__device__ __forceinline__ uint4 fill_lane(uint4 v, int i)
+{
+    const uint32_t keep = (i & 1) ? 0x0000ffffu : 0xffff0000u;
+    const uint32_t fill = 0xff7fff7fu & ~keep;
+    const int w = i >> 1;
+    v.x = w == 0 ? (v.x & keep) | fill : v.x;
+    v.y = w == 1 ? (v.y & keep) | fill : v.y;
+    v.z = w == 2 ? (v.z & keep) | fill : v.z;
+    v.w = w == 3 ? (v.w & keep) | fill : v.w;
+    return v;
+}
+
 // Helper for the SMs the clusters leave free (15 eight-CTA clusters cover 120 of
 // 152): one CTA per row at a time, rows j0 + blockIdx.x, j0 + blockIdx.x +
 // gridDim.x, ... of the row list, j0 = the cluster kernel's share.  The
@@ -447,7 +483,7 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
 constexpr int kHelpThreads = 512;
 constexpr int kHelpU = 4;  // vectors of each model in flight per thread
 
-template <bool G32, int NTH = kHelpThreads, int MINB = 1>
+template <bool G32, bool SM, int NTH = kHelpThreads, int MINB = 1>
 __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
 {
     constexpr int kHelpThreads = NTH;
@@ -467,6 +503,7 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
         const size_t off = (size_t)m.y * (size_t)p.ld;
         const uint4 *vs = reinterpret_cast<const uint4 *>(zs + off);
         const uint4 *vt = reinterpret_cast<const uint4 *>(zt + off);
+        const int yvec = m.z >= 0 ? (m.z >> 3) : -1;     // the vector holding the sampled id
         float ms = -INFINITY, mt = -INFINITY, dd = 0.f;  // dd: reference difference (fp32 gradient)
         float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
         for (int q0 = tid; q0 < nvec; q0 += kHelpU * kHelpThreads) {
@@ -480,6 +517,14 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
                 } else {
                     a[u] = b[u] = make_uint4(kFill, kFill, kFill, kFill);
                 }
+            }
+            // a sampled-token row leaves y out of the student statistics (lowest finite
+            // bf16 in its place; add_sampled_term brings its term back at the merge)
+            if (SM && (unsigned)(yvec - q0) < (unsigned)(kHelpU * kHelpThreads)) {
+#pragma unroll
+                for (int u = 0; u < kHelpU; ++u)
+                    if (yvec == q0 + u * kHelpThreads)
+                        a[u] = fill_lane(a[u], m.z & 7);
             }
             uint32_t bs = hmax4(a[0]), bt = hmax4(b[0]);
 #pragma unroll
@@ -549,9 +594,10 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
             }
             lane_merge<NW, G32>(A, B);
             if (lane == 0) {
+                const int y = m.z;  // SM: in [0, V) (the compaction drops ids out of range); else -1
+                const float omp = SM ? add_sampled_term(A, to_float(zs[off + y])) : 0.f;  // 1 - p_y
                 const RowConst rc = row_const(A, B);
-                const int y = m.z;  // in [0, V) or -1: the compaction drops other rows
-                const float e = y >= 0 ? (to_float(zs[off + y]) - to_float(zt[off + y])) - rc.dl : rc.kl;
+                const float e = SM ? (to_float(zs[off + y]) - to_float(zt[off + y])) - rc.dl : rc.kl;
                 const float wi = __int_as_float(m.w), wl = wi * e;
                 const float sg = wi < 0.f ? -1.f : 1.f;
                 if (!isfinite(rc.lse_s) || !isfinite(rc.lse_t) || !isfinite(e))
@@ -559,11 +605,11 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
                 p.token_loss[m.x] = e;
                 p.row_wl[j] = (double)wi * (double)e;
                 // the gradient constants of the cluster kernel
-                bc[0] = -rc.lse_s * kLog2e + log2f(fabsf(y < 0 ? wi : wl));  // nlw
+                bc[0] = -rc.lse_s * kLog2e + log2f(fabsf(SM ? wl : wi));  // nlw
                 bc[1] = sg;
                 bc[2] = -sg * (rc.d + rc.cp);  // bf16 output: one rounding of d + cp
                 bc[3] = wl > 0.f ? -1.f : 1.f;
-                bc[4] = wl;
+                bc[4] = wl * omp;              // sampled: g_y = w l (1 - p_y)
                 bc[5] = -sg * rc.d;            // fp32 output
                 bc[6] = -sg * rc.cp;
             }
@@ -572,7 +618,7 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
         if (p.grad) {
             const float2 NLW = splat(bc[0]), SG = splat(bc[1]), NC = splat(bc[2]), SGL = splat(bc[3]);
             const float2 ND = splat(bc[5]), NCP = splat(bc[6]);
-            const float wl = bc[4];
+            const float gy = bc[4];
             const int y = m.z;
             for (int q0 = tid; q0 < nvec; q0 += kHelpU * kHelpThreads) {
                 uint4 a[kHelpU], b[kHelpU];
@@ -581,7 +627,7 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
                     const int q = q0 + u * kHelpThreads;
                     if (q < nvec) {
                         a[u] = __ldg(vs + q);
-                        if (y < 0)
+                        if (!SM)
                             b[u] = __ldg(vt + q);
                     }
                 }
@@ -591,27 +637,17 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
                     if (q >= nvec)
                         break;
                     float2 g[4];
-                    if (y < 0) {  // full vocabulary: g = w p ((z_s - z_t) - d - cp)
+                    if (!SM) {  // full vocabulary: g = w p ((z_s - z_t) - d - cp)
 #pragma unroll
                         for (int w = 0; w < 4; ++w) {
                             const float2 a2 = unpack2(word(a[u], w)), b2 = unpack2(word(b[u], w));
                             const float2 pw = ex2x2(ffma2(a2, L2, NLW)), x = fsub2(a2, b2);
                             g[w] = G32 ? fmul2(pw, fadd2(ffma2(x, SG, ND), NCP)) : fmul2(pw, ffma2(x, SG, NC));
                         }
-                    } else {  // sampled token: g = w l (e_y - p)
+                    } else {  // sampled token: g = -w l p (g_y is written after the loop)
 #pragma unroll
                         for (int w = 0; w < 4; ++w)
                             g[w] = fmul2(ex2x2(ffma2(unpack2(word(a[u], w)), L2, NLW)), SGL);
-                        if (q == (y >> 3)) {  // the vector holding y
-                            const int yi = y & 7;
-#pragma unroll
-                            for (int w = 0; w < 4; ++w) {
-                                if (yi == 2 * w)
-                                    g[w].x += wl;
-                                if (yi == 2 * w + 1)
-                                    g[w].y += wl;
-                            }
-                        }
                     }
                     if (G32) {
                         float4 *dst = reinterpret_cast<float4 *>(static_cast<float *>(p.grad) + off) + 2 * (size_t)q;
@@ -627,6 +663,14 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
                     }
                 }
             }
+            // sampled token: g_y = w l (1 - p_y), over the value the vector store wrote
+            // (same thread, so the later store wins)
+            if (SM && (y >> 3) % kHelpThreads == tid) {
+                if (G32)
+                    static_cast<float *>(p.grad)[off + y] = gy;
+                else
+                    static_cast<__nv_bfloat16 *>(p.grad)[off + y] = __float2bfloat16_rn(gy);
+            }
         }
         __syncthreads();  // red and bc are reused by the next row
     }
@@ -640,15 +684,23 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
 #ifndef TURNOPD_ROW_GROUPS
 #define TURNOPD_ROW_GROUPS 2
 #endif
-constexpr int kCS = 8;
 constexpr int kNT = TURNOPD_ROW_THREADS;
 constexpr int kG = TURNOPD_ROW_GROUPS;
 constexpr int kMaxSlice = 2400;                      // vectors per CTA: 3 stages fit 227 KB
 constexpr int kVPT = (kMaxSlice + kNT - 1) / kNT;    // vectors per thread
-// Below this many columns the clusters' slices are too short to hide the per-row
-// record exchange: the helper kernel alone, on every SM, is faster (V = 65,536:
-// 0.72 of the copy bandwidth against 0.58; V = 100,000: 0.68 against 0.73).
-constexpr int64_t kClusterMinVocab = 81920;
+// The cluster size is the smallest of 2, 3, 4, 5, 6, 8 and 16 CTAs whose slices fit
+// three stages, which keeps the slices long (a short slice cannot hide the per-row
+// record exchange) and, for short rows, puts more SMs in clusters (76 pairs cover
+// all 152).  Below kMinSlice vectors per CTA the helper kernel alone, on every SM,
+// takes the rows (measured: slices of 2,000-2,400 vectors reach 0.87-0.93 of the
+// copy bandwidth, the helper alone on rows of up to 8,192 vectors about 0.73).
+// Clusters of 16 are exempt: the rows that need them are long, and the helper
+// alone streams those poorly (V = 200,000: 0.58 against 0.77 with clusters of 16
+// and 1,563-vector slices).
+#ifndef TURNOPD_CLUSTER_MIN_SLICE
+#define TURNOPD_CLUSTER_MIN_SLICE 1700
+#endif
+constexpr int kMinSlice = TURNOPD_CLUSTER_MIN_SLICE;
 constexpr int kSmallRowVec = 7168;  // up to this many vectors per row: 256-thread helpers, 2 per SM
 // The helper's rows per SM and second against the clusters', which decides the
 // split of the row list.  It depends on the clusters' slice length: 0.61 for
@@ -678,24 +730,24 @@ size_t cluster_smem_bytes(int slice_vec, int cs)
     return (size_t)kStages * 2 * slice_vec * 16 + 2 * kG * cs * 8 * sizeof(float) +
            kStages * sizeof(int4) + (2 * kStages + 2 * kG) * sizeof(uint64_t) +
            kG * (kNT / 32) * 8 * sizeof(float) +  // per-group warp partials
-           4 * sizeof(int) +                        // row held by each stage
+           8 * sizeof(int) +                        // row held by each stage, thread reading y
            kG * 16 * sizeof(float);                 // broadcast row constants
 }
 
 // The cluster grid (as many clusters as are co-resident, cached per device) and
 // the helper grid on the SMs the clusters leave free, with the row list split so
 // that both finish together.
-template <bool G32, int CS>
+template <bool G32, int CS, bool SM>
 cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaStream_t stream)
 {
-    auto kern = k_row_cluster<CS, kNT, kVPT, kG, G32>;
+    auto kern = k_row_cluster<CS, kNT, kVPT, kG, G32, SM>;
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess)
         return e;
     static int grid_cache[64][2];
     static size_t smem_cache[64][2];
-    const int gi = G32 ? 1 : 0;  // per instantiation (cluster size and gradient type)
+    const int gi = G32 ? 1 : 0;  // (the statics are per instantiation: cluster size, gradient type, mode)
     if (dev >= 64)
         return cudaErrorInvalidDevice;
     if (smem_cache[dev][gi] < smem) {
@@ -749,7 +801,33 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
     hc.gridDim = dim3(free_sm * kSideBlocks);
     hc.blockDim = dim3(kSideThreads);
     hc.stream = stream;
-    return cudaLaunchKernelEx(&hc, k_row_helper<G32, kSideThreads, kSideBlocks>, pl);
+    return cudaLaunchKernelEx(&hc, k_row_helper<G32, SM, kSideThreads, kSideBlocks>, pl);
+}
+
+// Cluster sizes offered: 7 is left out (only 15 clusters of 7 are co-resident, 105 SMs).
+template <bool G32, bool SM>
+cudaError_t launch_cs(int cs, const RowIn &p, int slice_vec, int nvec, size_t smem, cudaStream_t stream)
+{
+    switch (cs) {
+    case 2: return launch_t<G32, 2, SM>(p, slice_vec, nvec, smem, stream);
+    case 3: return launch_t<G32, 3, SM>(p, slice_vec, nvec, smem, stream);
+    case 4: return launch_t<G32, 4, SM>(p, slice_vec, nvec, smem, stream);
+    case 5: return launch_t<G32, 5, SM>(p, slice_vec, nvec, smem, stream);
+    case 6: return launch_t<G32, 6, SM>(p, slice_vec, nvec, smem, stream);
+    case 8: return launch_t<G32, 8, SM>(p, slice_vec, nvec, smem, stream);
+    default: return launch_t<G32, 16, SM>(p, slice_vec, nvec, smem, stream);
+    }
+}
+
+// The helper kernel alone, every row, every SM.
+template <bool G32, bool SM>
+void launch_helper_alone(const RowIn &p, int nvec, cudaStream_t stream)
+{
+    const int sms = device_sm_count();
+    if (nvec <= kSmallRowVec)
+        k_row_helper<G32, SM, 256, 2><<<sms * 2, 256, 0, stream>>>(p);
+    else
+        k_row_helper<G32, SM><<<sms, kHelpThreads, 0, stream>>>(p);
 }
 
 }  // namespace
@@ -760,27 +838,29 @@ cudaError_t launch_row_cluster(const RowIn &p, bool fp32_grad, cudaStream_t stre
     auto al16 = [](const void *q) { return (reinterpret_cast<uintptr_t>(q) & 15u) == 0; };
     if (p.vocab % 8 != 0 || p.ld % 8 != 0 || !al16(p.zs) || !al16(p.zt) || (p.grad && !al16(p.grad)))
         return cudaSuccess;
-    // clusters of 8, or of 16 (non-portable size) when an eighth of the row does not fit three stages
+    // the smallest cluster whose slices fit three stages (2, 3, 4, 5, 6, 8 or 16 CTAs;
+    // 16 is a non-portable size)
+    if (p.vocab / 8 > (int64_t)0x7fffffff)
+        return cudaSuccess;
     const int nvec = (int)(p.vocab / 8);
-    const int cs = (nvec + kCS - 1) / kCS <= kMaxSlice ? kCS : 2 * kCS;
+    static const int kSizes[] = {2, 3, 4, 5, 6, 8, 16};
+    int cs = 16;
+    for (int c : kSizes)
+        if ((nvec + c - 1) / c <= kMaxSlice) {
+            cs = c;
+            break;
+        }
     const int slice_vec = (nvec + cs - 1) / cs;
+    const bool sm = p.mode == TURNOPD_SAMPLED_TOKEN;
     // short rows, or a slice too long even for clusters of 16: the helper kernel alone, every row, every SM
-    if (p.vocab < kClusterMinVocab || slice_vec > kMaxSlice) {
+    if ((slice_vec < kMinSlice && cs < 16) || slice_vec > kMaxSlice) {
         RowIn pl = p;
         pl.split_den = 0;
-        const int sms = device_sm_count();
         *used = true;
-        if (p.vocab / 8 <= kSmallRowVec) {
-            if (fp32_grad)
-                k_row_helper<true, 256, 2><<<sms * 2, 256, 0, stream>>>(pl);
-            else
-                k_row_helper<false, 256, 2><<<sms * 2, 256, 0, stream>>>(pl);
-        } else {
-            if (fp32_grad)
-                k_row_helper<true><<<sms, kHelpThreads, 0, stream>>>(pl);
-            else
-                k_row_helper<false><<<sms, kHelpThreads, 0, stream>>>(pl);
-        }
+        if (fp32_grad)
+            sm ? launch_helper_alone<true, true>(pl, nvec, stream) : launch_helper_alone<true, false>(pl, nvec, stream);
+        else
+            sm ? launch_helper_alone<false, true>(pl, nvec, stream) : launch_helper_alone<false, false>(pl, nvec, stream);
         return cudaGetLastError();
     }
     const size_t smem = cluster_smem_bytes(slice_vec, cs);
@@ -794,11 +874,11 @@ cudaError_t launch_row_cluster(const RowIn &p, bool fp32_grad, cudaStream_t stre
     if (smem + 64 > (size_t)optin)  // room for the kernel's static shared memory
         return cudaSuccess;
     *used = true;
-    if (cs == kCS)
-        return fp32_grad ? launch_t<true, kCS>(p, slice_vec, nvec, smem, stream)
-                         : launch_t<false, kCS>(p, slice_vec, nvec, smem, stream);
-    return fp32_grad ? launch_t<true, 2 * kCS>(p, slice_vec, nvec, smem, stream)
-                     : launch_t<false, 2 * kCS>(p, slice_vec, nvec, smem, stream);
+    if (fp32_grad)
+        return sm ? launch_cs<true, true>(cs, p, slice_vec, nvec, smem, stream)
+                  : launch_cs<true, false>(cs, p, slice_vec, nvec, smem, stream);
+    return sm ? launch_cs<false, true>(cs, p, slice_vec, nvec, smem, stream)
+              : launch_cs<false, false>(cs, p, slice_vec, nvec, smem, stream);
 }
 
 }  // namespace turnopd

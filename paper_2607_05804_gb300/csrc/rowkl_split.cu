@@ -33,6 +33,7 @@
 // stops waiting, lets its own copies land and returns.
 
 #include <algorithm>
+#include <cfloat>
 
 #include "common.cuh"
 #include "kernels.h"
@@ -85,17 +86,27 @@ __device__ __forceinline__ float lane4(const float4 &v, int i)
     return i == 0 ? v.x : (i == 1 ? v.y : (i == 2 ? v.z : v.w));
 }
 
-// Gradient of one vector (4 columns) from the row constants c (set in
-// `constants` below): g = w p ((z_s - z_t) - d - cp), or w l (e_y - p) with the
-// w l term at column yi (-1: none).
-template <bool G32>
-__device__ __forceinline__ float4 grad4(const float4 &a, const float4 &b, const float *c, bool sampled, int yi)
+// v with lane i replaced by the lowest finite float (never a maximum, adds 0)
+__device__ __forceinline__ float4 fill_lane4(float4 v, int i)
+{
+    v.x = i == 0 ? -FLT_MAX : v.x;
+    v.y = i == 1 ? -FLT_MAX : v.y;
+    v.z = i == 2 ? -FLT_MAX : v.z;
+    v.w = i == 3 ? -FLT_MAX : v.w;
+    return v;
+}
+
+// Gradient of one vector (4 columns) from the row constants c (set by the
+// merge below): g = w p ((z_s - z_t) - d - cp), or -w l p for a sampled-token row
+// (SM; its g_y = w l (1 - p_y) is written apart).
+template <bool G32, bool SM>
+__device__ __forceinline__ float4 grad4(const float4 &a, const float4 &b, const float *c)
 {
     const float2 L2 = splat(kLog2e), NLW = splat(c[0]);
     const float2 a01 = make_float2(a.x, a.y), a23 = make_float2(a.z, a.w);
     const float2 p01 = ex2x2(ffma2(a01, L2, NLW)), p23 = ex2x2(ffma2(a23, L2, NLW));
     float2 g01, g23;
-    if (!sampled) {
+    if (!SM) {
         const float2 SG = splat(c[1]);
         const float2 x01 = fsub2(a01, make_float2(b.x, b.y)), x23 = fsub2(a23, make_float2(b.z, b.w));
         if (G32) {
@@ -111,16 +122,11 @@ __device__ __forceinline__ float4 grad4(const float4 &a, const float4 &b, const 
         const float2 SGL = splat(c[5]);
         g01 = fmul2(p01, SGL);
         g23 = fmul2(p23, SGL);
-        const float wl = c[6];
-        if (yi == 0) g01.x += wl;
-        if (yi == 1) g01.y += wl;
-        if (yi == 2) g23.x += wl;
-        if (yi == 3) g23.y += wl;
     }
     return make_float4(g01.x, g01.y, g23.x, g23.y);
 }
 
-template <bool G32>
+template <bool G32, bool SM>
 __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_vec, int nvec)
 {
     extern __shared__ __align__(128) unsigned char smem[];
@@ -309,15 +315,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
                     if (q0 >= cv)
                         break;
                     const bool v1ok = q1 < cv;
-                    const float4 x0 = cs[q0], z0 = ct[q0];
-                    const float4 x1 = v1ok ? cs[q1] : x0, z1 = v1ok ? ct[q1] : z0;
-                    if (c * kChunkVec + q0 == yq) {
+                    // a sampled-token row leaves y out of the student statistics (lowest
+                    // finite value in its place; add_sampled_term brings its term back at
+                    // the merge)
+                    float4 x0 = cs[q0];
+                    const float4 z0 = ct[q0];
+                    if (SM && c * kChunkVec + q0 == yq) {
                         ysv[0] = lane4(x0, y & 3);
                         ysv[1] = lane4(z0, y & 3);
+                        x0 = fill_lane4(x0, y & 3);
                     }
-                    if (v1ok && c * kChunkVec + q1 == yq) {
+                    float4 x1 = v1ok ? cs[q1] : x0;
+                    const float4 z1 = v1ok ? ct[q1] : z0;
+                    if (SM && v1ok && c * kChunkVec + q1 == yq) {
                         ysv[0] = lane4(x1, y & 3);
                         ysv[1] = lane4(z1, y & 3);
+                        x1 = fill_lane4(x1, y & 3);
                     }
                     // (x1, z1 repeat x0, z0 when the second vector is past the chunk: the
                     // maxima are unchanged and its sums are skipped)
@@ -411,23 +424,23 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
             }
             lane_merge<kCS, true>(A, B);
             if (lane == 0) {
+                const int owner = SM ? (y >> 2) / slice_vec : 0;
+                const float omp = SM ? add_sampled_term(A, r[owner * 8 + 6]) : 0.f;  // 1 - p_y
                 const RowConst rc = row_const(A, B);
                 float e = rc.kl;
-                if (y >= 0) {
-                    const int owner = (y >> 2) / slice_vec;
+                if (SM)
                     e = (r[owner * 8 + 6] - r[owner * 8 + 7]) - rc.dl;
-                }
                 // p |w| = 2^(z_s log2e - LSE_s log2e + log2 |w|); the sign of w enters
                 // through an fma by sg
                 const float wi = __int_as_float(m.w), wl = wi * e;
                 const float sg = wi < 0.f ? -1.f : 1.f;
-                bc[0] = -rc.lse_s * kLog2e + log2f(fabsf(y < 0 ? wi : wl));  // nlw
+                bc[0] = -rc.lse_s * kLog2e + log2f(fabsf(SM ? wl : wi));  // nlw
                 bc[1] = sg;
                 bc[2] = -sg * rc.d;             // fp32 output: d and cp added separately
                 bc[3] = -sg * rc.cp;
                 bc[4] = -sg * (rc.d + rc.cp);   // bf16 output: one rounding of d + cp
                 bc[5] = wl > 0.f ? -1.f : 1.f;  // sampled: sign of -w l
-                bc[6] = wl;
+                bc[6] = wl * omp;               // sampled: g_y = w l (1 - p_y)
                 if (rank == 0) {
                     if (!isfinite(rc.lse_s) || !isfinite(rc.lse_t) || !isfinite(e))
                         set_status(p.status, TURNOPD_ERR_NONFINITE);
@@ -454,12 +467,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
                         const int ql = gtid + u * kNT;
                         if (ql < cv) {
                             const int q = c * kChunkVec + ql;
-                            const float4 a = ga[ql], b = y < 0 ? gb[ql] : a;
+                            const float4 a = ga[ql], b = SM ? a : gb[ql];
                             if (kKeep && (ql & 7) == 0) {  // one thread per 128-byte line of each model
                                 l2_evict_normal(zs + off + (size_t)q * 4);
                                 l2_evict_normal(zt + off + (size_t)q * 4);
                             }
-                            const float4 g4 = grad4<G32>(a, b, bc, y >= 0, q == yq ? (y & 3) : -1);
+                            const float4 g4 = grad4<G32, SM>(a, b, bc);
                             if (G32) {
                                 __stcs(reinterpret_cast<float4 *>(static_cast<float *>(p.grad) + off) + q, g4);
                             } else {
@@ -474,6 +487,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
                 __syncwarp();
                 if (lane == 0)
                     mbar_arrive(&gempty[s]);
+            }
+            // sampled token: g_y = w l (1 - p_y), over the value the vector store wrote
+            // (the thread that stored y's vector, so the later store wins)
+            if (SM && yq >= 0 && yq < my_vec && yq % kNT == gtid) {
+                const size_t yo = (size_t)m.y * (size_t)p.ld + (size_t)y;
+                if (G32)
+                    static_cast<float *>(p.grad)[yo] = bc[6];
+                else
+                    static_cast<__nv_bfloat16 *>(p.grad)[yo] = __float2bfloat16_rn(bc[6]);
             }
         }
         m = m_next;
@@ -496,15 +518,17 @@ cudaError_t launch_row_split(const RowIn &p, bool fp32_grad, cudaStream_t stream
         return cudaSuccess;
     const int nvec = (int)(p.vocab / 4);
     const int slice_vec = (nvec + kCS - 1) / kCS;
-    auto kern = fp32_grad ? k_row_split<true> : k_row_split<false>;
+    const bool sm = p.mode == TURNOPD_SAMPLED_TOKEN;  // every listed row then carries y in [0, V)
+    auto kern = fp32_grad ? (sm ? k_row_split<true, true> : k_row_split<true, false>)
+                          : (sm ? k_row_split<false, true> : k_row_split<false, false>);
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess)
         return e;
     if (dev >= 64)
         return cudaErrorInvalidDevice;
-    static int grid_cache[64][2];
-    const int gi = fp32_grad ? 1 : 0;
+    static int grid_cache[64][4];
+    const int gi = (fp32_grad ? 1 : 0) + (sm ? 2 : 0);  // per instantiation: attributes are per kernel
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;

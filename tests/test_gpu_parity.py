@@ -54,8 +54,10 @@ def bits_or_f32(z):
 
 
 def run_chain(P, oracle, b, V, zs, zt, *, mode, alpha, flags=0, grad_dtype=None, compact=False,
-              scope=0, n_min=0, seed_y=1):
-    """GPU chain vs oracle chain on every row of the batch."""
+              scope=0, n_min=0, seed_y=1, y_rel=None):
+    """GPU chain vs oracle chain on every row of the batch.  y_rel (sampled mode): also
+    hold each row's g_y = w l (1 - p_y) to y_rel of the oracle's (after the l rescaling);
+    returns the oracle's 1 - p_y of the rows as a third value then."""
     y = per_token_ids(b, W.sample_ids(zs, seed_y, V), compact) if mode == 1 else None
     step = make_step(P, b, V, compact=compact, mode=mode, alpha=alpha, flags=flags, y=y,
                      scope=scope, n_min=n_min)
@@ -83,9 +85,24 @@ def run_chain(P, oracle, b, V, zs, zt, *, mode, alpha, flags=0, grad_dtype=None,
     assert_grad_rows(g[rows][:, :V], g_ref[rows], bf16=(gdt == torch.bfloat16),
                      zs=zs[rsel, :V], w=w_ref.astype(np.float32)[toks], ell=tl_ref[toks],
                      ell_gpu=tl[toks], sampled=(mode == 1))
+    omp = None
+    if y_rel is not None:
+        assert mode == 1
+        yk = ynp[toks].astype(np.int64)
+        gy, gy_ref = g[rows, yk], g_ref[rows, yk]
+        wl_ref = w_ref.astype(np.float32)[toks].astype(np.float64) * tl_ref[toks]
+        nz = wl_ref != 0
+        omp = gy_ref[nz] / wl_ref[nz]
+        ref = gy_ref[nz] * (tl[toks][nz] / tl_ref[toks][nz])
+        err = np.abs(gy[nz] - ref)
+        assert (err <= y_rel * np.abs(ref)).all(), (
+            f"g_y off: worst relative {float((err / np.abs(ref)).max()):.3g} at 1 - p_y = "
+            f"{float(omp[np.argmax(err / np.abs(ref))]):.3g}")
     st_ref = oracle.turn_stats(tl_ref, b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns)
     st = {k: v.cpu().numpy() for k, v in step.stats().items()}
     assert_stats(st, st_ref, tl_ref, b.turn_id, b.loss_mask, b.traj_offsets, b.max_turns)
+    if y_rel is not None:
+        return step, grad, omp
     return step, grad
 
 
@@ -158,17 +175,45 @@ def test_paper_turn_floor_on_household(P, oracle):
 
 # ---------------------------------------------------------------- cluster kernel, all rows
 
-@pytest.mark.parametrize("V", [50000, W.V_QWEN, 262144])
+@pytest.mark.parametrize("V", [8192, 32000, 50000, W.V_QWEN, 200000, 262144])
 @pytest.mark.parametrize("mode", [0, 1], ids=["full", "sampled"])
 @pytest.mark.parametrize("gdt", ["bf16", "f32"])
 def test_cluster_kernel_all_rows(P, oracle, V, mode, gdt):
-    """The bf16 row path on every row (vocabulary a multiple of 8): V = 50,000 takes the
-    helper kernel alone, V = 151,936 clusters of 8 beside it (ragged last slice), and
-    V = 262,144 clusters of 16 beside it."""
+    """The bf16 row path on every row (vocabulary a multiple of 8): V = 8,192 takes the
+    helper kernel alone, V = 32,000 clusters of 2 on every SM, V = 50,000 clusters of 3
+    beside the helper (ragged last slice), V = 151,936 clusters of 8 beside it, and
+    V = 200,000 and 262,144 clusters of 16 beside it (200,000: slices of 1,563 vectors,
+    the shortest the clusters of 16 take)."""
     b = W.packed(seed=11, num_traj=2, traj_len=256)
     zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=12, device="cuda")
     run_chain(P, oracle, b, V, zs, zt, mode=mode, alpha=0.5, compact=True,
               grad_dtype=torch.bfloat16 if gdt == "bf16" else torch.float32)
+
+
+@pytest.mark.parametrize("kernel,V,idt,flags", [
+    ("helper alone", 8192, "bf16", 0), ("clusters of 2", 32000, "bf16", 0),
+    ("clusters of 8 + helper", W.V_QWEN, "bf16", 0), ("split rows", 4100, "f32", 0),
+    ("split rows", W.V_QWEN, "f32", 0), ("portable", 4099, "bf16", FORCE_PORTABLE),
+    ("portable", 4100, "f32", FORCE_PORTABLE)])
+@pytest.mark.parametrize("gdt", ["bf16", "f32"])
+def test_sampled_peaked_rows(P, oracle, kernel, V, idt, flags, gdt):
+    """Sampled-token rows whose student logit at y stands delta = 0 ... 30 above the rest
+    of the row, so that p_y runs from ordinary values to within ~1e-9 of 1: every row
+    path keeps g_y = w l (1 - p_y) to fp32 relative precision (a gradient formed as
+    w l - w l p_y keeps no digit of it there).  Raising z_s at the Gumbel-max sample
+    keeps it the sample, so run_chain draws the same y."""
+    b = W.packed(seed=41, num_traj=2, traj_len=256)
+    dt = torch.bfloat16 if idt == "bf16" else torch.float32
+    zs, zt = W.make_logits(b.num_valid, V, "agent", dt, seed=42, device="cuda")
+    y = W.sample_ids(zs, 43, V).long()
+    r = torch.arange(b.num_valid, device="cuda")
+    delta = torch.tensor([0.0, 3.0, 6.0, 10.0, 15.0, 20.0, 25.0, 30.0], device="cuda")[r % 8]
+    zs[r, y] = (zs[:, :V].float().amax(dim=1) + delta).to(dt)
+    assert torch.equal(W.sample_ids(zs, 43, V).long(), y)
+    gd = torch.bfloat16 if gdt == "bf16" else torch.float32
+    out = run_chain(P, oracle, b, V, zs, zt, mode=1, alpha=0.5, flags=flags, compact=True,
+                    grad_dtype=gd, seed_y=43, y_rel=(1e-4 if gdt == "f32" else 2.0 ** -7))
+    assert out[2].min() < 1e-8  # the test reaches p_y within 1e-8 of 1
 
 
 @pytest.mark.parametrize("V,ld", [(4100, 4100), (4100, 4104), (W.V_QWEN, W.V_QWEN), (262144, 262144)])
