@@ -610,8 +610,10 @@ def main():
                            "+ compaction + loss sum)"),
                 "algorithmic_bytes_per_launch": alg_bytes,
                 "launch_ms": loss_avg_ms,
+                # the committed records cover the full-vocabulary bf16-gradient row grids and the
+                # top-K kernel at V = 151,936; any other instantiation or byte count has none
                 "traffic": (None if (args.vocab_shards or dense_layout(args) or args.fp32_logits
-                                     or V != V_QWEN)
+                                     or V != V_QWEN or args.fp32_grad or args.mode == "sampled")
                             else committed_traffic(args.workload, R, "topk") if args.mode == "topk"
                             else committed_traffic(args.workload)),
             },
