@@ -37,7 +37,8 @@ METRIC = "loss fwd+bwd tokens/s at V=151936 bf16 on 1 GB300; achieved HBM GB/s v
 UNIT = "tokens/s"
 V_QWEN = 151_936  # the workloads' vocabulary (a --vocab run has no committed traffic record)
 # counts(2) + weights(1) + compaction(2) + row kernel + loss sum + stats(2); the full and
-# sampled modes on bf16 logits add the helper grid that runs beside the cluster grid
+# sampled modes add the helper grid that runs beside the cluster grid (k_row_helper for
+# bf16 logits, k_split_helper for fp32)
 KERNELS_PER_STEP = 9
 ROW_KERNEL_SOURCES = ["paper_2607_05804_gb300/csrc/rowkl_cluster.cu",
                       "paper_2607_05804_gb300/csrc/loss_kernels.cu",
@@ -604,8 +605,9 @@ def main():
                            if args.mode == "topk" else
                            f"vocabulary-parallel path, {args.vocab_shards} shards of one GPU "
                            "(shard stats + merge + shard gradients)" if args.vocab_shards else
-                           "turnopd_loss_fwd_bwd launch sequence (split-row kernel on clusters of 4 "
-                           "+ compaction + loss sum)" if args.fp32_logits else
+                           "turnopd_loss_fwd_bwd launch sequence (split-row kernel on clusters of "
+                           f"{4 if args.mode == 'sampled' else 8} beside the fp32 helper grid + compaction "
+                           "+ loss sum)" if args.fp32_logits else
                            "turnopd_loss_fwd_bwd launch sequence (cluster row kernel beside the helper grid "
                            "+ compaction + loss sum)"),
                 "algorithmic_bytes_per_launch": alg_bytes,
@@ -620,7 +622,7 @@ def main():
             # vocabulary shards: counts(2) + weights(1) + per shard the statistics call (compaction(2),
             # statistics) and the gradient call (compaction(2), gradient, loss sum) + merge + stats(2)
             "gpu_launches": ((KERNELS_PER_STEP + (1 if args.zero_masked else 0)
-                              + (0 if args.mode == "topk" or args.fp32_logits else 1))
+                              + (0 if args.mode == "topk" else 1))
                              if not args.vocab_shards
                              else 6 + 7 * args.vocab_shards) * args.steps,
             "clocks": clocks,

@@ -3,10 +3,13 @@
 // One fp32 logit row of V = 151,936 values is 607,744 bytes per model, so the
 // two rows of a token (1.2 MB) fit no SM, and one row in flight per SM would
 // ask 185 MB of the 126 MB L2 for the gradient pass's second read.  A cluster
-// of kCS CTAs therefore shares every row: CTA c owns the c-th quarter of the
-// columns (its slice), and the 36 co-resident clusters keep 36 rows in flight.
-// The gradient's second read of a chunk follows its first within about one
-// row's statistics, so it mostly hits L2.
+// of CS CTAs therefore shares every row: CTA c owns the c-th of CS column slices.
+// Full-vocabulary rows take clusters of 8 (15 co-resident, 120 SMs, two rows in
+// flight each: 36 MB of rows between their first and second reads); sampled-token
+// rows, whose second read carries the student only, clusters of 4 (36 co-resident,
+// 144 SMs).  The SMs the clusters leave free run k_split_helper on a share of the
+// rows.  The gradient's second read of a chunk follows its first within about
+// one row's statistics, so it mostly hits L2.
 //
 // Per CTA (persistent, one per SM, rows cid, cid + nclusters, ...):
 //   * a producer warp streams the slice, both models, through a ring of
@@ -21,7 +24,7 @@
 //     across the CTA in a fixed lane order and push the CTA's 32-byte record
 //     to every CTA of the cluster (st.async into a record ring, completion on
 //     the receiver's mbarrier: no cluster barrier per row);
-//   * every CTA merges the kCS records in the same fixed order, so all use
+//   * every CTA merges the CS records in the same fixed order, so all use
 //     bit-identical LSE and KL (deterministic), then writes the gradient of its
 //     slice, g = w p_s ((z_s - z_t) - LSE_s + LSE_t - KL) (full vocabulary) or
 //     g = w l (e_y - p_s) (sampled token), from the slice read again -- from L2,
@@ -44,10 +47,17 @@
 namespace turnopd {
 namespace {
 
-#ifndef TURNOPD_SPLIT_CS
-#define TURNOPD_SPLIT_CS 4
+// CTAs per row: full vocabulary / sampled token (measured on the packed 8 x 4096 fp32
+// batch with the helper grid at split rate 0.6: full 6.53 ms with clusters of 8, 6.98
+// with 4 (6.83 with 4 and no helper); sampled 6.10 with 4, 6.55 with 8)
+#ifndef TURNOPD_SPLIT_CS_FULL
+#define TURNOPD_SPLIT_CS_FULL 8
 #endif
-constexpr int kCS = TURNOPD_SPLIT_CS;           // CTAs per row
+#ifndef TURNOPD_SPLIT_CS_SAMPLED
+#define TURNOPD_SPLIT_CS_SAMPLED 4
+#endif
+constexpr int kCSFull = TURNOPD_SPLIT_CS_FULL;
+constexpr int kCSSampled = TURNOPD_SPLIT_CS_SAMPLED;
 constexpr int kG = 2;                           // row groups per CTA (alternate rows)
 constexpr int kNT = 256;                        // threads per group
 constexpr int kNWG = kNT / 32;                  // warps per group
@@ -69,17 +79,46 @@ constexpr int kGStages = 7 - kSStages;          // chunks read again for the gra
 // back to normal priority.  Forward-only calls (no second read) leave the
 // default priority.
 constexpr bool kKeep = TURNOPD_SPLIT_KEEP != 0;
+// The helper grid on the SMs the clusters leave free (k_split_helper): vectors per
+// model and thread in one batch, threads per CTA, and its rows per second per SM
+// against a cluster SM's, which sets the split of the row list (measured on the
+// packed 8 x 4096 fp32 batch: full vocabulary 6.66 / 6.56 / 6.45 / 6.68 / 7.04 ms at
+// 0.5 / 0.6 / 0.7 / 0.8 / 0.9; sampled 6.15 / 6.11 / 6.41 ms at 0.45 / 0.6 / 0.8;
+// batches of 8 vectors no faster than 4).
+#ifndef TURNOPD_SPLIT_HELPER
+#define TURNOPD_SPLIT_HELPER 1
+#endif
+#ifndef TURNOPD_SPLIT_RATE_FULL
+#define TURNOPD_SPLIT_RATE_FULL 0.7
+#endif
+#ifndef TURNOPD_SPLIT_RATE_SAMPLED
+#define TURNOPD_SPLIT_RATE_SAMPLED 0.6
+#endif
+#ifndef TURNOPD_SPLIT_HELPER_U
+#define TURNOPD_SPLIT_HELPER_U 4
+#endif
+#ifndef TURNOPD_SPLIT_HELPER_THREADS
+#define TURNOPD_SPLIT_HELPER_THREADS 512
+#endif
+constexpr bool kSplitHelper = TURNOPD_SPLIT_HELPER != 0;
+constexpr double kRateFull = TURNOPD_SPLIT_RATE_FULL;
+constexpr double kRateSampled = TURNOPD_SPLIT_RATE_SAMPLED;
+constexpr int kHelperU = TURNOPD_SPLIT_HELPER_U;
+constexpr int kHelperThreads = TURNOPD_SPLIT_HELPER_THREADS;
 constexpr int kSlots = 2 * kG;                  // record ring
 constexpr uint32_t kWaitLimit = 1u << 22;       // mbarrier polls before giving up
 constexpr uint32_t kStageBytes = 2u * kChunkVec * 16u;
 
-constexpr size_t kSmemBytes = (size_t)(kSStages + kGStages) * kStageBytes  // the two rings
-                              + kSlots * kCS * 8 * sizeof(float)             // records
-                              + (2 * kSStages + 2 * kGStages + kSlots) * sizeof(uint64_t)
-                              + (kSStages + kGStages) * sizeof(uint32_t)     // chunk held by each stage
-                              + kG * kNWG * 8 * sizeof(float)                // per-warp partials
-                              + kG * 8 * sizeof(float)                       // row constants
-                              + kG * 2 * sizeof(float);                      // sampled-token logits
+constexpr size_t split_smem_bytes(int cs)
+{
+    return (size_t)(kSStages + kGStages) * kStageBytes  // the two rings
+           + kSlots * cs * 8 * sizeof(float)             // records
+           + (2 * kSStages + 2 * kGStages + kSlots) * sizeof(uint64_t)
+           + (kSStages + kGStages) * sizeof(uint32_t)    // chunk held by each stage
+           + kG * kNWG * 8 * sizeof(float)               // per-warp partials
+           + kG * 8 * sizeof(float)                      // row constants
+           + kG * 2 * sizeof(float);                     // sampled-token logits
+}
 
 __device__ __forceinline__ float lane4(const float4 &v, int i)
 {
@@ -126,15 +165,15 @@ __device__ __forceinline__ float4 grad4(const float4 &a, const float4 &b, const 
     return make_float4(g01.x, g01.y, g23.x, g23.y);
 }
 
-template <bool G32, bool SM>
+template <int CS, bool G32, bool SM>
 __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_vec, int nvec)
 {
     extern __shared__ __align__(128) unsigned char smem[];
     __shared__ int s_dead;
     float4 *sring = reinterpret_cast<float4 *>(smem);                       // [kSStages][2][kChunkVec]
     float4 *gring = sring + (size_t)kSStages * 2 * kChunkVec;              // [kGStages][2][kChunkVec]
-    float *rec = reinterpret_cast<float *>(gring + (size_t)kGStages * 2 * kChunkVec);  // [kSlots][kCS][8]
-    uint64_t *sfull = reinterpret_cast<uint64_t *>(rec + kSlots * kCS * 8);  // [kSStages]
+    float *rec = reinterpret_cast<float *>(gring + (size_t)kGStages * 2 * kChunkVec);  // [kSlots][CS][8]
+    uint64_t *sfull = reinterpret_cast<uint64_t *>(rec + kSlots * CS * 8);  // [kSStages]
     uint64_t *sempty = sfull + kSStages;                                     // [kSStages]
     uint64_t *gfull = sempty + kSStages;                                     // [kGStages]
     uint64_t *gempty = gfull + kGStages;                                     // [kGStages]
@@ -170,12 +209,17 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
         for (int s = 0; s < kSlots; ++s)
-            mbar_arrive_expect_tx(&recv[s], kCS * 32u);  // first record of each slot
+            mbar_arrive_expect_tx(&recv[s], CS * 32u);  // first record of each slot
     }
     __syncthreads();
     cluster_sync();  // peers' barriers are initialised before any record is sent
+    // Every CTA of this grid is resident: a helper grid launched after this one may
+    // start now, on the SMs the clusters left free.
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-    const int nv = *p.nvalid;
+    // split_den > 0: the clusters take rows [0, nvalid split_num / split_den) of the list
+    const int nv_all = *p.nvalid;
+    const int nv = p.split_den ? (int)((int64_t)nv_all * p.split_num / p.split_den) : nv_all;
     const int n = nv > cid ? (nv - cid + ncl - 1) / ncl : 0;  // same for the whole cluster
     if (n == 0)
         return;
@@ -403,26 +447,26 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
             A.d = __shfl_sync(0xffffffffu, A.d, 0);
             B.m = __shfl_sync(0xffffffffu, B.m, 0);
             B.s = __shfl_sync(0xffffffffu, B.s, 0);
-            if (lane < kCS) {
+            if (lane < CS) {
                 const bool mine = yq >= 0 && yq < my_vec;
                 const float ys = mine ? ysv[0] : 0.f, yt = mine ? ysv[1] : 0.f;
-                const uint32_t ra = mapa(smem_u32(rec + (slot * kCS + (int)rank) * 8), (uint32_t)lane);
+                const uint32_t ra = mapa(smem_u32(rec + (slot * CS + (int)rank) * 8), (uint32_t)lane);
                 const uint32_t rbar = mapa(smem_u32(&recv[slot]), (uint32_t)lane);
                 st_async16(ra, rbar, make_float4(A.m, A.s, A.a, A.d));
                 st_async16(ra + 16, rbar, make_float4(B.m, B.s, ys, yt));
             }
-            // the row's constants from the kCS records, in the same order in every CTA
+            // the row's constants from the CS records, in the same order in every CTA
             wait_bar(&recv[slot], (uint32_t)((k / kSlots) & 1), true);
-            const float *r = rec + slot * kCS * 8;
+            const float *r = rec + slot * CS * 8;
             A = student_empty();
             B = teacher_empty();
-            if (lane < kCS) {
+            if (lane < CS) {
                 const float4 x = *reinterpret_cast<const float4 *>(r + lane * 8);
                 const float4 z = *reinterpret_cast<const float4 *>(r + lane * 8 + 4);
                 A = Student{x.x, x.y, x.z, x.w};
                 B = Teacher{z.x, z.y};
             }
-            lane_merge<kCS, true>(A, B);
+            lane_merge<CS, true>(A, B);
             if (lane == 0) {
                 const int owner = SM ? (y >> 2) / slice_vec : 0;
                 const float omp = SM ? add_sampled_term(A, r[owner * 8 + 6]) : 0.f;  // 1 - p_y
@@ -447,7 +491,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
                     p.token_loss[m.x] = e;
                     p.row_wl[cid + k * ncl] = (double)wi * (double)e;
                 }
-                mbar_arrive_expect_tx(&recv[slot], kCS * 32u);  // re-arm for row k + kSlots
+                mbar_arrive_expect_tx(&recv[slot], CS * 32u);  // re-arm for row k + kSlots
             }
         }
         group_sync();
@@ -503,11 +547,253 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
     cluster_sync();  // no CTA leaves while a peer may still address its shared memory
 }
 
+
+// Helper for the SMs the clusters leave free, fp32 logits: one CTA per row at a time,
+// rows j0 + blockIdx.x, j0 + blockIdx.x + gridDim.x, ... of the row list (j0 = the
+// cluster grid's share).  The statistics pass streams both rows from HBM in batches of
+// U vectors per model and thread, with a running maximum per thread (one rescale per
+// batch when it moves) and A relative to the reference difference d at the running
+// student argmax, as the cluster kernel keeps it; the gradient pass reads the row
+// again from L2.  Launched as a dependent of the cluster grid (it starts once every
+// cluster is resident) and completes only after it.
+template <bool G32, bool SM, int U, int NTH>
+__global__ void __launch_bounds__(NTH, 1) k_split_helper(RowIn p)
+{
+    constexpr int NW = NTH / 32;
+    __shared__ float red[NW][8];
+    __shared__ float bc[8];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int nvalid = *p.nvalid;
+    const int j0 = p.split_den ? (int)((int64_t)nvalid * p.split_num / p.split_den) : 0;
+    const int nvec = (int)(p.vocab / 4);
+    const float *zs = static_cast<const float *>(p.zs);
+    const float *zt = static_cast<const float *>(p.zt);
+    const float2 L2 = splat(kLog2e);
+    const float4 kFill4 = make_float4(-FLT_MAX, -FLT_MAX, -FLT_MAX, -FLT_MAX);
+    for (int j = j0 + (int)blockIdx.x; j < nvalid; j += gridDim.x) {
+        const int4 m = p.rows[j];
+        const size_t off = (size_t)m.y * (size_t)p.ld;
+        const float4 *vs = reinterpret_cast<const float4 *>(zs + off);
+        const float4 *vt = reinterpret_cast<const float4 *>(zt + off);
+        const int yvec = SM ? (m.z >> 2) : -1;  // the vector holding the sampled id
+        float ms = -INFINITY, mt = -INFINITY, dd = 0.f;
+        float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
+        for (int q0 = tid; q0 < nvec; q0 += U * NTH) {
+            float4 a[U], b[U];
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const int q = q0 + u * NTH;
+                if (q < nvec) {
+                    a[u] = __ldg(vs + q);
+                    b[u] = __ldg(vt + q);
+                } else {
+                    a[u] = b[u] = kFill4;  // adds 0, never the maximum
+                }
+            }
+            // a sampled-token row leaves y out of the student statistics (lowest finite
+            // value in its place; add_sampled_term brings its term back at the merge)
+            if (SM && (unsigned)(yvec - q0) < (unsigned)(U * NTH)) {
+#pragma unroll
+                for (int u = 0; u < U; ++u)
+                    if (yvec == q0 + u * NTH)
+                        a[u] = fill_lane4(a[u], m.z & 3);
+            }
+            float cm = fmaxf(fmaxf(a[0].x, a[0].y), fmaxf(a[0].z, a[0].w));
+            float cmt = fmaxf(fmaxf(b[0].x, b[0].y), fmaxf(b[0].z, b[0].w));
+#pragma unroll
+            for (int u = 1; u < U; ++u) {
+                cm = fmaxf(cm, fmaxf(fmaxf(a[u].x, a[u].y), fmaxf(a[u].z, a[u].w)));
+                cmt = fmaxf(cmt, fmaxf(fmaxf(b[u].x, b[u].y), fmaxf(b[u].z, b[u].w)));
+            }
+            if (cm > ms) {
+                // reference difference at the first element of the batch equal to the new maximum
+                float xd = 0.f;
+                bool found = false;
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    if (!found && a[u].x == cm) { xd = a[u].x - b[u].x; found = true; }
+                    if (!found && a[u].y == cm) { xd = a[u].y - b[u].y; found = true; }
+                    if (!found && a[u].z == cm) { xd = a[u].z - b[u].z; found = true; }
+                    if (!found && a[u].w == cm) { xd = a[u].w - b[u].w; found = true; }
+                }
+                const float2 f = splat(ex2((ms - cm) * kLog2e));
+                A2 = fmul2(ffma2(S2, splat(dd - xd), A2), f);
+                S2 = fmul2(S2, f);
+                dd = xd;
+                ms = cm;
+            }
+            if (cmt > mt) {
+                T2 = fmul2(T2, splat(ex2((mt - cmt) * kLog2e)));
+                mt = cmt;
+            }
+            const float2 NS = splat(-ms * kLog2e), NTT = splat(-mt * kLog2e), D = splat(dd);
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+                const float2 a01 = make_float2(a[u].x, a[u].y), a23 = make_float2(a[u].z, a[u].w);
+                const float2 b01 = make_float2(b[u].x, b[u].y), b23 = make_float2(b[u].z, b[u].w);
+                const float2 e01 = ex2x2(ffma2(a01, L2, NS)), e23 = ex2x2(ffma2(a23, L2, NS));
+                S2 = fadd2(S2, fadd2(e01, e23));
+                A2 = ffma2(e01, fsub2(fsub2(a01, b01), D), A2);
+                A2 = ffma2(e23, fsub2(fsub2(a23, b23), D), A2);
+                T2 = fadd2(T2, fadd2(ex2x2(ffma2(b01, L2, NTT)), ex2x2(ffma2(b23, L2, NTT))));
+            }
+        }
+        Student S = ms == -INFINITY ? student_empty() : Student{ms, S2.x + S2.y, A2.x + A2.y, dd};
+        Teacher T = mt == -INFINITY ? teacher_empty() : Teacher{mt, T2.x + T2.y};
+        lane_merge<32, true>(S, T);
+        if (lane == 0) {
+            red[warp][0] = S.m, red[warp][1] = S.s, red[warp][2] = S.a, red[warp][3] = S.d;
+            red[warp][4] = T.m, red[warp][5] = T.s;
+        }
+        __syncthreads();
+        if (warp == 0) {
+            Student A = student_empty();
+            Teacher B = teacher_empty();
+            if (lane < NW) {
+                A = Student{red[lane][0], red[lane][1], red[lane][2], red[lane][3]};
+                B = Teacher{red[lane][4], red[lane][5]};
+            }
+            lane_merge<NW, true>(A, B);
+            if (lane == 0) {
+                const int y = m.z;  // SM: in [0, V) (the compaction drops ids out of range); else -1
+                const float zy = SM ? zs[off + y] : 0.f;
+                const float omp = SM ? add_sampled_term(A, zy) : 0.f;  // 1 - p_y
+                const RowConst rc = row_const(A, B);
+                const float e = SM ? (zy - zt[off + y]) - rc.dl : rc.kl;
+                const float wi = __int_as_float(m.w), wl = wi * e;
+                const float sg = wi < 0.f ? -1.f : 1.f;
+                if (!isfinite(rc.lse_s) || !isfinite(rc.lse_t) || !isfinite(e))
+                    set_status(p.status, TURNOPD_ERR_NONFINITE);
+                p.token_loss[m.x] = e;
+                p.row_wl[j] = (double)wi * (double)e;
+                // the row constants of grad4, as the cluster kernel sets them
+                bc[0] = -rc.lse_s * kLog2e + log2f(fabsf(SM ? wl : wi));  // nlw
+                bc[1] = sg;
+                bc[2] = -sg * rc.d;
+                bc[3] = -sg * rc.cp;
+                bc[4] = -sg * (rc.d + rc.cp);
+                bc[5] = wl > 0.f ? -1.f : 1.f;
+                bc[6] = wl * omp;  // sampled: g_y = w l (1 - p_y)
+            }
+        }
+        __syncthreads();
+        if (p.grad) {
+            float c[7];
+#pragma unroll
+            for (int i = 0; i < 7; ++i)
+                c[i] = bc[i];
+            for (int q0 = tid; q0 < nvec; q0 += U * NTH) {
+                float4 a[U], b[U];
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    const int q = q0 + u * NTH;
+                    if (q < nvec) {
+                        a[u] = __ldg(vs + q);
+                        b[u] = SM ? a[u] : __ldg(vt + q);
+                    }
+                }
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    const int q = q0 + u * NTH;
+                    if (q >= nvec)
+                        break;
+                    const float4 g4 = grad4<G32, SM>(a[u], b[u], c);
+                    if (G32) {
+                        __stcs(reinterpret_cast<float4 *>(static_cast<float *>(p.grad) + off) + q, g4);
+                    } else {
+                        uint2 o;
+                        o.x = pack_bf16x2(g4.x, g4.y);
+                        o.y = pack_bf16x2(g4.z, g4.w);
+                        __stcs(reinterpret_cast<uint2 *>(static_cast<__nv_bfloat16 *>(p.grad) + off) + q, o);
+                    }
+                }
+            }
+            // sampled token: g_y = w l (1 - p_y), over the value the vector store wrote
+            // (same thread, so the later store wins)
+            if (SM && yvec % NTH == tid) {
+                if (G32)
+                    static_cast<float *>(p.grad)[off + m.z] = c[6];
+                else
+                    static_cast<__nv_bfloat16 *>(p.grad)[off + m.z] = __float2bfloat16_rn(c[6]);
+            }
+        }
+        __syncthreads();  // red and bc are reused by the next row
+    }
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // complete only after the cluster grid
+}
+
+// The cluster grid (as many clusters of CS as are co-resident, cached per device)
+// and the helper grid on the SMs the clusters leave free.
+template <int CS, bool SM>
+cudaError_t launch_split_t(const RowIn &p, bool fp32_grad, int nvec, double rate, cudaStream_t stream)
+{
+    constexpr size_t kSmem = split_smem_bytes(CS);
+    const int slice_vec = (nvec + CS - 1) / CS;
+    auto kern = fp32_grad ? k_row_split<CS, true, SM> : k_row_split<CS, false, SM>;
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess)
+        return e;
+    if (dev >= 64)
+        return cudaErrorInvalidDevice;
+    static int grid_cache[64][2];  // per instantiation (cluster size, mode) and gradient type
+    const int gi = fp32_grad ? 1 : 0;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CS;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = kSmem;
+    cfg.stream = stream;
+    if (grid_cache[dev][gi] == 0) {
+        if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmem)) != cudaSuccess)
+            return e;
+        if (CS > 8 && (e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) != cudaSuccess)
+            return e;
+        cfg.gridDim = dim3(CS);
+        int ncl = 0;
+        if ((e = cudaOccupancyMaxActiveClusters(&ncl, kern, &cfg)) != cudaSuccess)
+            return e;
+        if (ncl < 1)
+            return cudaErrorInvalidConfiguration;
+        grid_cache[dev][gi] = ncl;
+    }
+    cfg.gridDim = dim3(grid_cache[dev][gi] * CS);
+    // the helper grid on the SMs the clusters leave free, with the row list split so
+    // that both grids finish together
+    RowIn pl = p;
+    const int free_sm = kSplitHelper ? device_sm_count() - grid_cache[dev][gi] * CS : 0;
+    if (free_sm > 0) {
+        const double cl = (double)(grid_cache[dev][gi] * CS);
+        pl.split_den = 1 << 20;
+        pl.split_num = (int32_t)(pl.split_den * cl / (cl + rate * free_sm) + 0.5);
+    }
+    e = cudaLaunchKernelEx(&cfg, kern, pl, slice_vec, nvec);
+    if (e != cudaSuccess || pl.split_den == 0)
+        return e;
+    cudaLaunchConfig_t hc = {};
+    cudaLaunchAttribute ha[1];
+    ha[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    ha[0].val.programmaticStreamSerializationAllowed = 1;
+    hc.attrs = ha;
+    hc.numAttrs = 1;
+    hc.gridDim = dim3(free_sm);
+    hc.blockDim = dim3(kHelperThreads);
+    hc.stream = stream;
+    auto helper = fp32_grad ? k_split_helper<true, SM, kHelperU, kHelperThreads>
+                            : k_split_helper<false, SM, kHelperU, kHelperThreads>;
+    return cudaLaunchKernelEx(&hc, helper, pl);
+}
+
 }  // namespace
 
 // fp32 logits, 16-byte aligned rows (V and ld multiples of 4): the split-row
-// kernel on as many clusters as are co-resident.  *used = false leaves the row
-// to the portable kernel.
+// kernel on as many clusters as are co-resident, the helper kernel beside it.
+// *used = false leaves the row to the portable kernel.
 cudaError_t launch_row_split(const RowIn &p, bool fp32_grad, cudaStream_t stream, bool *used)
 {
     *used = false;
@@ -517,46 +803,11 @@ cudaError_t launch_row_split(const RowIn &p, bool fp32_grad, cudaStream_t stream
     if (p.vocab / 4 > (int64_t)0x7fffffff)
         return cudaSuccess;
     const int nvec = (int)(p.vocab / 4);
-    const int slice_vec = (nvec + kCS - 1) / kCS;
-    const bool sm = p.mode == TURNOPD_SAMPLED_TOKEN;  // every listed row then carries y in [0, V)
-    auto kern = fp32_grad ? (sm ? k_row_split<true, true> : k_row_split<true, false>)
-                          : (sm ? k_row_split<false, true> : k_row_split<false, false>);
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess)
-        return e;
-    if (dev >= 64)
-        return cudaErrorInvalidDevice;
-    static int grid_cache[64][4];
-    const int gi = (fp32_grad ? 1 : 0) + (sm ? 2 : 0);  // per instantiation: attributes are per kernel
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = kCS;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    cfg.blockDim = dim3(kThreads);
-    cfg.dynamicSmemBytes = kSmemBytes;
-    cfg.stream = stream;
-    if (grid_cache[dev][gi] == 0) {
-        if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes)) !=
-            cudaSuccess)
-            return e;
-        if (kCS > 8 && (e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1)) != cudaSuccess)
-            return e;
-        cfg.gridDim = dim3(kCS);
-        int ncl = 0;
-        if ((e = cudaOccupancyMaxActiveClusters(&ncl, kern, &cfg)) != cudaSuccess)
-            return e;
-        if (ncl < 1)
-            return cudaErrorInvalidConfiguration;
-        grid_cache[dev][gi] = ncl;
-    }
-    cfg.gridDim = dim3(grid_cache[dev][gi] * kCS);
     *used = true;
-    return cudaLaunchKernelEx(&cfg, kern, p, slice_vec, nvec);
+    // every listed row of a sampled-token call carries y in [0, V)
+    if (p.mode == TURNOPD_SAMPLED_TOKEN)
+        return launch_split_t<kCSSampled, true>(p, fp32_grad, nvec, kRateSampled, stream);
+    return launch_split_t<kCSFull, false>(p, fp32_grad, nvec, kRateFull, stream);
 }
 
 }  // namespace turnopd
