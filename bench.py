@@ -40,7 +40,8 @@ V_QWEN = 151_936  # the workloads' vocabulary (a --vocab run has no committed tr
 # sampled modes add the helper grid that runs beside the cluster grid (k_row_helper for
 # bf16 logits, k_split_helper for fp32)
 KERNELS_PER_STEP = 9
-ROW_KERNEL_SOURCES = ["paper_2607_05804_gb300/csrc/rowkl_cluster.cu",
+ROW_KERNEL_SOURCES = ["paper_2607_05804_gb300/csrc/rowkl_cluster.cuh",
+                      "paper_2607_05804_gb300/csrc/rowkl_cluster.cu",
                       "paper_2607_05804_gb300/csrc/loss_kernels.cu",
                       "paper_2607_05804_gb300/csrc/common.cuh",
                       "paper_2607_05804_gb300/csrc/row_math.cuh",

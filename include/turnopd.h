@@ -152,7 +152,9 @@ size_t turnopd_weights_workspace_bytes(int32_t num_traj, int32_t max_turns);
  *      full-vocabulary gradient; l_i itself is treated as a constant).
  * Inputs:
  *   z_student, z_teacher  [num_rows, ld] row-major, in_dtype (F32 or BF16);
- *                          columns [vocab, ld) are never read.
+ *                          the values of columns [vocab, ld) never enter a result
+ *                          (bf16 rows with ld a multiple of 8 read up to the next
+ *                          multiple of 8 of vocab, inside the buffer, and mask it).
  *   row_of_token           int32[num_tokens] or NULL (then num_rows >= num_tokens);
  *                          read only where loss_mask = 1, must lie in [0, num_rows).
  *   sampled_ids            int32[num_tokens], required for SAMPLED_TOKEN, in [0, vocab).
@@ -171,12 +173,15 @@ size_t turnopd_weights_workspace_bytes(int32_t num_traj, int32_t max_turns);
  *   l_i = 0), TURNOPD_ERR_NONFINITE (non-finite LSE or l_i).
  * Precision: fp32 arithmetic on exact fp32/bf16 inputs, fp64 loss sum.
  * Kernels (the results agree within the tolerances above whichever runs):
- *   bf16 logits, vocab and ld multiples of 8, 16-byte aligned arrays: row
- *     clusters of 8 CTAs beside a helper grid on the remaining SMs;
+ *   bf16 logits, ld a multiple of 8, 16-byte aligned arrays: row clusters of
+ *     2 to 16 CTAs (the smallest whose slices fit three shared-memory stages)
+ *     beside a helper grid on the remaining SMs, or the helper grid alone for
+ *     short rows; a vocab that is not a multiple of 8 ends in a masked vector;
  *   fp32 logits, vocab and ld multiples of 4, 16-byte aligned arrays: the
- *     split-row kernel (clusters of 4 CTAs per row), which marks its first
- *     read of each logit chunk L2 evict-last and returns the lines to normal
- *     priority after the gradient's second read;
+ *     split-row kernel (clusters of 8 CTAs per row, 4 for sampled-token rows)
+ *     beside a helper grid on the remaining SMs; it marks its first read of
+ *     each logit chunk L2 evict-last and returns the lines to normal priority
+ *     after the gradient's second read;
  *   any other shape: one CTA per row.
  */
 turnopd_status turnopd_loss_fwd_bwd(const void *z_student, const void *z_teacher,

@@ -161,6 +161,8 @@ cudaError_t launch_fused(const FusedCall &c, cudaStream_t stream);
 // Cluster-resident kernel for aligned bf16 rows; sets *used = false (and
 // launches nothing) when the shape does not fit it.
 cudaError_t launch_row_cluster(const RowIn &p, bool fp32_grad, cudaStream_t stream, bool *used);
+// The same for a vocabulary that is not a multiple of 8 (a masked last vector).
+cudaError_t launch_row_cluster_tail(const RowIn &p, bool fp32_grad, cudaStream_t stream, bool *used);
 // Split-row kernel (clusters of CTAs share each row) for aligned fp32 rows; sets
 // *used = false (and launches nothing) when the shape does not fit it.
 cudaError_t launch_row_split(const RowIn &p, bool fp32_grad, cudaStream_t stream, bool *used);

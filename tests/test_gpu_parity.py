@@ -248,6 +248,32 @@ def test_odd_vocabulary_full_size(P, oracle, ld, idt):
             assert (grad[:, V:].float() == 7.0).all()
 
 
+@pytest.mark.parametrize("V", [8193, 32007, 50005, W.V_QWEN + 1, W.V_QWEN + 7])
+@pytest.mark.parametrize("mode", [0, 1], ids=["full", "sampled"])
+@pytest.mark.parametrize("gdt", ["bf16", "f32"])
+def test_masked_tail_vocab(P, oracle, V, mode, gdt):
+    """bf16 rows with V % 8 != 0 and the stride padded to a multiple of 8 take the row
+    grids with a masked last vector: V = 8,193 the helper alone, 32,007 clusters of 2,
+    50,005 clusters of 3 beside the helper, 151,937 and 151,943 clusters of 8 beside it.
+    NaN and inf fill the padding; its gradient columns stay untouched.  In sampled mode
+    every third row's y is pushed into the masked vector (its student logit 30 above the
+    row, so the Gumbel-max draw picks it)."""
+    b = W.packed(seed=51, num_traj=2, traj_len=256)
+    ld = (V + 7) // 8 * 8
+    zs, zt = W.make_logits(b.num_valid, V, "agent", torch.bfloat16, seed=52, device="cuda", ld=ld)
+    if mode == 1:
+        r = torch.arange(0, b.num_valid, 3, device="cuda")
+        zs[r, V - 1] = (zs[r, :V].float().amax(dim=1) + 30.0).to(torch.bfloat16)
+    zs[:, V:] = float("nan")
+    zt[:, V:] = float("inf")
+    _, grad = run_chain(P, oracle, b, V, zs, zt, mode=mode, alpha=0.5, compact=True, seed_y=53,
+                        grad_dtype=torch.bfloat16 if gdt == "bf16" else torch.float32)
+    assert (grad[:, V:].float() == 7.0).all()
+    if mode == 1:
+        y = W.sample_ids(zs, 53, V)
+        assert (y[r] == V - 1).all()
+
+
 @pytest.mark.parametrize("n_sup", [1, 5])
 def test_split_kernel_fewer_rows_than_clusters(P, oracle, n_sup):
     """fp32 rows at the full vocabulary with fewer rows than clusters: most clusters
@@ -486,6 +512,8 @@ def test_zero_masked_grad_and_untouched_rows(P, oracle, ld, gdt):
 
 
 def test_padding_never_read(P, oracle):
+    """NaN and inf in the padding columns change no bit of any result (V = 500: the bf16
+    row path reads the last vector's padding up to column 504 and masks it)."""
     b = W.packed(seed=6, num_traj=2, traj_len=256)
     V = 500
     zs, zt = W.make_logits(b.num_tokens, V, "agent", torch.bfloat16, seed=6, device="cuda", ld=512)
