@@ -58,41 +58,63 @@ struct CompactIn {
     int32_t *status;
 };
 
-// Token i enters the row list iff it is supervised and its row (and sampled
-// id) are in range; otherwise its loss is 0 (and a range error is recorded).
-__device__ __forceinline__ bool token_valid(const CompactIn &c, int64_t i, bool record)
-{
-    if (!c.mask[i])
-        return false;
-    const int64_t r = c.row_of_token ? (int64_t)c.row_of_token[i] : i;
-    bool ok = r >= 0 && r < c.num_rows;
-    if (ok && c.mode == TURNOPD_SAMPLED_TOKEN) {
-        const int32_t y = c.sampled_ids[i];
-        ok = y >= 0 && y < c.vocab;
-    }
-    if (!ok && record)
-        set_status(c.status, TURNOPD_ERR_TOKEN_RANGE);
-    return ok;
-}
-
 constexpr int kCompactThreads = 256;
 constexpr int kPerThread = kCompactBlock / kCompactThreads;  // 16 contiguous tokens
 
+// The kPerThread tokens i0, i0 + 1, ... of one thread.  Token i enters the row list
+// iff it is supervised and its row (and sampled id) are in range; a supervised token
+// out of range is "bad" (its loss is 0 and a range error is recorded).  Every array
+// read is issued for all the thread's tokens before any is used, so the checks cost
+// one memory round trip per array rather than one per token.
+struct TokenSlice {
+    uint32_t valid, bad;  // bit k: token i0 + k
+    int32_t r[kPerThread], y[kPerThread];
+};
+
+__device__ __forceinline__ void load_tokens(const CompactIn &c, int64_t i0, TokenSlice &t)
+{
+    uint32_t sup = 0;
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k)
+        if (i0 + k < c.T && c.mask[i0 + k])
+            sup |= 1u << k;
+    const bool sampled = c.mode == TURNOPD_SAMPLED_TOKEN;
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k) {
+        const bool m = (sup >> k) & 1u;
+        t.r[k] = m && c.row_of_token ? c.row_of_token[i0 + k] : (int32_t)(i0 + k);
+        t.y[k] = m && sampled ? c.sampled_ids[i0 + k] : -1;
+    }
+    t.valid = t.bad = 0;
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k) {
+        if (!((sup >> k) & 1u))
+            continue;
+        bool ok = t.r[k] >= 0 && (int64_t)t.r[k] < c.num_rows;
+        if (ok && sampled)
+            ok = t.y[k] >= 0 && (int64_t)t.y[k] < c.vocab;
+        if (ok)
+            t.valid |= 1u << k;
+        else
+            t.bad |= 1u << k;
+    }
+}
+
 __global__ void k_compact_count(CompactIn c, int32_t *__restrict__ blk_count)
 {
+    // the scatter kernel may start now: its token loads do not need these counts
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     __shared__ int warp_tot[kCompactThreads / 32];
     const int64_t i0 = (int64_t)blockIdx.x * kCompactBlock + (int64_t)threadIdx.x * kPerThread;
-    int n = 0;
-    for (int k = 0; k < kPerThread; ++k) {
-        const int64_t i = i0 + k;
-        if (i >= c.T)
-            break;
-        if (token_valid(c, i, true))
-            ++n;
-        else
-            c.token_loss[i] = 0.f;
-    }
-    n = warp_sum_i32(n);
+    TokenSlice t;
+    load_tokens(c, i0, t);
+    if (t.bad)
+        set_status(c.status, TURNOPD_ERR_TOKEN_RANGE);
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k)
+        if (i0 + k < c.T && !((t.valid >> k) & 1u))
+            c.token_loss[i0 + k] = 0.f;
+    int n = warp_sum_i32(__popc(t.valid));
     if ((threadIdx.x & 31) == 0)
         warp_tot[threadIdx.x >> 5] = n;
     __syncthreads();
@@ -104,6 +126,8 @@ __global__ void k_compact_count(CompactIn c, int32_t *__restrict__ blk_count)
     }
 }
 
+// Launched as a programmatic dependent of k_compact_count: the thread's tokens are
+// loaded before the wait for the block counts.
 __global__ void k_compact_scatter(CompactIn c, const int32_t *__restrict__ blk_count,
                                   int4 *__restrict__ rows, int32_t *__restrict__ nvalid)
 {
@@ -111,6 +135,14 @@ __global__ void k_compact_scatter(CompactIn c, const int32_t *__restrict__ blk_c
     __shared__ int warp_off[kCompactThreads / 32];
     __shared__ int64_t base_s;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int64_t i0 = (int64_t)blockIdx.x * kCompactBlock + (int64_t)threadIdx.x * kPerThread;
+    TokenSlice t;
+    load_tokens(c, i0, t);
+    float wv[kPerThread];
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k)
+        wv[k] = ((t.valid >> k) & 1u) ? c.w[i0 + k] : 0.f;
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // every block's count is written
     // exclusive prefix over the preceding blocks
     int64_t pre = 0;
     for (int k = threadIdx.x; k < (int)blockIdx.x; k += kCompactThreads)
@@ -128,13 +160,7 @@ __global__ void k_compact_scatter(CompactIn c, const int32_t *__restrict__ blk_c
     __syncthreads();
     const int64_t base = base_s;
 
-    const int64_t i0 = (int64_t)blockIdx.x * kCompactBlock + (int64_t)threadIdx.x * kPerThread;
-    uint32_t bits = 0;
-    for (int k = 0; k < kPerThread; ++k) {
-        const int64_t i = i0 + k;
-        if (i < c.T && token_valid(c, i, false))
-            bits |= 1u << k;
-    }
+    const uint32_t bits = t.valid;
     const int n = __popc(bits);
     // exclusive scan of n across the block (thread order = token order)
     int incl = n;
@@ -159,14 +185,10 @@ __global__ void k_compact_scatter(CompactIn c, const int32_t *__restrict__ blk_c
     }
     __syncthreads();
     int64_t pos = base + warp_off[warp] + (incl - n);
-    for (int k = 0; k < kPerThread; ++k) {
-        if (bits & (1u << k)) {
-            const int64_t i = i0 + k;
-            const int32_t r = c.row_of_token ? c.row_of_token[i] : (int32_t)i;
-            const int32_t y = c.mode == TURNOPD_SAMPLED_TOKEN ? c.sampled_ids[i] : -1;
-            rows[pos++] = make_int4((int32_t)i, r, y, __float_as_int(c.w[i]));
-        }
-    }
+#pragma unroll
+    for (int k = 0; k < kPerThread; ++k)
+        if ((bits >> k) & 1u)
+            rows[pos++] = make_int4((int32_t)(i0 + k), t.r[k], t.y[k], __float_as_int(wv[k]));
 }
 
 // ---------------------------------------------------------------- row kernel
@@ -322,10 +344,23 @@ __global__ void k_loss_sum(const double *__restrict__ row_wl, const int32_t *__r
                            double *__restrict__ loss, int32_t *status)
 {
     __shared__ double part[32];
+    // launched as a programmatic dependent of the row grid: every row's w l is written
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     const int n = *nvalid;
-    double s = 0.0;
-    for (int j = threadIdx.x; j < n; j += blockDim.x)
-        s += row_wl[j];
+    const int nt = (int)blockDim.x;
+    // eight loads in flight per thread, summed in a fixed order
+    double s8[8] = {0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0};
+    int j = threadIdx.x;
+    for (; j + 7 * nt < n; j += 8 * nt) {
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+            s8[u] += row_wl[j + u * nt];
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+        if (j + u * nt < n)
+            s8[u] += row_wl[j + u * nt];
+    double s = ((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7]));
     s = warp_sum_f64(s);
     if ((threadIdx.x & 31) == 0)
         part[threadIdx.x >> 5] = s;
@@ -362,14 +397,35 @@ cudaError_t launch_compaction(const LossArgs &a, int4 *rows, int32_t *blk_count,
     CompactIn c{a.mask, a.row_of_token, a.sampled_ids, a.w, a.num_rows, a.vocab, a.T, a.mode,
                 a.token_loss, a.status};
     k_compact_count<<<nblk, kCompactThreads, 0, stream>>>(c, blk_count);
-    k_compact_scatter<<<nblk, kCompactThreads, 0, stream>>>(c, blk_count, rows, nvalid);
-    return cudaGetLastError();
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.gridDim = dim3(nblk);
+    cfg.blockDim = dim3(kCompactThreads);
+    cfg.stream = stream;
+    const int32_t *cnt = blk_count;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, k_compact_scatter, c, cnt, rows, nvalid);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
+// A programmatic dependent of the kernel before it: row grids that signal early let it
+// take the first SM they free, and it waits for their completion before reading.
 void launch_loss_sum(const double *row_wl, const int32_t *nvalid, double *loss, int32_t *status,
                      cudaStream_t stream)
 {
-    k_loss_sum<<<1, 1024, 0, stream>>>(row_wl, nvalid, loss, status);
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cfg.gridDim = dim3(1);
+    cfg.blockDim = dim3(1024);
+    cfg.stream = stream;
+    cudaLaunchKernelEx(&cfg, k_loss_sum, row_wl, nvalid, loss, status);
 }
 
 void launch_zero_masked_f32(const uint8_t *mask, int64_t T, int64_t d, float *out, cudaStream_t stream)

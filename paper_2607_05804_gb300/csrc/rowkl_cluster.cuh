@@ -548,6 +548,8 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
     constexpr uint32_t kFill = 0xff7fff7fu;  // lowest finite bf16 pair: adds 0, never the max
     __shared__ float red[NW][8];
     __shared__ float bc[8];
+    // the loss sum after this grid may take the first SM it frees (it waits for the grid)
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int nvalid = *p.nvalid;
     const int j0 = p.split_den ? (int)((int64_t)nvalid * p.split_num / p.split_den) : 0;

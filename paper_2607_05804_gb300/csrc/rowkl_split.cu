@@ -562,6 +562,8 @@ __global__ void __launch_bounds__(NTH, 1) k_split_helper(RowIn p)
     constexpr int NW = NTH / 32;
     __shared__ float red[NW][8];
     __shared__ float bc[8];
+    // the loss sum after this grid may take the first SM it frees (it waits for the grid)
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int nvalid = *p.nvalid;
     const int j0 = p.split_den ? (int)((int64_t)nvalid * p.split_num / p.split_den) : 0;

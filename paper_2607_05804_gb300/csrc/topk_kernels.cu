@@ -45,11 +45,15 @@
 namespace turnopd {
 namespace {
 
+// streaming warps per CTA and CTAs per SM (measured, K = 50, full-size batches, fraction
+// of the copy bandwidth packed / household / multihop: 8 x 3: 0.923 / 0.889 / 0.865;
+// 12 x 2: 0.942 / 0.910 / 0.874; 10 x 2: 0.926 / 0.895 / 0.864; 14 x 2: 0.921 / 0.884 /
+// 0.855; 8 x 2: 0.881 / 0.851 / 0.821; 24 x 1: 0.771 / 0.740 / 0.713)
 #ifndef TURNOPD_TOPK_STREAM_WARPS
-#define TURNOPD_TOPK_STREAM_WARPS 8
+#define TURNOPD_TOPK_STREAM_WARPS 12
 #endif
 #ifndef TURNOPD_TOPK_MINB
-#define TURNOPD_TOPK_MINB 3
+#define TURNOPD_TOPK_MINB 2
 #endif
 constexpr int kTkStreamWarps = TURNOPD_TOPK_STREAM_WARPS;  // pass A, row after row
 constexpr int kTkSelThreads = 64;                           // two selector warps
@@ -345,6 +349,8 @@ size_t topk_smem_bytes(int64_t V, int K) { return topk_fixed_bytes(K) + 2 * topk
 template <bool BF16>
 __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs a)
 {
+    // the loss sum after this grid may take the first SM it frees (it waits for the grid)
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     extern __shared__ __align__(128) uint64_t tk_smem[];
     const int K = a.K;
     uint64_t *s_cand = tk_smem;
