@@ -102,8 +102,9 @@ __device__ __forceinline__ void load_tokens(const CompactIn &c, int64_t i0, Toke
 
 __global__ void k_compact_count(CompactIn c, int32_t *__restrict__ blk_count)
 {
-    // the scatter kernel may start now: its token loads do not need these counts
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    // a programmatic dependent of the caller's work; the scatter kernel may start
+    // once this has begun: its token loads do not need these counts
+    pdl_begin();
     __shared__ int warp_tot[kCompactThreads / 32];
     const int64_t i0 = (int64_t)blockIdx.x * kCompactBlock + (int64_t)threadIdx.x * kPerThread;
     TokenSlice t;
@@ -345,7 +346,8 @@ __global__ void k_loss_sum(const double *__restrict__ row_wl, const int32_t *__r
 {
     __shared__ double part[32];
     // launched as a programmatic dependent of the row grid: every row's w l is written
-    asm volatile("griddepcontrol.wait;" ::: "memory");
+    // (and the turn statistics after this may launch)
+    pdl_begin();
     const int n = *nvalid;
     const int nt = (int)blockDim.x;
     // eight loads in flight per thread, summed in a fixed order
@@ -396,7 +398,9 @@ cudaError_t launch_compaction(const LossArgs &a, int4 *rows, int32_t *blk_count,
     const int nblk = (int)((a.T + kCompactBlock - 1) / kCompactBlock);
     CompactIn c{a.mask, a.row_of_token, a.sampled_ids, a.w, a.num_rows, a.vocab, a.T, a.mode,
                 a.token_loss, a.status};
-    k_compact_count<<<nblk, kCompactThreads, 0, stream>>>(c, blk_count);
+    cudaError_t e0 = launch_dependent(k_compact_count, dim3(nblk), dim3(kCompactThreads), 0, stream, c, blk_count);
+    if (e0 != cudaSuccess)
+        return e0;
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

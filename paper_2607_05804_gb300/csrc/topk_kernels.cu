@@ -56,7 +56,12 @@ namespace {
 #define TURNOPD_TOPK_MINB 2
 #endif
 constexpr int kTkStreamWarps = TURNOPD_TOPK_STREAM_WARPS;  // pass A, row after row
-constexpr int kTkSelThreads = 64;                           // two selector warps
+#ifndef TURNOPD_TOPK_SEL_WARPS
+#define TURNOPD_TOPK_SEL_WARPS 2
+#endif
+constexpr int kTkSelWarps = TURNOPD_TOPK_SEL_WARPS;         // the later phases, a row behind
+constexpr int kTkSelThreads = kTkSelWarps * 32;
+static_assert(kTkSelWarps >= 1 && kTkSelWarps <= 4, "sort_desc needs n >= 2 kTkSelThreads, n >= 256");
 constexpr int kTkStreamThreads = kTkStreamWarps * 32;
 constexpr int kTkThreads = kTkStreamThreads + kTkSelThreads;
 constexpr int kTkMinBlocks = TURNOPD_TOPK_MINB;  // CTAs (rows in flight) per SM
@@ -368,7 +373,7 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
     __shared__ uint32_t s_tau[2];                     // per buffer: the bound (ordered logit)
     __shared__ int s_ng[2];                           // per buffer: candidate groups found
     __shared__ uint16_t s_glist[2][kTkGroupCap];      // per buffer: their indices
-    __shared__ uint16_t s_wq[2][kTkQueue];            // per selector warp: groups found, not yet read
+    __shared__ uint16_t s_wq[kTkSelWarps][kTkQueue];  // per selector warp: groups found, not yet read
     __shared__ int s_scnt[2][kTkStreamWarps];         // per streaming warp: a count of buckets
     __shared__ uint32_t s_smax[kTkStreamWarps];       // per streaming warp: its largest bucket
 
@@ -783,7 +788,8 @@ __global__ void __launch_bounds__(kTkThreads, kTkMinBlocks) k_topk_rows(TopkArgs
                 }
             } else {
                 // ---- the K largest: each candidate's rank among the candidates is its position
-                // (keys are unique); a buffer above 64 is first cut to the K largest by radix select
+                // (keys are unique); a buffer larger than the selector threads is first cut to the
+                // K largest by radix select
                 const uint64_t kth = nc <= kTkSelThreads ? 0 : sel_kth_largest(s_cand, nc, K, hi_val, 0, s_sel, stid);
                 for (int i = stid; i < nc; i += kTkSelThreads) {
                     const uint64_t k = s_cand[i];

@@ -40,6 +40,7 @@ __global__ void k_traj_counts(const int32_t *__restrict__ turn_id,
                               const int64_t *__restrict__ off, int32_t B, int64_t T,
                               int32_t Tmax, int32_t *__restrict__ n_bt, int32_t *status)
 {
+    pdl_begin();
     extern __shared__ int32_t hist[];
     const int b = blockIdx.x;
     for (int t = threadIdx.x; t < Tmax; t += blockDim.x)
@@ -48,15 +49,28 @@ __global__ void k_traj_counts(const int32_t *__restrict__ turn_id,
     int64_t lo, hi;
     traj_range(off, B, T, b, lo, hi, status);
     bool bad = false;
-    for (int64_t i = lo + threadIdx.x; i < hi; i += blockDim.x) {
-        if (!mask[i])
-            continue;
-        int32_t t = turn_id[i];
-        if (t < 0 || t >= Tmax) {
-            bad = true;
-            continue;
+    // four tokens per thread in flight; mask and turn id loaded together (a token's turn
+    // id is read whether or not it is supervised: the index lies inside the trajectory)
+    const int64_t step = blockDim.x;
+    for (int64_t i0 = lo + threadIdx.x; i0 < hi; i0 += 4 * step) {
+        uint8_t m[4];
+        int32_t t[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int64_t i = i0 + u * step;
+            m[u] = i < hi ? mask[i] : 0;
+            t[u] = i < hi ? turn_id[i] : 0;
         }
-        atomicAdd(&hist[t], 1);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            if (!m[u])
+                continue;
+            if (t[u] < 0 || t[u] >= Tmax) {
+                bad = true;
+                continue;
+            }
+            atomicAdd(&hist[t[u]], 1);
+        }
     }
     if (bad)
         set_status(status, TURNOPD_ERR_TURN_RANGE);
@@ -69,13 +83,21 @@ __global__ void k_traj_counts(const int32_t *__restrict__ turn_id,
 __global__ void k_counts_reduce(const int32_t *__restrict__ n_bt, int32_t B, int32_t Tmax,
                                 int64_t *__restrict__ counts)
 {
+    pdl_begin();
     __shared__ int64_t warp_bp[32];
+    // eight table entries loaded at a time (integer sums: any order gives the same result)
     for (int t = threadIdx.x; t < Tmax; t += blockDim.x) {
         int64_t s = 0, c = 0;
-        for (int b = 0; b < B; ++b) {
-            int32_t n = n_bt[(int64_t)b * Tmax + t];
-            s += n > 0;
-            c += n;
+        for (int b0 = 0; b0 < B; b0 += 8) {
+            int32_t n[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                n[u] = b0 + u < B ? n_bt[(int64_t)(b0 + u) * Tmax + t] : 0;
+#pragma unroll
+            for (int u = 0; u < 8; ++u) {
+                s += n[u] > 0;
+                c += n[u];
+            }
         }
         counts[t] = s;
         counts[Tmax + t] = c;
@@ -84,8 +106,15 @@ __global__ void k_counts_reduce(const int32_t *__restrict__ n_bt, int32_t B, int
     int64_t bp = 0;
     for (int b = threadIdx.x; b < B; b += blockDim.x) {
         int64_t nb = 0;
-        for (int t = 0; t < Tmax; ++t)
-            nb += n_bt[(int64_t)b * Tmax + t];
+        for (int t0 = 0; t0 < Tmax; t0 += 8) {
+            int32_t n[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                n[u] = t0 + u < Tmax ? n_bt[(int64_t)b * Tmax + t0 + u] : 0;
+#pragma unroll
+            for (int u = 0; u < 8; ++u)
+                nb += n[u];
+        }
         bp += nb > 0;
     }
     bp = warp_sum_i64(bp);
@@ -115,6 +144,7 @@ __global__ void k_weights(const int32_t *__restrict__ turn_id, const uint8_t *__
                           const int32_t *__restrict__ n_bt, const int64_t *__restrict__ counts,
                           float *__restrict__ w_out, int32_t *status)
 {
+    pdl_begin();
     __shared__ int64_t red[4][32];
     __shared__ double coef[3];  // token weight 1/N_b (or 1/N), reliable-turn numerator, R
     __shared__ float s_wt[TURNOPD_MAX_TURNS];  // this trajectory's token weight per turn
@@ -176,9 +206,23 @@ __global__ void k_weights(const int32_t *__restrict__ turn_id, const uint8_t *__
 
     int64_t lo, hi;
     traj_range(off, B, T, b, lo, hi, status);
-    for (int64_t i = lo + threadIdx.x; i < hi; i += blockDim.x) {
-        const int32_t t = mask[i] ? turn_id[i] : -1;
-        w_out[i] = t >= 0 && t < Tmax ? s_wt[t] : 0.f;
+    // four tokens per thread in flight, mask and turn id loaded together
+    const int64_t step = blockDim.x;
+    for (int64_t i0 = lo + threadIdx.x; i0 < hi; i0 += 4 * step) {
+        uint8_t m[4];
+        int32_t t[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int64_t i = i0 + u * step;
+            m[u] = i < hi ? mask[i] : 0;
+            t[u] = i < hi ? turn_id[i] : -1;
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int64_t i = i0 + u * step;
+            if (i < hi)
+                w_out[i] = m[u] && t[u] >= 0 && t[u] < Tmax ? s_wt[t[u]] : 0.f;
+        }
     }
     // tokens outside every trajectory range (only with bad offsets) stay untouched
 }
@@ -196,6 +240,7 @@ __global__ void k_turn_stats_traj(const float *__restrict__ token_loss,
                                   int32_t Tmax, double *__restrict__ traj_turn_sum,
                                   int32_t *__restrict__ traj_turn_cnt, int32_t *status)
 {
+    pdl_begin();
     extern __shared__ unsigned char smem_raw[];
     const int nw = blockDim.x >> 5;
     double *bsum = reinterpret_cast<double *>(smem_raw);                    // [nw][Tmax]
@@ -214,31 +259,45 @@ __global__ void k_turn_stats_traj(const float *__restrict__ token_loss,
     const int64_t c0 = lo + (int64_t)warp * chunk;
     const int64_t c1 = min(hi, c0 + chunk);
     bool bad = false;
-    for (int64_t base = c0; base < c1; base += 32) {
-        const int64_t i = base + lane;
-        int32_t key = -1;
-        float val = 0.f;
-        if (i < c1 && mask[i]) {
-            int32_t t = turn_id[i];
-            if (t >= 0 && t < Tmax) {
-                key = t;
-                val = token_loss[i];
-            } else {
-                bad = true;
-            }
+    // four 32-token steps per iteration: every load of the four is issued first (mask,
+    // turn id and loss together), then the steps are folded in order as before
+    for (int64_t base = c0; base < c1; base += 4 * 32) {
+        uint8_t mk[4];
+        int32_t tt[4];
+        float lv[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int64_t i = base + u * 32 + lane;
+            const bool in = i < c1;
+            mk[u] = in ? mask[i] : 0;
+            tt[u] = in ? turn_id[i] : -1;
+            lv[u] = in ? token_loss[i] : 0.f;
         }
-        unsigned todo = __ballot_sync(0xffffffffu, key >= 0);
-        while (todo) {
-            const int leader = __ffs(todo) - 1;
-            const int k0 = __shfl_sync(0xffffffffu, key, leader);
-            const bool mine = key == k0 && key >= 0;
-            const unsigned members = __ballot_sync(0xffffffffu, mine);
-            const double s = warp_sum_f64(mine ? (double)val : 0.0);
-            if (lane == 0) {
-                bsum[(size_t)warp * Tmax + k0] += s;
-                bcnt[(size_t)warp * Tmax + k0] += __popc(members);
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            int32_t key = -1;
+            float val = 0.f;
+            if (mk[u]) {
+                if (tt[u] >= 0 && tt[u] < Tmax) {
+                    key = tt[u];
+                    val = lv[u];
+                } else {
+                    bad = true;
+                }
             }
-            todo &= ~members;
+            unsigned todo = __ballot_sync(0xffffffffu, key >= 0);
+            while (todo) {
+                const int leader = __ffs(todo) - 1;
+                const int k0 = __shfl_sync(0xffffffffu, key, leader);
+                const bool mine = key == k0 && key >= 0;
+                const unsigned members = __ballot_sync(0xffffffffu, mine);
+                const double s = warp_sum_f64(mine ? (double)val : 0.0);
+                if (lane == 0) {
+                    bsum[(size_t)warp * Tmax + k0] += s;
+                    bcnt[(size_t)warp * Tmax + k0] += __popc(members);
+                }
+                todo &= ~members;
+            }
         }
     }
     if (bad)
@@ -262,17 +321,30 @@ __global__ void k_turn_stats_index(const double *__restrict__ traj_turn_sum,
                                    int32_t Tmax, double *__restrict__ turn_sum,
                                    int64_t *__restrict__ turn_cnt, int32_t *__restrict__ turn_surv)
 {
+    pdl_begin();
     const int t = blockIdx.x * blockDim.x + threadIdx.x;
     if (t >= Tmax)
         return;
     double s = 0.0;
     int64_t c = 0;
     int32_t v = 0;
-    for (int b = 0; b < B; ++b) {
-        s += traj_turn_sum[(int64_t)b * Tmax + t];
-        int32_t n = traj_turn_cnt[(int64_t)b * Tmax + t];
-        c += n;
-        v += n > 0;
+    // eight trajectories' entries loaded at a time, added in trajectory order
+    for (int b0 = 0; b0 < B; b0 += 8) {
+        double sv[8];
+        int32_t nv[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+            const int b = b0 + u;
+            sv[u] = b < B ? traj_turn_sum[(int64_t)b * Tmax + t] : 0.0;
+            nv[u] = b < B ? traj_turn_cnt[(int64_t)b * Tmax + t] : 0;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u)
+            if (b0 + u < B) {
+                s += sv[u];
+                c += nv[u];
+                v += nv[u] > 0;
+            }
     }
     turn_sum[t] = s;
     turn_cnt[t] = c;
@@ -288,11 +360,13 @@ cudaError_t launch_turn_counts(const int32_t *turn_id, const uint8_t *mask, cons
                                int32_t B, int64_t T, int32_t Tmax, int32_t *n_bt,
                                int64_t *counts, int32_t *status, cudaStream_t stream)
 {
-    if (B > 0) {
-        k_traj_counts<<<B, kTrajThreads, sizeof(int32_t) * Tmax, stream>>>(turn_id, mask, off, B, T, Tmax,
-                                                                            n_bt, status);
-    }
-    k_counts_reduce<<<1, 256, 0, stream>>>(n_bt, B, Tmax, counts);
+    cudaError_t e = cudaSuccess;
+    if (B > 0 &&
+        (e = launch_dependent(k_traj_counts, dim3(B), dim3(kTrajThreads), sizeof(int32_t) * Tmax, stream,
+                              turn_id, mask, off, B, T, Tmax, n_bt, status)) != cudaSuccess)
+        return e;
+    if ((e = launch_dependent(k_counts_reduce, dim3(1), dim3(256), 0, stream, n_bt, B, Tmax, counts)) != cudaSuccess)
+        return e;
     return cudaGetLastError();
 }
 
@@ -301,9 +375,12 @@ cudaError_t launch_weights(const int32_t *turn_id, const uint8_t *mask, const in
                            int32_t n_min, const int32_t *n_bt, const int64_t *counts,
                            float *w_out, int32_t *status, cudaStream_t stream)
 {
-    if (B > 0)
-        k_weights<<<B, kTrajThreads, 0, stream>>>(turn_id, mask, off, B, T, Tmax, alpha, scope, n_min, n_bt,
-                                                  counts, w_out, status);
+    if (B > 0) {
+        const cudaError_t e = launch_dependent(k_weights, dim3(B), dim3(kTrajThreads), 0, stream, turn_id, mask,
+                                               off, B, T, Tmax, alpha, scope, n_min, n_bt, counts, w_out, status);
+        if (e != cudaSuccess)
+            return e;
+    }
     return cudaGetLastError();
 }
 
@@ -331,12 +408,15 @@ cudaError_t launch_turn_stats(const float *token_loss, const int32_t *turn_id,
             if (e != cudaSuccess)
                 return e;
         }
-        k_turn_stats_traj<<<B, nw * 32, smem, stream>>>(token_loss, turn_id, mask, off, B, T, Tmax,
-                                                       traj_turn_sum, traj_turn_cnt, status);
+        const cudaError_t e = launch_dependent(k_turn_stats_traj, dim3(B), dim3(nw * 32), smem, stream,
+                                               token_loss, turn_id, mask, off, B, T, Tmax, traj_turn_sum,
+                                               traj_turn_cnt, status);
+        if (e != cudaSuccess)
+            return e;
     }
-    k_turn_stats_index<<<(Tmax + 127) / 128, 128, 0, stream>>>(traj_turn_sum, traj_turn_cnt, B,
-                                                               Tmax, turn_sum, turn_cnt, turn_surv);
-    return cudaGetLastError();
+    const cudaError_t e = launch_dependent(k_turn_stats_index, dim3((Tmax + 127) / 128), dim3(128), 0, stream,
+                                           traj_turn_sum, traj_turn_cnt, B, Tmax, turn_sum, turn_cnt, turn_surv);
+    return e != cudaSuccess ? e : cudaGetLastError();
 }
 
 }  // namespace turnopd
