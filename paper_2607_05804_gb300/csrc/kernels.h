@@ -35,6 +35,17 @@ struct LossWorkspace {
 
 constexpr int kCompactBlock = 4096;  // tokens per compaction block
 
+// The row-count slot of every loss workspace layout is 256 bytes; beside the count it
+// holds the loss sum's scratch: a ticket (zeroed by the compaction, reset by the last
+// CTA of the sum) and one partial sum per CTA of the sum.
+constexpr int kSumCTAs = 24;
+static_assert(8 + 8 * kSumCTAs <= 256, "the loss sum's scratch fits the row-count slot");
+__host__ __device__ inline uint32_t *sum_ticket(int32_t *nvalid) { return reinterpret_cast<uint32_t *>(nvalid + 1); }
+__host__ __device__ inline double *sum_partials(int32_t *nvalid)
+{
+    return reinterpret_cast<double *>(reinterpret_cast<char *>(nvalid) + 8);
+}
+
 size_t loss_workspace_bytes(int64_t T);
 LossWorkspace loss_workspace_layout(void *ws, int64_t T);
 
@@ -88,7 +99,7 @@ cudaError_t launch_wait_selftest(uint32_t limit, int32_t *status, cudaStream_t s
 // Pieces of the loss path reused by the fused LM-head path.
 cudaError_t launch_compaction(const LossArgs &a, int4 *rows, int32_t *blk_count, int32_t *nvalid,
                               cudaStream_t stream);
-void launch_loss_sum(const double *row_wl, const int32_t *nvalid, double *loss, int32_t *status,
+void launch_loss_sum(const double *row_wl, int32_t *nvalid, double *loss, int32_t *status,
                      cudaStream_t stream);
 // Zero rows i (of d fp32 values) of out where mask[i] == 0.
 void launch_zero_masked_f32(const uint8_t *mask, int64_t T, int64_t d, float *out, cudaStream_t stream);

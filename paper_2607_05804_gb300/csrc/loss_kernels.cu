@@ -181,8 +181,10 @@ __global__ void k_compact_scatter(CompactIn c, const int32_t *__restrict__ blk_c
             warp_off[wi] = s;
             s += warp_tot[wi];
         }
-        if (blockIdx.x == gridDim.x - 1)
+        if (blockIdx.x == gridDim.x - 1) {
             *nvalid = (int32_t)(base + s);
+            *sum_ticket(nvalid) = 0u;  // for the loss sum after the row grids
+        }
     }
     __syncthreads();
     int64_t pos = base + warp_off[warp] + (incl - n);
@@ -341,39 +343,59 @@ __global__ void k_zero_masked(const uint8_t *__restrict__ mask, const int32_t *_
 // ---------------------------------------------------------------- loss sum
 
 // loss = sum_j row_wl[j] over the compacted rows (= token order), fixed tree.
-__global__ void k_loss_sum(const double *__restrict__ row_wl, const int32_t *__restrict__ nvalid,
-                           double *__restrict__ loss, int32_t *status)
+// sum_i w_i l_i over the row list in a fixed order, on kSumCTAs CTAs: CTA c sums a fixed
+// chunk of the rows (threads strided, then the warps' xor trees, then in warp order),
+// and the CTA that finishes last adds the partials by a fixed xor tree.  One CTA alone
+// was bound by its SM's fp64 rate (a small fraction of the fp32 rate on this part).
+// A programmatic dependent of the row grid.
+constexpr int kSumThreads = 256;
+
+__global__ void __launch_bounds__(kSumThreads) k_loss_sum(const double *__restrict__ row_wl,
+                                                          int32_t *__restrict__ nvalid,
+                                                          double *__restrict__ loss, int32_t *status)
 {
-    __shared__ double part[32];
-    // launched as a programmatic dependent of the row grid: every row's w l is written
-    // (and the turn statistics after this may launch)
+    __shared__ double part[kSumThreads / 32];
+    __shared__ int last;
+    // every row's w l is written (and the turn statistics after this may launch)
     pdl_begin();
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int n = *nvalid;
-    const int nt = (int)blockDim.x;
-    // eight loads in flight per thread, summed in a fixed order
-    double s8[8] = {0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0, 0.0};
-    int j = threadIdx.x;
-    for (; j + 7 * nt < n; j += 8 * nt) {
+    const int chunk = (n + kSumCTAs - 1) / kSumCTAs;
+    const int j0 = (int)blockIdx.x * chunk, j1 = min(n, j0 + chunk);
+    double s4[4] = {0.0, 0.0, 0.0, 0.0};
+    int j = j0 + (int)threadIdx.x;
+    for (; j + 3 * kSumThreads < j1; j += 4 * kSumThreads) {
 #pragma unroll
-        for (int u = 0; u < 8; ++u)
-            s8[u] += row_wl[j + u * nt];
+        for (int u = 0; u < 4; ++u)
+            s4[u] += row_wl[j + u * kSumThreads];
     }
 #pragma unroll
-    for (int u = 0; u < 8; ++u)
-        if (j + u * nt < n)
-            s8[u] += row_wl[j + u * nt];
-    double s = ((s8[0] + s8[1]) + (s8[2] + s8[3])) + ((s8[4] + s8[5]) + (s8[6] + s8[7]));
-    s = warp_sum_f64(s);
-    if ((threadIdx.x & 31) == 0)
-        part[threadIdx.x >> 5] = s;
+    for (int u = 0; u < 4; ++u)
+        if (j + u * kSumThreads < j1)
+            s4[u] += row_wl[j + u * kSumThreads];
+    double s = warp_sum_f64((s4[0] + s4[1]) + (s4[2] + s4[3]));
+    if (lane == 0)
+        part[warp] = s;
     __syncthreads();
     if (threadIdx.x == 0) {
-        double tot = 0.0;
-        for (int k = 0; k < (int)(blockDim.x >> 5); ++k)
-            tot += part[k];
-        if (!isfinite(tot))
-            set_status(status, TURNOPD_ERR_NONFINITE);
-        *loss = tot;
+        double t = 0.0;
+        for (int w = 0; w < kSumThreads / 32; ++w)
+            t += part[w];
+        sum_partials(nvalid)[blockIdx.x] = t;
+        __threadfence();
+        last = atomicAdd(sum_ticket(nvalid), 1u) == (unsigned)(kSumCTAs - 1);
+    }
+    __syncthreads();
+    if (last && warp == 0) {
+        __threadfence();
+        double v = lane < kSumCTAs ? __ldcg(sum_partials(nvalid) + lane) : 0.0;
+        v = warp_sum_f64(v);
+        if (lane == 0) {
+            if (!isfinite(v))
+                set_status(status, TURNOPD_ERR_NONFINITE);
+            *loss = v;
+            *sum_ticket(nvalid) = 0u;
+        }
     }
 }
 
@@ -417,19 +439,10 @@ cudaError_t launch_compaction(const LossArgs &a, int4 *rows, int32_t *blk_count,
 
 // A programmatic dependent of the kernel before it: row grids that signal early let it
 // take the first SM they free, and it waits for their completion before reading.
-void launch_loss_sum(const double *row_wl, const int32_t *nvalid, double *loss, int32_t *status,
+void launch_loss_sum(const double *row_wl, int32_t *nvalid, double *loss, int32_t *status,
                      cudaStream_t stream)
 {
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    cfg.gridDim = dim3(1);
-    cfg.blockDim = dim3(1024);
-    cfg.stream = stream;
-    cudaLaunchKernelEx(&cfg, k_loss_sum, row_wl, nvalid, loss, status);
+    launch_dependent(k_loss_sum, dim3(kSumCTAs), dim3(kSumThreads), 0, stream, row_wl, nvalid, loss, status);
 }
 
 void launch_zero_masked_f32(const uint8_t *mask, int64_t T, int64_t d, float *out, cudaStream_t stream)
