@@ -538,9 +538,17 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
 // of the cluster grid (it starts once every cluster is resident) and completes
 // only after it, so stream order after it covers both grids.
 constexpr int kHelpThreads = 512;
-constexpr int kHelpU = 4;  // vectors of each model in flight per thread
+constexpr int kHelpU = 4;  // vectors of each model per thread and batch
+// AS: the statistics pass's batches land in a kHelpStages-deep ring in shared memory by
+// cp.async, kHelpStages - 1 batches ahead (each thread copies and reads only its own
+// slots): twice the loads in flight of the register path, with no registers held by
+// them.  The helper beside the clusters takes it (packed 8 x 4096, V = 151,936: 2.776 ->
+// 2.743 ms per loss call with the split rate raised to 0.7); the helper alone on every
+// SM keeps the register path (V = 16,384: 0.405 against 0.433 ms).
+constexpr int kHelpStages = 3;
+constexpr size_t helper_smem_bytes(bool as, int nth) { return as ? (size_t)kHelpStages * 2 * kHelpU * nth * 16 : 0; }
 
-template <bool G32, bool SM, bool TL, int NTH = kHelpThreads, int MINB = 1>
+template <bool G32, bool SM, bool TL, bool AS, int NTH = kHelpThreads, int MINB = 1>
 __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
 {
     constexpr int kHelpThreads = NTH;
@@ -548,6 +556,7 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
     constexpr uint32_t kFill = 0xff7fff7fu;  // lowest finite bf16 pair: adds 0, never the max
     __shared__ float red[NW][8];
     __shared__ float bc[8];
+    extern __shared__ uint4 hring[];  // [kHelpStages][2][kHelpU][NTH] (AS)
     // the loss sum after this grid may take the first SM it frees (it waits for the grid)
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -569,14 +578,44 @@ __global__ void __launch_bounds__(NTH, MINB) k_row_helper(RowIn p)
         const int yvec = m.z >= 0 ? (m.z >> 3) : -1;     // the vector holding the sampled id
         float ms = -INFINITY, mt = -INFINITY, dd = 0.f;  // dd: reference difference (fp32 gradient)
         float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
-        for (int q0 = tid; q0 < nvec; q0 += kHelpU * kHelpThreads) {
+        // this thread's batches of the row: kHelpU vectors of each model, kHelpThreads apart
+        const int nbt = nvec > tid ? (nvec - tid + kHelpU * kHelpThreads - 1) / (kHelpU * kHelpThreads) : 0;
+        auto slot = [&](int s, int mdl, int u) { return ((s * 2 + mdl) * kHelpU + u) * kHelpThreads + tid; };
+        auto issue = [&](int bi) {  // batch bi into the ring (an empty group past the last)
+            if (bi < nbt) {
+                const int s = bi % kHelpStages, q0 = tid + bi * kHelpU * kHelpThreads;
+#pragma unroll
+                for (int u = 0; u < kHelpU; ++u) {
+                    const int q = q0 + u * kHelpThreads;
+                    if (q < nvec) {
+                        cp_async16(&hring[slot(s, 0, u)], vs + q);
+                        cp_async16(&hring[slot(s, 1, u)], vt + q);
+                    }
+                }
+            }
+            cp_async_commit();
+        };
+        if (AS)
+            for (int bi = 0; bi < kHelpStages - 1; ++bi)
+                issue(bi);
+        for (int bi = 0; bi < nbt; ++bi) {
+            const int q0 = tid + bi * kHelpU * kHelpThreads;
             uint4 a[kHelpU], b[kHelpU];
+            if (AS) {
+                issue(bi + kHelpStages - 1);
+                cp_async_wait<kHelpStages - 1>();  // batch bi has landed
+            }
 #pragma unroll
             for (int u = 0; u < kHelpU; ++u) {
                 const int q = q0 + u * kHelpThreads;
                 if (q < nvec) {
-                    a[u] = __ldg(vs + q);
-                    b[u] = __ldg(vt + q);
+                    if (AS) {
+                        a[u] = hring[slot(bi % kHelpStages, 0, u)];
+                        b[u] = hring[slot(bi % kHelpStages, 1, u)];
+                    } else {
+                        a[u] = __ldg(vs + q);
+                        b[u] = __ldg(vt + q);
+                    }
                 } else {
                     a[u] = b[u] = make_uint4(kFill, kFill, kFill, kFill);
                 }
@@ -796,17 +835,30 @@ constexpr int kVPT = (kMaxSlice + kNT - 1) / kNT;    // vectors per thread
 constexpr int kMinSlice = TURNOPD_CLUSTER_MIN_SLICE;
 constexpr int kSmallRowVec = 7168;  // up to this many vectors per row: 256-thread helpers, 2 per SM
 // The helper's rows per SM and second against the clusters', which decides the
-// split of the row list.  It depends on the clusters' slice length: 0.61 for
-// slices of 2048 vectors or more (V = 151,936 in clusters of 8, 262,144 in
-// clusters of 16), about 0.9 for 1563 (V = 100,000 / 200,000); linear between.
-double helper_rate(int slice_vec)
+// split of the row list.  A cluster SM is less efficient on a shorter slice and in a
+// larger cluster (more records per row), so the rate rises with both.  Measured best
+// (packed 8 x 4096, the ring-fed helper): clusters of 8, 0.72 at 2,374 vectors
+// (V = 151,936) and 0.85 at 2,004 (128,256); clusters of 16, 0.80 at 2,048 (262,144)
+// and about 1.0 at 1,563 (200,000); clusters of 3 to 6 (few helper SMs, where an
+// overloaded helper decides the call), 0.60: V = 50,000 (3) 0.946 ms against 1.042 at
+// 0.70, 90,000 (5) 1.623 against 1.709, 110,000 (6) 1.968 against 2.017, 65,536 (4)
+// flat from 0.65 to 0.75.  Sampled-token rows, whose helper gradient pass reads the
+// student only, 0.03 more (0.75 at 2,374).
+double helper_rate(int slice_vec, int cs, bool sampled)
 {
 #ifdef TURNOPD_HELPER_RATE
     (void)slice_vec;
+    (void)cs;
+    (void)sampled;
     return TURNOPD_HELPER_RATE;
 #else
-    const double r = 0.61 + (2048 - slice_vec) * 0.0006;
-    return r < 0.61 ? 0.61 : (r > 1.0 ? 1.0 : r);
+    double r = 0.60;
+    if (cs == 8)
+        r = 0.72 + (2374 - slice_vec) * 0.00035;
+    else if (cs > 8)
+        r = 0.80 + (2048 - slice_vec) * 0.00041;
+    r = r < 0.60 ? 0.60 : (r > 1.1 ? 1.1 : r);
+    return sampled ? r + 0.03 : r;
 #endif
 }
 // The helper grid beside the clusters: CTAs of kSideThreads threads, kSideBlocks per free SM.
@@ -878,7 +930,7 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
     if (free_sm > 0) {
         const double cl = (double)(grid_cache[dev][gi] * CS);
         pl.split_den = 1 << 20;
-        pl.split_num = (int32_t)(pl.split_den * cl / (cl + helper_rate(slice_vec) * free_sm) + 0.5);
+        pl.split_num = (int32_t)(pl.split_den * cl / (cl + helper_rate(slice_vec, CS, SM) * free_sm) + 0.5);
     }
     cfg.gridDim = dim3(grid_cache[dev][gi] * CS);
     e = cudaLaunchKernelEx(&cfg, kern, pl, slice_vec, nvec);
@@ -893,8 +945,13 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
     hc.numAttrs = 1;
     hc.gridDim = dim3(free_sm * kSideBlocks);
     hc.blockDim = dim3(kSideThreads);
+    hc.dynamicSmemBytes = helper_smem_bytes(true, kSideThreads);
     hc.stream = stream;
-    return cudaLaunchKernelEx(&hc, k_row_helper<G32, SM, TL, kSideThreads, kSideBlocks>, pl);
+    auto helper = k_row_helper<G32, SM, TL, true, kSideThreads, kSideBlocks>;
+    if ((e = cudaFuncSetAttribute(helper, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)helper_smem_bytes(true, kSideThreads))) != cudaSuccess)
+        return e;
+    return cudaLaunchKernelEx(&hc, helper, pl);
 }
 
 // Cluster sizes offered: 7 is left out (only 15 clusters of 7 are co-resident, 105 SMs).
@@ -918,9 +975,9 @@ void launch_helper_alone(const RowIn &p, int nvec, cudaStream_t stream)
 {
     const int sms = device_sm_count();
     if (nvec <= kSmallRowVec)
-        k_row_helper<G32, SM, TL, 256, 2><<<sms * 2, 256, 0, stream>>>(p);
+        k_row_helper<G32, SM, TL, false, 256, 2><<<sms * 2, 256, 0, stream>>>(p);
     else
-        k_row_helper<G32, SM, TL><<<sms, kHelpThreads, 0, stream>>>(p);
+        k_row_helper<G32, SM, TL, false><<<sms, kHelpThreads, 0, stream>>>(p);
 }
 
 // The row grids for bf16 logits; TL: V % 8 != 0 (a masked last vector).
