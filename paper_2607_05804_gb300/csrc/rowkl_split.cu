@@ -81,18 +81,20 @@ constexpr int kGStages = 7 - kSStages;          // chunks read again for the gra
 constexpr bool kKeep = TURNOPD_SPLIT_KEEP != 0;
 // The helper grid on the SMs the clusters leave free (k_split_helper): vectors per
 // model and thread in one batch, threads per CTA, and its rows per second per SM
-// against a cluster SM's, which sets the split of the row list (measured on the
-// packed 8 x 4096 fp32 batch: full vocabulary 6.66 / 6.56 / 6.45 / 6.68 / 7.04 ms at
-// 0.5 / 0.6 / 0.7 / 0.8 / 0.9; sampled 6.15 / 6.11 / 6.41 ms at 0.45 / 0.6 / 0.8;
-// batches of 8 vectors no faster than 4).
+// against a cluster SM's, which sets the split of the row list.  Measured on the packed
+// 8 x 4096 fp32 batch with the helper's statistics fed by its cp.async ring: full
+// vocabulary 6.45 / 6.35 / 6.27 / 6.28 / 6.59 ms at 0.7 / 0.8 / 0.9 / 1.0 / 1.1;
+// sampled 6.08 / 6.06 / 6.05 / 6.04 / 6.02 ms at 0.6 / 0.7 / 0.8 / 0.9 / 1.0 (with
+// register-fed batches the best had been 0.7 and 0.6: 6.41 and 6.07 ms).  Batches of 8
+// vectors were no faster than 4.
 #ifndef TURNOPD_SPLIT_HELPER
 #define TURNOPD_SPLIT_HELPER 1
 #endif
 #ifndef TURNOPD_SPLIT_RATE_FULL
-#define TURNOPD_SPLIT_RATE_FULL 0.7
+#define TURNOPD_SPLIT_RATE_FULL 0.9
 #endif
 #ifndef TURNOPD_SPLIT_RATE_SAMPLED
-#define TURNOPD_SPLIT_RATE_SAMPLED 0.6
+#define TURNOPD_SPLIT_RATE_SAMPLED 1.0
 #endif
 #ifndef TURNOPD_SPLIT_HELPER_U
 #define TURNOPD_SPLIT_HELPER_U 4
@@ -101,6 +103,8 @@ constexpr bool kKeep = TURNOPD_SPLIT_KEEP != 0;
 #define TURNOPD_SPLIT_HELPER_THREADS 512
 #endif
 constexpr bool kSplitHelper = TURNOPD_SPLIT_HELPER != 0;
+constexpr int kSplitHelpStages = 3;  // cp.async ring of the helper's statistics pass
+constexpr size_t split_helper_smem(int u, int nth) { return (size_t)kSplitHelpStages * 2 * u * nth * 16; }
 constexpr double kRateFull = TURNOPD_SPLIT_RATE_FULL;
 constexpr double kRateSampled = TURNOPD_SPLIT_RATE_SAMPLED;
 constexpr int kHelperU = TURNOPD_SPLIT_HELPER_U;
@@ -551,10 +555,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_row_split(RowIn p, int slice_ve
 // Helper for the SMs the clusters leave free, fp32 logits: one CTA per row at a time,
 // rows j0 + blockIdx.x, j0 + blockIdx.x + gridDim.x, ... of the row list (j0 = the
 // cluster grid's share).  The statistics pass streams both rows from HBM in batches of
-// U vectors per model and thread, with a running maximum per thread (one rescale per
-// batch when it moves) and A relative to the reference difference d at the running
-// student argmax, as the cluster kernel keeps it; the gradient pass reads the row
-// again from L2.  Launched as a dependent of the cluster grid (it starts once every
+// U vectors per model and thread, staged two batches ahead in a cp.async ring in shared
+// memory, with a running maximum per thread (one rescale per batch when it moves) and A
+// relative to the reference difference d at the running student argmax, as the cluster
+// kernel keeps it; the gradient pass reads the row again from L2.  Launched as a dependent of the cluster grid (it starts once every
 // cluster is resident) and completes only after it.
 template <bool G32, bool SM, int U, int NTH>
 __global__ void __launch_bounds__(NTH, 1) k_split_helper(RowIn p)
@@ -562,6 +566,7 @@ __global__ void __launch_bounds__(NTH, 1) k_split_helper(RowIn p)
     constexpr int NW = NTH / 32;
     __shared__ float red[NW][8];
     __shared__ float bc[8];
+    extern __shared__ float4 hring4[];  // [kSplitHelpStages][2][U][NTH]: the statistics pass's ring
     // the loss sum after this grid may take the first SM it frees (it waits for the grid)
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -580,14 +585,37 @@ __global__ void __launch_bounds__(NTH, 1) k_split_helper(RowIn p)
         const int yvec = SM ? (m.z >> 2) : -1;  // the vector holding the sampled id
         float ms = -INFINITY, mt = -INFINITY, dd = 0.f;
         float2 S2 = make_float2(0.f, 0.f), A2 = S2, T2 = S2;
-        for (int q0 = tid; q0 < nvec; q0 += U * NTH) {
+        // the statistics pass's batches land in a ring in shared memory by cp.async,
+        // kSplitHelpStages - 1 batches ahead; each thread copies and reads only its own slots
+        const int nbt = nvec > tid ? (nvec - tid + U * NTH - 1) / (U * NTH) : 0;
+        auto slot = [&](int s, int mdl, int u) { return ((s * 2 + mdl) * U + u) * NTH + tid; };
+        auto issue = [&](int bi) {  // batch bi into the ring (an empty group past the last)
+            if (bi < nbt) {
+                const int s = bi % kSplitHelpStages, q0 = tid + bi * U * NTH;
+#pragma unroll
+                for (int u = 0; u < U; ++u) {
+                    const int q = q0 + u * NTH;
+                    if (q < nvec) {
+                        cp_async16(&hring4[slot(s, 0, u)], vs + q);
+                        cp_async16(&hring4[slot(s, 1, u)], vt + q);
+                    }
+                }
+            }
+            cp_async_commit();
+        };
+        for (int bi = 0; bi < kSplitHelpStages - 1; ++bi)
+            issue(bi);
+        for (int bi = 0; bi < nbt; ++bi) {
+            const int q0 = tid + bi * U * NTH;
             float4 a[U], b[U];
+            issue(bi + kSplitHelpStages - 1);
+            cp_async_wait<kSplitHelpStages - 1>();  // batch bi has landed
 #pragma unroll
             for (int u = 0; u < U; ++u) {
                 const int q = q0 + u * NTH;
                 if (q < nvec) {
-                    a[u] = __ldg(vs + q);
-                    b[u] = __ldg(vt + q);
+                    a[u] = hring4[slot(bi % kSplitHelpStages, 0, u)];
+                    b[u] = hring4[slot(bi % kSplitHelpStages, 1, u)];
                 } else {
                     a[u] = b[u] = kFill4;  // adds 0, never the maximum
                 }
@@ -785,9 +813,13 @@ cudaError_t launch_split_t(const RowIn &p, bool fp32_grad, int nvec, double rate
     hc.numAttrs = 1;
     hc.gridDim = dim3(free_sm);
     hc.blockDim = dim3(kHelperThreads);
+    hc.dynamicSmemBytes = split_helper_smem(kHelperU, kHelperThreads);
     hc.stream = stream;
     auto helper = fp32_grad ? k_split_helper<true, SM, kHelperU, kHelperThreads>
                             : k_split_helper<false, SM, kHelperU, kHelperThreads>;
+    if ((e = cudaFuncSetAttribute(helper, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                  (int)split_helper_smem(kHelperU, kHelperThreads))) != cudaSuccess)
+        return e;
     return cudaLaunchKernelEx(&hc, helper, pl);
 }
 
