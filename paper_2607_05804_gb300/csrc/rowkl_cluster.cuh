@@ -25,8 +25,8 @@
 // registers for the maxima and sums, once for the gradient (3 exponentials
 // per element in all).
 // Clusters of 8 fill 120 of the 152 SMs; a helper grid of one 512-thread CTA per
-// free SM takes the last share of the rows, each row read from HBM once and again
-// from L2 (k_row_helper below).
+// free SM takes the last share of the rows, each row read from HBM once (staged
+// through a cp.async ring) and again from L2 (k_row_helper below).
 // Waits are bounded: on timeout the kernel records TURNOPD_ERR_TIMEOUT, stops
 // computing and runs its remaining barriers without waiting, so it terminates.
 
@@ -528,8 +528,9 @@ __global__ void __launch_bounds__(G * NT, 1) k_row_cluster(RowIn p, int slice_ve
 // Helper for the SMs the clusters leave free (15 eight-CTA clusters cover 120 of
 // 152): one CTA per row at a time, rows j0 + blockIdx.x, j0 + blockIdx.x +
 // gridDim.x, ... of the row list, j0 = the cluster kernel's share.  The
-// statistics pass streams both rows from HBM with a running maximum per thread
-// (one rescale per batch of kHelpU vectors when the maximum moves); the gradient
+// statistics pass streams both rows from HBM (beside the clusters through a cp.async
+// ring, AS) with a running maximum per thread (one rescale per batch of kHelpU
+// vectors when the maximum moves); the gradient
 // pass reads them again from L2, where the pass before left them (the clusters'
 // own copies are evict-first).  bf16 logits; a bf16 or fp32 gradient or none.
 // Like the cluster kernel, the fp32 gradient also keeps A relative to the
