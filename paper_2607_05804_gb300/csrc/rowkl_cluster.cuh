@@ -844,13 +844,16 @@ constexpr int kSmallRowVec = 7168;  // up to this many vectors per row: 256-thre
 // overloaded helper decides the call), 0.60: V = 50,000 (3) 0.946 ms against 1.042 at
 // 0.70, 90,000 (5) 1.623 against 1.709, 110,000 (6) 1.968 against 2.017, 65,536 (4)
 // flat from 0.65 to 0.75.  Sampled-token rows, whose helper gradient pass reads the
-// student only, 0.03 more (0.75 at 2,374).
-double helper_rate(int slice_vec, int cs, bool sampled)
+// student only, more: 0.03 with a bf16 gradient (0.75 at 2,374), 0.10 with an fp32 one
+// (0.82 at 2,374: 4.196 ms against 4.260 at 0.75 and 4.539 at 0.92), whose larger
+// gradient writes weigh more beside the skipped teacher read.
+double helper_rate(int slice_vec, int cs, bool sampled, bool g32)
 {
 #ifdef TURNOPD_HELPER_RATE
     (void)slice_vec;
     (void)cs;
     (void)sampled;
+    (void)g32;
     return TURNOPD_HELPER_RATE;
 #else
     double r = 0.60;
@@ -859,7 +862,7 @@ double helper_rate(int slice_vec, int cs, bool sampled)
     else if (cs > 8)
         r = 0.80 + (2048 - slice_vec) * 0.00041;
     r = r < 0.60 ? 0.60 : (r > 1.1 ? 1.1 : r);
-    return sampled ? r + 0.03 : r;
+    return sampled ? r + (g32 ? 0.10 : 0.03) : r;
 #endif
 }
 // The helper grid beside the clusters: CTAs of kSideThreads threads, kSideBlocks per free SM.
@@ -931,7 +934,7 @@ cudaError_t launch_t(const RowIn &p, int slice_vec, int nvec, size_t smem, cudaS
     if (free_sm > 0) {
         const double cl = (double)(grid_cache[dev][gi] * CS);
         pl.split_den = 1 << 20;
-        pl.split_num = (int32_t)(pl.split_den * cl / (cl + helper_rate(slice_vec, CS, SM) * free_sm) + 0.5);
+        pl.split_num = (int32_t)(pl.split_den * cl / (cl + helper_rate(slice_vec, CS, SM, G32) * free_sm) + 0.5);
     }
     cfg.gridDim = dim3(grid_cache[dev][gi] * CS);
     e = cudaLaunchKernelEx(&cfg, kern, pl, slice_vec, nvec);
