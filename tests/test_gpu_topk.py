@@ -164,11 +164,13 @@ def test_dense_gradient_misaligned_stride_and_zero_flag(P, oracle, dtype):
         assert np.array_equal(dn[rot_np[t], :V], want)
 
 
-def test_full_vocab_packed_sampled_rows_and_properties(P, oracle):
-    """The bench workload (packed 8 x 4096, 19,669 rows of V = 151,936 bf16, compact):
-    the oracle recomputes a few rows; every row is checked by the selection's
-    defining properties."""
-    b = W.packed(seed=0)
+@pytest.mark.parametrize("workload", ["packed", "household", "multihop"])
+def test_full_vocab_sampled_rows_and_properties(P, oracle, workload):
+    """The bench workloads at full size (packed 8 x 4096: 19,669 rows; household
+    16 x 8192: 10,918; multihop, 64 ragged trajectories: 8,020; V = 151,936 bf16,
+    compact rows): the oracle recomputes a few rows; every row is checked by the
+    selection's defining properties."""
+    b = W.CONFIGS[workload](seed=0)
     V, K = W.V_QWEN, 50
     R = b.num_valid
     zs, zt = W.make_logits(R, V, "agent", torch.bfloat16, seed=1000, device="cuda")
