@@ -187,6 +187,72 @@ def test_vocab_shard_host_validation(lib):
     assert call(ws=ctypes.c_void_p(0x10010)) == 10    # not 256-byte aligned
 
 
+def test_vocab_merge_and_shard_grad_host_validation(lib):
+    merge = lib.turnopd_vocab_stats_merge
+    assert merge(None, 2, FAKE, 64, FAKE, None) == 1
+    assert merge(FAKE, 2, FAKE, 64, None, None) == 1
+    assert merge(FAKE, 0, FAKE, 64, FAKE, None) == 2                    # no shard
+    assert merge(FAKE, 2, FAKE, -1, FAKE, None) == 2
+    assert merge(ctypes.c_void_p(0x10002), 2, FAKE, 64, FAKE, None) == 2  # misaligned float32 partials
+    assert merge(None, 2, None, 0, None, None) == 0                     # nothing to merge, no launch
+
+    f = lib.turnopd_vocab_shard_loss_grad
+    ws_need = lib.turnopd_loss_workspace_bytes(64)
+
+    def call(zs=FAKE, ld=1024, vocab=1024, rows=64, T=64, in_dtype=1, stats=FAKE, grad=FAKE, grad_dtype=1,
+             flags=0, tl=FAKE, loss=FAKE, ws=FAKE, wsb=None, status=FAKE):
+        return f(zs, FAKE, in_dtype, ld, vocab, rows, None, FAKE, FAKE, T, stats, grad, grad_dtype, flags, tl,
+                 loss, ws, ws_need if wsb is None else wsb, status, None)
+
+    assert call(zs=None) == 1
+    assert call(status=None) == 1
+    assert call(loss=None) == 1
+    assert call(stats=None) == 1
+    assert call(tl=None) == 1
+    assert call(in_dtype=3) == 6
+    assert call(grad_dtype=2) == 6
+    assert call(flags=0x2) == 6
+    assert call(ld=512) == 2                                            # ld < shard width
+    assert call(grad=ctypes.c_void_p(0x10001)) == 2                     # misaligned bf16 gradient
+    assert call(loss=ctypes.c_void_p(0x10004)) == 2                     # misaligned fp64 loss
+    assert call(ws=None) == 10
+    assert call(wsb=ws_need - 1) == 10
+
+
+def test_fused_host_validation(lib):
+    """Checks that answer before the workspace size is computed (which asks the
+    device for its SM count)."""
+    f = lib.turnopd_fused_lmhead_fwd_bwd
+
+    def call(hs=FAKE, Ws=FAKE, d_s=1024, ht=FAKE, Wt=FAKE, d_t=512, vocab=8192, T=64, mode=0, dh=FAKE, dW=None,
+             tl=FAKE, loss=FAKE, ws=None, status=FAKE):
+        return f(hs, Ws, d_s, ht, Wt, d_t, vocab, FAKE, FAKE, T, mode, dh, dW, tl, loss, ws, 1 << 30, status, None)
+
+    assert call(Ws=None) == 1
+    assert call(Wt=None) == 1
+    assert call(loss=None) == 1
+    assert call(status=None) == 1
+    assert call(hs=None) == 1
+    assert call(tl=None) == 1
+    assert call(mode=1) == 6                                            # sampled mode is not fused
+    assert call(d_s=1000) == 2                                          # d_s a multiple of 256
+    assert call(d_s=128) == 2
+    assert call(d_t=100) == 2                                           # d_t a multiple of 64
+    assert call(d_s=65536 + 256) == 2
+    assert call(vocab=0) == 2
+    assert call(T=-1) == 2
+    assert call(hs=ctypes.c_void_p(0x10008)) == 2                       # TMA operands 16-byte aligned
+    assert call(dW=ctypes.c_void_p(0x10004)) == 2
+    assert call() == 10                                                 # no workspace
+
+
+def test_static_entry_rejects_oversize_batches(lib):
+    f = lib.turnopd_loss_fwd_bwd_static
+    T = 65536 + 1                                                       # TURNOPD_STATIC_MAX_TOKENS + 1
+    assert f(FAKE, FAKE, 1, 1024, 1024, T, None, None, FAKE, FAKE, T, 0, None, 0, 0, FAKE, FAKE, FAKE,
+             None) == 10
+
+
 def test_selftest_wait_timeout_host_validation(lib):
     f = lib.turnopd_selftest_wait_timeout
     assert f(100, None, None) == 1                # TURNOPD_ERR_NULL
