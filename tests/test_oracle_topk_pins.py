@@ -76,6 +76,21 @@ def test_ties_take_the_lower_id():
     assert oracle.topk_row(np.zeros(4, np.uint16), z, 3)[1].tolist() == [3, 0, 1]
 
 
+@pytest.mark.parametrize("seed", range(6))
+def test_selection_equals_a_sort_by_logit_then_id(seed):
+    """The support against Python's own sort on (-logit, id), on rows drawn from a
+    handful of values (many ties, +0 and -0 among them), for several K."""
+    r = rng(100 + seed)
+    V = int(r.integers(5, 300))
+    levels = np.array([-3.5, -1.0, -0.0, 0.0, 0.25, 2.0, 7.0], np.float32)
+    zt = levels[r.integers(0, levels.size, V)]
+    zs = r.normal(0, 1, V).astype(np.float32)
+    want_all = sorted(range(V), key=lambda v: (-float(zt[v]), v))   # -0.0 == 0.0 as Python floats
+    for K in sorted({1, 2, V // 3 + 1, V // 2 + 1, V}):
+        ids = oracle.topk_row(zs, zt, K)[1]
+        assert ids.tolist() == want_all[:K], (V, K)
+
+
 def test_off_support_logits_do_not_matter():
     r = rng(2)
     V, K = 500, 20
